@@ -1,0 +1,415 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: published
+known-answer vectors, a product-form brute force of Eq. 1, a library special
+case, the KL-decomposition lemma (App. B), the lossless theorem (App. B.3) by
+exact enumeration and by Monte Carlo, Algorithm 1 on chains, and tree paths
+whose outcome is fixed by construction.
+"""
+
+import itertools
+import os
+
+import numpy as np
+import pytest
+from scipy import special, stats
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rows(rng, V, scale=2.0):
+    zp = scale * rng.standard_normal(V)
+    zq = 0.7 * zp + 1.5 * rng.standard_normal(V)
+    return zp, zq
+
+
+# ----------------------------------------------------------------------------- Philox
+
+def test_philox_known_answers():
+    """Random123 kat_vectors for Philox4x32-10 (Salmon et al., SC'11)."""
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "philox4x32_10_kat.txt")) if l.strip() and l[0] != "#"]
+    assert len(rows) == 3
+    for r in rows:
+        v = [int(x, 16) for x in r]
+        out = oracle.philox(v[0:4], v[4:6])
+        assert [int(x) for x in out] == v[6:10]
+
+
+def test_uniform_conversion_open_interval_and_fp32_exact():
+    for w in (0, 1, 511, 512, 0x7FFFFFFF, 0xFFFFFFFF, 0x12345678):
+        u = oracle.u01(w)
+        assert 0.0 < u < 1.0
+        assert float(np.float32(u)) == u  # fp32 holds every value exactly
+    assert oracle.u01(0) == 0.5 * 2.0 ** -23
+    assert oracle.u01(0xFFFFFFFF) == 1.0 - 0.5 * 2.0 ** -23
+
+
+def test_uniform_streams_are_uniform_and_distinct():
+    accept = np.array([oracle.accept_uniform(7, 3, g) for g in range(20000)])
+    race = np.array([oracle.race_uniform(7, 3, 11, x) for x in range(20000)])
+    for u in (accept, race):
+        assert stats.kstest(u, "uniform").pvalue > 1e-4
+    assert abs(np.corrcoef(accept, race)[0, 1]) < 0.05
+    # another offset gives another stream
+    other = np.array([oracle.accept_uniform(7, 4, g) for g in range(2000)])
+    assert np.mean(other == accept[:2000]) < 0.01
+
+
+# ----------------------------------------------------------------------------- Eq. 1 target
+
+@pytest.mark.parametrize("V", [7, 64, 1000])
+def test_alpha_zero_is_expert_log_softmax(V):
+    """alpha = 0: CD reduces to the expert distribution (Sec. 3.3, alpha = 0 boundary)."""
+    rng = np.random.default_rng(V)
+    zp, zq = _rows(rng, V)
+    r = oracle.row_logpi(zp, zq, alpha=0.0, beta=0.0, T=1.0)
+    np.testing.assert_allclose(r["logpi"], special.log_softmax(zp), rtol=0, atol=1e-12)
+    assert r["argmax"] == int(np.argmax(zp))
+
+
+@pytest.mark.parametrize("alpha,beta,T", [(0.1, 0.0, 1.0), (0.5, 0.0, 1.0), (1.0, 0.0, 0.7),
+                                          (0.2, 0.1, 1.0), (0.05, 0.5, 1.3), (0.3, 1e-3, 0.5)])
+def test_product_form_brute_force(alpha, beta, T):
+    """pi_CD = pi_p^(1+a) pi_q^(-a) / Z (Eq. 1), masked to P_beta (Sec. 2.1), evaluated as products."""
+    rng = np.random.default_rng(int(alpha * 100 + beta * 1000 + T * 10))
+    for V in (5, 17, 64):
+        zp, zq = _rows(rng, V, scale=1.0)
+        p = np.exp(zp) / np.exp(zp).sum()
+        qa = np.exp(zq) / np.exp(zq).sum()
+        w = (p ** (1.0 + alpha) * qa ** (-alpha)) ** (1.0 / T)
+        w = np.where(p >= beta * p.max(), w, 0.0)
+        pi = w / w.sum()
+        r = oracle.row_logpi(zp, zq, alpha=alpha, beta=beta, T=T)
+        np.testing.assert_allclose(np.exp(r["logpi"]), pi, rtol=1e-11, atol=1e-15)
+        assert r["argmax"] == int(np.argmax(np.where(w > 0, np.log(p ** (1 + alpha) * qa ** (-alpha)), -np.inf)))
+
+
+def test_kl_decomposition_lemma():
+    """App. B, Lemma kl_decomposition, at beta = 0 and T = 1."""
+    rng = np.random.default_rng(5)
+    for V, alpha in [(50, 0.1), (500, 0.5), (3000, 1.0), (200, 0.0)]:
+        zp, zq = _rows(rng, V)
+        lp, lq = special.log_softmax(zp), special.log_softmax(zq)
+        p, qa = np.exp(lp), np.exp(lq)
+        r = oracle.row_logpi(zp, zq, alpha=alpha, beta=0.0, T=1.0)
+        lpi = r["logpi"]
+        logZ = r["log_zcd"]
+        kl = lambda a, la, lb: float(np.sum(a * (la - lb)))  # noqa: E731
+        assert abs(kl(p, lp, lpi) - (logZ - alpha * kl(p, lp, lq))) < 1e-10
+        assert abs(kl(qa, lq, lpi) - (logZ + (1 + alpha) * kl(qa, lq, lp))) < 1e-10
+        # Z_CD = sum pi_p^(1+a) pi_q^(-a) (App. B.3)
+        assert abs(logZ - np.log(np.sum(p ** (1 + alpha) * qa ** (-alpha)))) < 1e-10
+        # the raw-logit normaliser differs from log Z_CD by (1+a) lse_p - a lse_q
+        assert abs(r["cd_lse"] - (logZ + (1 + alpha) * r["lse_p"] - alpha * r["lse_q"])) < 1e-9
+
+
+def test_plausibility_mask_invariants():
+    """P_beta (Sec. 2.1): nested in beta, always holds argmax pi_p, pi_CD = 0 outside (App. B.3 remark)."""
+    rng = np.random.default_rng(9)
+    V = 400
+    zp, zq = _rows(rng, V)
+    p = special.softmax(zp)
+    prev = None
+    for alpha in (0.0, 0.05, 0.1, 0.2, 0.5, 1.0):
+        prev = None
+        for beta in (0.0, 1e-3, 0.1, 0.5, 1.0):
+            r = oracle.row_logpi(zp, zq, alpha=alpha, beta=beta, T=1.0)
+            inside = np.isfinite(r["logpi"])
+            assert inside.sum() == int(np.sum(p >= beta * p.max()))
+            assert inside[np.argmax(zp)]
+            assert inside[r["argmax"]]
+            assert abs(np.exp(r["logpi"][inside]).sum() - 1.0) < 1e-12
+            if prev is not None:
+                assert not np.any(inside & ~prev)  # nested: growing beta only removes tokens
+            prev = inside
+            if beta == 1.0:
+                assert r["argmax"] == int(np.argmax(zp))
+                assert inside.sum() == 1
+
+
+# ----------------------------------------------------------------------------- lossless theorem
+
+def _dyadic_distribution(p, zero_last=False, bits=12):
+    """A float32 distribution with entries k / 2^bits summing to exactly one."""
+    p = np.array(p, dtype=np.float64)
+    if zero_last:
+        p[-1] = 0.0
+    k = np.floor(p / p.sum() * 2 ** bits)
+    k[np.argmax(k)] += 2 ** bits - k.sum()
+    return (k / 2 ** bits).astype(np.float32)
+
+
+def _emission_from_chain(zp, zq, alpha, beta, T, q, tokens):
+    ratios, rm = oracle.row_chain(zp, zq, alpha, beta, T, q, tokens)
+    V = len(zp)
+    emit = np.zeros(V)
+    reach = 1.0
+    for t, rho in zip(tokens, ratios):
+        a = min(1.0, rho)
+        emit[t] += reach * a
+        reach *= 1.0 - a
+    emit += reach * rm
+    return emit
+
+
+@pytest.mark.parametrize("m", [1, 2, 3])
+@pytest.mark.parametrize("alpha,beta,T", [(0.1, 0.0, 1.0), (0.5, 0.2, 1.0), (1.0, 0.0, 0.6)])
+def test_lossless_exact_enumeration(m, alpha, beta, T):
+    """App. B.3: with m siblings drawn i.i.d. from q, the first emitted token is distributed as pi_CD.
+
+    Every sibling tuple is enumerated and the acceptance uniforms are integrated analytically
+    (accept with probability min(1, ratio)); only the oracle's ratios and residuals are used.
+    """
+    rng = np.random.default_rng(m * 31 + int(alpha * 10))
+    V = 5
+    zp, zq = _rows(rng, V, scale=1.0)
+    qd = _dyadic_distribution(special.softmax(zp + rng.standard_normal(V)), zero_last=True)
+    q64 = qd.astype(np.float64)
+    assert q64.sum() == 1.0
+    total = np.zeros(V)
+    for tup in itertools.product(range(V), repeat=m):
+        w = np.prod([q64[t] for t in tup])
+        if w == 0.0:
+            continue
+        total += w * _emission_from_chain(zp, zq, alpha, beta, T, qd, list(tup))
+    total /= np.prod([q64.sum()] * m)
+    pi = np.exp(oracle.row_logpi(zp, zq, alpha, beta, T)["logpi"])
+    np.testing.assert_allclose(total, pi, rtol=0, atol=1e-12)
+
+
+def _first_emitted(res, tokens):
+    B = len(res["accept_len"])
+    out = np.where(res["accept_len"] > 0, tokens[np.arange(B), res["accept_path"][:, 1].clip(0)], res["bonus"])
+    return out
+
+
+@pytest.mark.parametrize("beta", [0.0, 0.15])
+def test_lossless_monte_carlo_full_verify(beta):
+    """Full sampled verification (Philox, ratio test, residuals, exponential race) emits pi_CD."""
+    rng = np.random.default_rng(123)
+    V, B, m = 6, 120000, 3
+    zp, zq = _rows(rng, V, scale=1.0)
+    alpha, T = 0.3, 1.0
+    qd = special.softmax(zp + 0.8 * rng.standard_normal(V)).astype(np.float32)
+    qd = (qd / qd.sum(dtype=np.float64)).astype(np.float32)
+    N = 1 + m
+    parents = np.tile(np.array([-1, 0, 0, 0], dtype=np.int32), (B, 1))
+    tokens = np.zeros((B, N), dtype=np.int32)
+    tokens[:, 1:] = rng.choice(V, size=(B, m), p=qd.astype(np.float64) / qd.sum(dtype=np.float64))
+    res = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, ld=0, tokens=tokens,
+                        parents=parents, alpha=np.full(B, alpha), beta=np.full(B, beta),
+                        temperature=np.full(B, T), q=qd, ldq=0, seed=99, offset=5, nthreads=4)
+    first = _first_emitted(res, tokens)
+    counts = np.bincount(first, minlength=V)
+    pi = np.exp(oracle.row_logpi(zp, zq, alpha, beta, T)["logpi"])
+    tv = 0.5 * np.abs(counts / B - pi).sum()
+    assert tv < 3.0 * np.sqrt(V / B)
+    nz = pi > 0
+    assert counts[~nz].sum() == 0  # never emits outside the plausibility set
+    chi = stats.chisquare(counts[nz], B * pi[nz])
+    assert chi.pvalue > 1e-4
+
+
+def test_exponential_race_samples_target():
+    """A leaf row's bonus is drawn from pi_CD by the race (Algorithm 1, final sample)."""
+    rng = np.random.default_rng(77)
+    V, B = 8, 100000
+    zp, zq = _rows(rng, V, scale=1.0)
+    res = oracle.verify(B=B, N=1, V=V, dtype="f64", z_exp=zp, z_ama=zq, ld=0,
+                        tokens=np.zeros((B, 1), np.int32), parents=np.full((B, 1), -1, np.int32),
+                        alpha=np.full(B, 0.2), temperature=np.full(B, 0.8), q=np.zeros(V, np.float32), ldq=0,
+                        seed=1, offset=0, nthreads=4)
+    pi = np.exp(oracle.row_logpi(zp, zq, 0.2, 0.0, 0.8)["logpi"])
+    counts = np.bincount(res["bonus"], minlength=V)
+    assert stats.chisquare(counts, B * pi).pvalue > 1e-4
+    assert np.all(res["accept_len"] == 0)
+
+
+# ----------------------------------------------------------------------------- Algorithm 1 on chains
+
+def _algorithm1_chain(zp_rows, zq_rows, q_rows, drafts, alpha, T, seed, offset, b, N):
+    """Algorithm 1 (one DCD round) for a chain of gamma drafts, from the pinned row target."""
+    gamma = len(drafts)
+    V = zp_rows.shape[1]
+    pis = [np.exp(oracle.row_logpi(zp_rows[i], zq_rows[i], alpha, 0.0, T)["logpi"]) for i in range(gamma + 1)]
+    k = gamma + 1
+    for i in range(1, gamma + 1):
+        r_i = oracle.accept_uniform(seed, offset, b * N + i)
+        # row i-1 holds the logits after draft i-1, i.e. the distribution of draft i
+        pi_i, q_i = pis[i - 1], q_rows[i - 1].astype(np.float64)
+        ratio = pi_i[drafts[i - 1]] / q_i[drafts[i - 1]] if q_i[drafts[i - 1]] > 0 else np.inf
+        if r_i > ratio:
+            k = i
+            break
+    if k <= gamma:
+        P = np.maximum(0.0, pis[k - 1] - q_rows[k - 1].astype(np.float64))
+        P = P / P.sum()
+        row = k - 1
+    else:
+        P = pis[gamma]
+        row = gamma
+    keys = [np.log(P[x]) - np.log(-np.log(oracle.race_uniform(seed, offset, b * N + row, x))) if P[x] > 0 else -np.inf
+            for x in range(V)]
+    return k - 1, int(np.argmax(keys))
+
+
+def test_chain_reduces_to_algorithm1():
+    rng = np.random.default_rng(2024)
+    V, gamma, B = 12, 5, 300
+    N = gamma + 1
+    alpha, T = 0.4, 1.0
+    zp = rng.standard_normal((B * N, V))
+    zq = 0.7 * zp + 0.8 * rng.standard_normal((B * N, V))
+    q = special.softmax(zp + 0.5 * rng.standard_normal((B * N, V)), axis=1).astype(np.float32)
+    tokens = np.zeros((B, N), dtype=np.int32)
+    for b in range(B):
+        for i in range(1, N):
+            qq = q[b * N + i - 1].astype(np.float64)
+            tokens[b, i] = rng.choice(V, p=qq / qq.sum())
+    parents = np.tile(np.arange(-1, N - 1, dtype=np.int32), (B, 1))
+    res = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=tokens, parents=parents,
+                        alpha=np.full(B, alpha), temperature=np.full(B, T), q=q, seed=3, offset=8)
+    for b in range(B):
+        acc, y = _algorithm1_chain(zp[b * N:(b + 1) * N], zq[b * N:(b + 1) * N], q[b * N:(b + 1) * N],
+                                   tokens[b, 1:], alpha, T, 3, 8, b, N)
+        assert res["accept_len"][b] == acc
+        assert res["bonus"][b] == y
+        assert list(res["accept_path"][b, :acc + 1]) == list(range(acc + 1))
+
+
+# ----------------------------------------------------------------------------- greedy walk
+
+def _spiked_rows(rng, R, V, winners, alpha):
+    """Rows whose CD argmax is `winners[g]` by construction: a +30 spike dominates every score."""
+    zp = rng.standard_normal((R, V))
+    zp[np.arange(R), winners] += 30.0
+    zq = 0.7 * zp + 0.5 * rng.standard_normal((R, V))
+    return zp, zq
+
+
+def test_greedy_paths_fixed_by_construction():
+    rng = np.random.default_rng(11)
+    V, B = 50, 40
+    from paper_2608_12913_gb300 import workloads
+    for b_trial in range(3):
+        parents = np.stack([workloads.tree_parents(np.random.default_rng(100 * b_trial + b)) for b in range(B)])
+        N = parents.shape[1]
+        winners = rng.integers(0, V, size=B * N)
+        zp, zq = _spiked_rows(rng, B * N, V, winners, 0.1)
+        tokens = rng.integers(0, V, size=(B, N)).astype(np.int32)
+        expect_len, expect_bonus, expect_path = [], [], []
+        for b in range(B):
+            kids = workloads.children_lists(parents[b])
+            cur, path = 0, [0]
+            # choose a target path: descend through a random child while there is one
+            while kids[cur] and rng.random() < 0.85:
+                c = kids[cur][rng.integers(len(kids[cur]))]
+                path.append(c)
+                cur = c
+            # tokens: the path's children carry their parent's winner, every other sibling
+            # (and the path's last node's children) carry something else
+            for n in range(N):
+                for c in kids[n]:
+                    w = winners[b * N + n]
+                    if n in path[:-1] and c == path[path.index(n) + 1]:
+                        tokens[b, c] = w
+                    elif tokens[b, c] == w:
+                        tokens[b, c] = (w + 1) % V
+            expect_len.append(len(path) - 1)
+            expect_bonus.append(winners[b * N + cur])
+            expect_path.append(path)
+        res = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=tokens, parents=parents,
+                            alpha=np.full(B, 0.1))
+        assert list(res["accept_len"]) == expect_len
+        assert list(res["bonus"]) == expect_bonus
+        for b in range(B):
+            p = expect_path[b]
+            assert list(res["accept_path"][b, :len(p)]) == p
+            assert np.all(res["accept_path"][b, len(p):] == -1)
+
+
+def test_greedy_duplicate_siblings_take_lowest_node():
+    rng = np.random.default_rng(3)
+    V = 20
+    parents = np.array([[-1, 0, 0, 0, 2, 3]], dtype=np.int32)
+    winners = np.array([7, 1, 2, 3, 4, 5])
+    zp, zq = _spiked_rows(rng, 6, V, winners, 0.1)
+    tokens = np.array([[0, 9, 7, 7, 2, 3]], dtype=np.int32)
+    res = oracle.verify(B=1, N=6, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=tokens, parents=parents,
+                        alpha=np.full(1, 0.1))
+    # nodes 2 and 3 both carry the root's winner 7: node 2 is taken; its child 4 carries
+    # row 2's winner 2, so the path is 0 -> 2 -> 4 and the bonus is row 4's winner
+    assert res["accept_len"][0] == 2
+    assert list(res["accept_path"][0]) == [0, 2, 4, -1, -1, -1]
+    assert res["bonus"][0] == 4
+
+
+def test_full_acceptance_chain():
+    rng = np.random.default_rng(8)
+    V, N = 30, 9
+    winners = rng.integers(0, V, size=N)
+    zp, zq = _spiked_rows(rng, N, V, winners, 0.2)
+    tokens = np.concatenate([[0], winners[:-1]]).astype(np.int32)[None, :]
+    res = oracle.verify(B=1, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=tokens,
+                        parents=np.arange(-1, N - 1, dtype=np.int32)[None, :], alpha=np.full(1, 0.2))
+    assert res["accept_len"][0] == N - 1
+    assert res["bonus"][0] == winners[-1]
+
+
+def test_sampled_rule_tends_to_greedy_as_T_vanishes():
+    """T -> 0 with a uniform drafter: the sampled rule accepts exactly the greedy matches."""
+    from paper_2608_12913_gb300 import workloads
+    w = workloads.make_config(1, V=300, B=4, seed=21, margin_fn=oracle.margin_fn)
+    B, N, V = w.B, w.N, w.V
+    zp = w.z_exp.float().double().numpy()
+    zq = w.z_ama.float().double().numpy()
+    g = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=w.tokens, parents=w.parents,
+                      alpha=w.alpha)
+    # make the drafts hit the argmax often: every first child takes its parent's argmax
+    tokens = w.tokens.numpy().copy()
+    rows = g["rows"]
+    for b in range(B):
+        kids = workloads.children_lists(w.parents[b].numpy())
+        for n in range(N):
+            if kids[n]:
+                tokens[b, kids[n][-1]] = rows[b, n]["argmax"]
+    g = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=tokens, parents=w.parents,
+                      alpha=w.alpha)
+    qu = np.full((B * N, V), 1.0 / V, dtype=np.float32)
+    s = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, tokens=tokens, parents=w.parents,
+                      alpha=w.alpha, temperature=np.full(B, 1e-6, np.float32), q=qu, seed=4, offset=1)
+    assert np.array_equal(g["accept_len"], s["accept_len"])
+    assert np.array_equal(g["accept_path"], s["accept_path"])
+    assert np.array_equal(g["bonus"], s["bonus"])
+    assert g["accept_len"].max() >= 1
+
+
+def test_residual_output_matches_chain():
+    """The residual a sequence's bonus was drawn from equals the row chain's final residual."""
+    from paper_2608_12913_gb300 import workloads
+    w = workloads.make_config(2, V=200, B=6, seed=5)
+    res = oracle.verify_workload(w, want_residual=True)
+    zp = w.z_exp.float().double().numpy()
+    zq = w.z_ama.float().double().numpy()
+    for b in range(w.B):
+        cur = res["accept_path"][b, res["accept_len"][b]]
+        kids = workloads.children_lists(w.parents[b].numpy())[cur]
+        g = b * w.N + cur
+        _, rm = oracle.row_chain(zp[g], zq[g], float(w.alpha[b]), 0.0, float(w.temperature[b]), w.q[g].numpy(),
+                                 [int(w.tokens[b, c]) for c in kids])
+        np.testing.assert_allclose(res["residual"][b], rm, atol=1e-15)
+        assert rm[res["bonus"][b]] > 0
+
+
+def test_invalid_trees_rejected():
+    V = 10
+    z = np.zeros((3, V))
+    base = dict(B=1, N=3, V=V, dtype="f64", z_exp=z, z_ama=z, alpha=np.zeros(1))
+    with pytest.raises(ValueError):
+        oracle.verify(tokens=np.zeros((1, 3), np.int32), parents=np.array([[-1, 0, 2]], np.int32), **base)
+    with pytest.raises(ValueError):
+        oracle.verify(tokens=np.array([[0, 0, V]], np.int32), parents=np.array([[-1, 0, 1]], np.int32), **base)
+    with pytest.raises(ValueError):
+        oracle.verify(tokens=np.zeros((1, 3), np.int32), parents=np.array([[0, 0, 1]], np.int32), **base)
