@@ -1,0 +1,343 @@
+"""Benchmark of the CD verification step on GB300.
+
+One step = one pass of the whole hot path over one batch: the per-row kernel
+(Eq. 1 target, reductions, greedy/sampled acceptance, terminal draws) and the tree
+walk, through the C ABI (dcd_score_rows + dcd_tree_walk, i.e. dcd_verify_sample
+without the test-only residual output), on the batched-serving workload:
+32 sequences x 60-node trees of depth 7 (1920 rows), V = 128256, bf16 logits,
+alpha in {0.05, 0.1, 0.2}, even sequences greedy and odd ones sampled at T = 1.
+Inputs are seeded synthetic data resident in HBM (1.48 GB per step, larger than
+the 126 MB L2, so no flush is needed); each step advances the Philox offset.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle on a
+bounded sample of the same workload instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "batched_B32_tree60_V128256_bf16_mixed"
+METRIC = "verified draft nodes/sec (CD verification step, 1 GPU)"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in ("dcd_rows.cu", "dcd_internal.h"):
+        with open(os.path.join(ROOT, "paper_2608_12913_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def _profiled_traffic(kernel_hash: str):
+    """DRAM bytes per launch of the row kernel from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "score_rows_kernel_batched_B32_tree60_V128256.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    m_bytes = re.search(r"dram_bytes_per_launch:\s*([0-9.e+]+)", text)
+    if not m_hash or not m_bytes or m_hash.group(1) != kernel_hash:
+        return None
+    return float(m_bytes.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampler (50 ms period) around the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.samples = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+
+    def summary(self, t0: float, t1: float):
+        win = [s for t, s in self.samples if t0 - 1.0 <= t <= t1 + 0.1]
+        if not win:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]}
+        sm = [float(s[0]) for s in win if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in win if s[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in win for i in range(4) if len(s) > 4 + i and "Active" in s[4 + i]
+                          and "Not" not in s[4 + i]})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(win), "window": "from 1 s before the timed region to its end"}
+
+
+def algorithmic_bytes(w) -> int:
+    """Bytes the path must move per step: both logit rows of every node (bf16), q for the
+    non-leaf rows of sampled sequences (fp32), the tree, parameters and outputs."""
+    es = 2 if w.dtype == "bf16" else 4
+    logits = 2 * w.R * w.V * es
+    qb = w.sampled_rows_with_children() * w.V * 4
+    small = w.R * (4 + 4) + w.B * 12 + w.R * 12 + w.B * (8 + w.N * 4)
+    return logits + qb + small
+
+
+def _dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args):
+    """The fp64 CPU oracle timed as the reference arm (rank 0 only)."""
+    ws, rank, _ = _dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2608_12913_gb300 import workloads
+    w = workloads.make_config(3, B=2)  # sequences 0 (greedy) and 1 (sampled) of the batched workload
+    threads = oracle.max_threads()
+    for _ in range(args.warmup):
+        oracle.verify_workload(w, nthreads=threads)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.verify_workload(w, nthreads=threads)
+    dt = (time.perf_counter() - t0) / max(1, args.steps)
+    value = w.R / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample": "sequences 0-1 of the batch (120 rows, one greedy, one sampled)",
+                   "V": w.V, "N": w.N},
+        "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": threads, "kind": "oracle",
+                         "sample": "2 of 32 sequences (120 of 1920 rows) per step"},
+        "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def cpu_baseline(w_dev, budget_s: float = 8.0):
+    """Times the oracle, as it stands, on the first k sequences of the benchmark batch."""
+    import oracle
+    threads = oracle.max_threads()
+    k = 2
+    best = None
+    while True:
+        t0 = time.perf_counter()
+        oracle.verify_workload(w_dev, nthreads=threads, seqs=list(range(k)))
+        dt = time.perf_counter() - t0
+        best = (k, dt)
+        if dt * 2.2 > budget_s or k >= w_dev.B:
+            break
+        k = min(w_dev.B, 2 * k)
+    k, dt = best
+    return {"value": k * w_dev.N / dt, "unit": "nodes/s", "cores": threads, "kind": "oracle",
+            "sample": f"first {k} of {w_dev.B} sequences ({k * w_dev.N} rows, V={w_dev.V}), {dt:.1f} s wall"}
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_12913_gb300 import dcd, workloads
+
+    world, rank, local = _dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    # weak scaling: every rank verifies its own full batch
+    w = workloads.make_config_torch(3, device=dev, seed=3 + rank)
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    out = dcd.alloc_outputs(B, N, dev)
+    ws = dcd.alloc_workspace(B, N, V, dev)
+    stream = torch.cuda.current_stream()
+
+    def step(i, evs=None):
+        if evs is not None:
+            evs[0].record(stream)
+        dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q, temperature=w.temperature,
+                           seed=w.seed, offset=i, out=out, workspace=ws, stream=stream)
+        if evs is not None:
+            evs[1].record(stream)
+        dcd.dcd_tree_walk(B, N, V, out, ws, stream=stream)
+
+    for i in range(args.warmup):
+        step(i)
+    if dcd.dcd_get_device_error(ws) != 0:
+        raise RuntimeError("device error bits set during warm-up")
+    sampler = ClockSampler(local)
+    sampler.start()
+    # keep the GPU busy for a second so the clock samples describe the loaded state
+    t_soak = time.time()
+    i = args.warmup
+    while time.time() - t_soak < 1.0:
+        step(i)
+        i += 1
+        if i % 64 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    start.record(stream)
+    for k in range(args.steps):
+        step(1_000_000 + k, evs[k])
+    stop.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t_wall1 = time.time()
+    sampler.stop()
+    elapsed_ms = start.elapsed_time(stop)
+    row_ms = [a.elapsed_time(b) for a, b in evs]
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    if dcd.dcd_get_device_error(ws) != 0:
+        raise RuntimeError("device error bits set during the timed region")
+    ms_per_step = elapsed_ms / args.steps
+    value = world * R / (ms_per_step / 1e3)
+
+    # roofline of the dominant kernel (the row kernel) from its own events
+    alg = algorithmic_bytes(w)
+    row_avg_s = statistics.mean(row_ms) / 1e3
+    achieved = alg / row_avg_s / 1e9
+    peak, peak_kind = _peaks()
+    khash = _kernel_source_hash()
+    traffic = _profiled_traffic(khash)
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": traffic, "kernel": "score_rows_kernel", "peak_source": f"{peak_kind} hbm_gbs",
+                "algorithmic_bytes_per_launch": alg, "row_kernel_ms": row_avg_s * 1e3,
+                "kernel_source_sha256_16": khash}
+
+    # end to end through the public API: pinned host inputs -> device, verify, results -> host
+    e2e = None
+    if rank == 0 or world > 1:
+        host = {k: getattr(w, k).cpu().pin_memory() for k in ("z_exp", "z_ama", "q", "tokens", "parents", "alpha",
+                                                               "beta", "temperature")}
+        dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
+        res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory() for k in ("accept_len", "accept_path",
+                                                                                     "bonus")}
+        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+        n_e2e = max(3, min(args.steps, 10))
+
+        def e2e_step(i):
+            for k in host:
+                dst[k].copy_(host[k], non_blocking=True)
+            o = dcd.dcd_verify_sample(dst["z_exp"], dst["z_ama"], dst["q"], dst["tokens"], dst["parents"],
+                                      dst["alpha"], dst["temperature"], w.seed, 2_000_000 + i, dst["beta"], out=out,
+                                      workspace=ws, stream=stream)
+            for k in res_host:
+                res_host[k].copy_(o[k], non_blocking=True)
+
+        e2e_step(0)
+        torch.cuda.synchronize()
+        a, b2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(n_e2e):
+            e2e_step(i + 1)
+        b2.record(stream)
+        torch.cuda.synchronize()
+        e_ms = a.elapsed_time(b2) / n_e2e
+        e2e = {"value": world * R / (e_ms / 1e3), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
+        del dst, host
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "B": B, "N": N, "V": V, "rows": R, "logits": "bf16",
+                       "sampled_sequences": int((w.temperature > 0).sum().item()),
+                       "bytes_per_step": alg, "l2": "inputs (1.48 GB per step) larger than L2; no flush",
+                       "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
+            "roofline": roofline,
+            "clocks": sampler.summary(t_wall0, t_wall1),
+            "e2e": e2e,
+            "gpu_launches": 2 * args.steps,
+        }
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(w)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,192 @@
+/*
+ * dcd.h -- C ABI of the GB300 (sm_103a) contrastive-decoding verification library.
+ *
+ * The library implements the verification step of Decoupled Contrastive Decoding
+ * (arxiv 2608.12913, Algorithm 1): for every node of a drafted token tree it turns
+ * the expert's and the amateur's vocabulary-wide logits into the CD target
+ *
+ *     log pi_CD(x) = (1 + alpha) log pi_p(x) - alpha log pi_q(x) - log Z_CD      (Eq. 1)
+ *
+ * optionally restricted to the expert-plausibility set
+ *     P_beta = { x : pi_p(x) >= beta * max_x' pi_p(x') }                          (Sec. 2.1)
+ * and sharpened by a temperature T (pi_CD,T proportional to exp(score / T) on P_beta),
+ * applies the greedy (T = 0) or the speculative-sampling acceptance rule, and walks
+ * the tree to the longest accepted path and its bonus token.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - B sequences, N tree nodes per sequence (the root included), vocabulary V.
+ *   Rows are numbered g = b * N + n; row g of a logit matrix holds the next-token
+ *   logits after node n of sequence b, i.e. the distribution node n's children
+ *   were drafted from.  The root's own token is context and is not verified.
+ * - parents[b*N + 0] = -1 and 0 <= parents[b*N + n] < n for n >= 1 (BFS-compatible
+ *   order); tokens[b*N + n] in [0, V) for n >= 1.  These device-resident arrays are
+ *   checked on the device: a violation sets a bit of the device error word (read
+ *   it with dcd_get_device_error) and that sequence reports accept_len = 0,
+ *   bonus = -1; nothing traps.
+ * - Siblings are tried in ascending node id.  Greedy: a child is accepted iff its
+ *   token equals the argmax of the CD score over P_beta (ties -> lowest token id;
+ *   duplicate sibling tokens -> lowest node id).  Sampled (T > 0): with r_0 = pi_CD,T
+ *   child j is accepted iff u_j <= r_{j-1}(t_j) / q(t_j); after a rejection
+ *   r_j = normalise(max(0, r_{j-1} - q)) (Algorithm 1, generalised to sibling lists);
+ *   a node with no accepted child draws its terminal token from its last residual
+ *   (pi_CD,T at a leaf) by an exponential race argmax_x log r(x) - log(-log u_x).
+ * - Randomness: Philox4x32-10 (Salmon et al., SC'11), key = (seed_lo, seed_hi).
+ *   The acceptance uniform of node c uses counter (b*N + c, 0, offset_lo, offset_hi)
+ *   word 0; the race uniform of token x in row g uses counter (g, 1 + x/4, offset_lo,
+ *   offset_hi) word x%4; a word w maps to u = ((w >> 9) + 0.5) * 2^-23 in (0, 1).
+ *   One call consumes one offset value: advance `offset` by one per call.
+ * - accept_len[b] counts accepted drafted tokens (the bonus token is excluded, as in
+ *   the paper's mean accepted length L, App. D).  accept_path[b*N + i] lists the
+ *   accepted node ids from the root (accept_path[b*N] = 0), padded with -1.
+ * - Optional outputs (may be NULL): cd_logprob[b*N + n] = log pi_CD,T_eff(token_n)
+ *   under the parent's row (root: 0; -inf outside P_beta), cd_argmax[g] = argmax of
+ *   the CD score of row g, cd_lse[g] = log sum_{x in P_beta} exp(s'(x) / T_eff) with
+ *   the raw-logit score s' = (1 + alpha) z_p - alpha z_q (so log pi_CD,T(x) =
+ *   s'(x) / T_eff - cd_lse[g]); T_eff = T, or 1 for greedy sequences.
+ * - Memory: every array pointer is a DEVICE pointer owned by the caller.  The
+ *   library allocates nothing per call; scratch lives in the caller's workspace
+ *   (dcd_workspace_bytes).  Calls are asynchronous and ordered on `stream`; host-side
+ *   argument checks return a negative status before anything is launched.  Two
+ *   calls that share a workspace must not overlap on the device.
+ * - Thread safety: entry points may be called from several host threads, each with
+ *   its own workspace.
+ */
+#ifndef DCD_H_
+#define DCD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* dcd_stream_t;
+
+/* Status codes returned by every entry point. */
+enum {
+  DCD_OK = 0,
+  DCD_ERR_INVALID_ARG = -1, /* null pointer, bad size, stride or dtype */
+  DCD_ERR_BAD_TREE = -2,    /* reserved: tree checks run on the device (see error word) */
+  DCD_ERR_UNSUPPORTED = -3, /* valid request this build cannot serve (e.g. N > DCD_MAX_NODES) */
+  DCD_ERR_CUDA = -4,        /* a CUDA runtime call or kernel launch failed */
+  DCD_ERR_TIMEOUT = -5,     /* a bounded device wait gave up (reported via the error word) */
+  DCD_ERR_DEVICE_INPUT = -6,/* dcd_get_device_error found a nonzero error word */
+  DCD_ERR_WORKSPACE = -7    /* workspace missing, misaligned (256 B) or too small */
+};
+
+/* Logit element types. */
+enum { DCD_F32 = 0, DCD_BF16 = 1 };
+
+/* Bits of the device error word (dcd_get_device_error). */
+#define DCD_DEVERR_BAD_PARENT 0x1u  /* parents[] violates the ordering rule */
+#define DCD_DEVERR_BAD_TOKEN 0x2u   /* a drafted token is outside [0, V) */
+#define DCD_DEVERR_NONFINITE 0x4u   /* NaN / +inf reached a row's max or normaliser */
+#define DCD_DEVERR_TIMEOUT 0x8u     /* a bounded wait on an asynchronous copy expired */
+#define DCD_DEVERR_BAD_PARAM 0x10u  /* alpha < 0, beta outside [0, 1], T < 0 or non-finite */
+
+/* Largest tree (nodes per sequence, root included) the library accepts. */
+#define DCD_MAX_NODES 1024
+
+typedef struct {
+  int32_t B;            /* sequences (>= 0) */
+  int32_t N;            /* nodes per sequence, root included (1 .. DCD_MAX_NODES) */
+  int64_t V;            /* vocabulary size (1 .. 2^31 - 1) */
+  int32_t logits_dtype; /* DCD_F32 or DCD_BF16, for z_exp and z_ama */
+  int32_t reserved;     /* must be 0 */
+  int64_t ld_logits;    /* row stride of z_exp / z_ama in elements (>= V) */
+  int64_t ld_q;         /* row stride of q in fp32 elements (>= V; sampled calls only) */
+} dcd_shape;
+
+/*
+ * Bytes of device workspace a call with this shape needs (the same value serves
+ * greedy and sampled calls).  Returns 0 for an invalid shape.
+ */
+size_t dcd_workspace_bytes(const dcd_shape* shape);
+
+/*
+ * Greedy CD verification (T = 0 for every sequence).  Eq. 1 with the plausibility
+ * mask of Sec. 2.1; acceptance is the T -> 0 limit of Algorithm 1.
+ *   z_exp, z_ama : [B*N rows, ld_logits] logits of the expert M_p and amateur M_q.
+ *   tokens, parents : int32 [B, N] draft tree (see conventions).
+ *   alpha : fp32 [B], contrastive strength alpha >= 0 (Eq. 1).
+ *   beta  : fp32 [B] plausibility threshold in [0, 1], or NULL for beta = 0.
+ *   accept_len [B], accept_path [B, N], bonus [B] : int32 outputs.
+ *   cd_logprob [B, N], cd_argmax [B, N], cd_lse [B, N] : optional outputs (NULL skips).
+ *   workspace : device scratch of at least dcd_workspace_bytes(shape), 256-byte aligned.
+ */
+int dcd_verify_greedy(const dcd_shape* shape, const void* z_exp, const void* z_ama, const int32_t* tokens,
+                      const int32_t* parents, const float* alpha, const float* beta, int32_t* accept_len,
+                      int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
+                      float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream);
+
+/*
+ * Speculative-sampling CD verification (Algorithm 1 on trees); sequences whose
+ * temperature is 0 follow the greedy rule within the same call.
+ *   q : fp32 [B*N rows, ld_q]; row g is the draft distribution pi_e that node n's
+ *       children were drawn from.  Read only for non-leaf rows of T > 0 sequences.
+ *   temperature : fp32 [B], T >= 0.
+ *   seed, offset : Philox key and stream position (see conventions).
+ *   residual : optional fp32 [B, V]; receives the distribution each sequence's bonus
+ *       token was drawn from (the last node's final residual; one-hot at the bonus
+ *       for greedy sequences).  Meant for tests; costs one extra pass per sequence.
+ * Other arguments as for dcd_verify_greedy.
+ */
+int dcd_verify_sample(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                      const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                      const float* temperature, uint64_t seed, uint64_t offset, int32_t* accept_len,
+                      int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
+                      float* cd_lse, float* residual, void* workspace, size_t workspace_bytes,
+                      dcd_stream_t stream);
+
+/*
+ * The two steps dcd_verify_sample is made of, exposed for step-level timing.
+ * dcd_score_rows runs the per-row work (Eq. 1 target, row reductions, sibling
+ * acceptance tests, terminal draws) and leaves one record per row in the workspace;
+ * q and temperature may be NULL for an all-greedy call.  dcd_tree_walk then
+ * follows the accepted children from each root and writes accept_len, accept_path
+ * and bonus.  Calling them back to back equals one dcd_verify_sample call with
+ * residual = NULL.
+ */
+int dcd_score_rows(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                   const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                   const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
+                   int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
+                   dcd_stream_t stream);
+
+int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_path, int32_t* bonus,
+                  void* workspace, size_t workspace_bytes, dcd_stream_t stream);
+
+/*
+ * dcd_score_rows with an explicit launch geometry, for tests and tuning: `cluster` is
+ * the number of CTAs sharing one row (0 = automatic, else 1, 2, 4, 8 or 16) and
+ * `plain_loads` = 1 stages rows with ordinary loads instead of bulk asynchronous
+ * copies.  Results equal dcd_score_rows up to fp32 summation order.
+ */
+int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                      const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                      const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
+                      int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
+                      dcd_stream_t stream, int cluster, int plain_loads);
+
+/*
+ * Synchronises `stream`, then copies the device error word of `workspace` (the OR of
+ * the DCD_DEVERR_* bits raised by the last call that used it) into *bits.  Returns
+ * DCD_OK when the word is zero, DCD_ERR_DEVICE_INPUT when it is not, DCD_ERR_CUDA if
+ * the copy fails.
+ */
+int dcd_get_device_error(const void* workspace, dcd_stream_t stream, uint32_t* bits);
+
+/* Static English text for a status code. */
+const char* dcd_status_string(int status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int dcd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DCD_H_ */

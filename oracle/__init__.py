@@ -87,7 +87,7 @@ def _load():
             lib.dcd_oracle_row_logpi.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, P, P, P, P, P, P]
             lib.dcd_oracle_row_chain.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, ctypes.c_int, P, P, P]
             lib.dcd_oracle_verify.argtypes = [I32, I32, I64, ctypes.c_int, I64, P, P, P, P, P, P, P, P, I64,
-                                              U64, U64, ctypes.c_int, P, P, P, P, P, P]
+                                              U64, U64, P, ctypes.c_int, P, P, P, P, P, P]
             lib.dcd_oracle_max_threads.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -177,7 +177,7 @@ def row_chain(zp, zq, alpha: float, beta: float, T: float, q, child_tokens, dtyp
 
 def verify(*, B: int, N: int, V: int, dtype: str, z_exp, z_ama, tokens, parents, alpha, beta=None,
            temperature=None, q=None, seed: int = 0, offset: int = 0, ld=None, ldq=None,
-           nthreads: int = 1, want_residual: bool = False) -> dict:
+           nthreads: int = 1, want_residual: bool = False, seq_ids=None) -> dict:
     """Full verification of B sequences x N nodes (see dcd_oracle_verify in the C source)."""
     zp = _logits(z_exp, dtype)
     zq = _logits(z_ama, dtype)
@@ -200,6 +200,7 @@ def verify(*, B: int, N: int, V: int, dtype: str, z_exp, z_ama, tokens, parents,
     be = _np(beta, np.float32)
     te = _np(temperature, np.float32)
     qq = _np(q, np.float32)
+    sid = _np(seq_ids, np.int32)
     ldq = (V if ldq is None else ldq) if qq is not None else 0
     R = B * N
     accept_len = np.zeros(B, dtype=np.int32)
@@ -210,7 +211,7 @@ def verify(*, B: int, N: int, V: int, dtype: str, z_exp, z_ama, tokens, parents,
     residual = np.zeros((B, V), dtype=np.float64) if want_residual else None
     rc = _load().dcd_oracle_verify(
         B, N, V, DTYPE_CODE[dtype], ld, _ptr(zp), _ptr(zq), _ptr(tok), _ptr(par), _ptr(al), _ptr(be),
-        _ptr(te), _ptr(qq), ldq, seed, offset, nthreads, _ptr(accept_len), _ptr(path), _ptr(bonus),
+        _ptr(te), _ptr(qq), ldq, seed, offset, _ptr(sid), nthreads, _ptr(accept_len), _ptr(path), _ptr(bonus),
         _ptr(logprob), _ptr(rows), _ptr(residual))
     if rc != 0:
         raise ValueError(f"oracle verify failed: {rc}")
@@ -223,14 +224,14 @@ def verify_workload(w, nthreads: int = 1, want_residual: bool = False, seqs=None
     import torch
     B, N, V = w.B, w.N, w.V
     sel = list(range(B)) if seqs is None else list(seqs)
-    rows = torch.cat([torch.arange(b * N, (b + 1) * N) for b in sel])
-    zp = w.z_exp.cpu()[rows]
-    zq = w.z_ama.cpu()[rows]
-    q = None if w.q is None else w.q.cpu()[rows]
+    rows = torch.cat([torch.arange(b * N, (b + 1) * N) for b in sel]).to(w.z_exp.device)
+    zp = w.z_exp[rows].cpu()
+    zq = w.z_ama[rows].cpu()
+    q = None if w.q is None else w.q[rows.to(w.q.device)].cpu()
     return verify(B=len(sel), N=N, V=V, dtype=w.dtype, z_exp=zp, z_ama=zq,
                   tokens=w.tokens.cpu()[sel], parents=w.parents.cpu()[sel], alpha=w.alpha.cpu()[sel],
                   beta=w.beta.cpu()[sel], temperature=w.temperature.cpu()[sel], q=q, seed=w.seed,
-                  offset=w.offset, nthreads=nthreads, want_residual=want_residual)
+                  offset=w.offset, nthreads=nthreads, want_residual=want_residual, seq_ids=np.asarray(sel))
 
 
 def margin_fn(zp_row, za_row, alpha: float, beta: float) -> float:

@@ -338,13 +338,15 @@ typedef struct {
  * (all zero).  Outputs: accept_len[B], accept_path[B*N] (node ids, padded with -1), bonus[B],
  * cd_logprob[B*N] (log pi_CD,T_eff(token_n) under the parent's row, root 0), rows[B*N], and
  * residual[B*V] (optional: the distribution each sequence's bonus was drawn from; one-hot at
- * the argmax for greedy sequences).
+ * the argmax for greedy sequences).  seq_ids (may be NULL = 0..B-1) gives each sequence's index
+ * in the batch it was drawn from; Philox counters use it, so a subset of a batch draws the same
+ * uniforms as the whole batch.
  * Returns 0, or a negative code for invalid arguments / a malformed tree.
  */
 int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, const void* zp, const void* zq,
                       const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                       const float* temperature, const float* q, int64_t ldq, uint64_t seed, uint64_t offset,
-                      int nthreads, int32_t* accept_len, int32_t* accept_path, int32_t* bonus,
+                      const int32_t* seq_ids, int nthreads, int32_t* accept_len, int32_t* accept_path, int32_t* bonus,
                       double* cd_logprob, dcd_oracle_row* rows, double* residual) {
   if (B < 0 || N < 1 || V < 1 || (dtype < 0 || dtype > 2) || ld < 0 || !zp || !zq || !tokens || !parents ||
       !alpha || !accept_len || !accept_path || !bonus || !cd_logprob || !rows)
@@ -426,7 +428,8 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
           const int32_t c = kids[k];
           const int32_t t = tokens[(int64_t)b * N + c];
           const double ratio = accept_ratio(r[t], (double)qr[t]);
-          const double u = dcd_oracle_accept_uniform(seed, offset, (uint32_t)((int64_t)b * N + c));
+          const int64_t sb = seq_ids ? seq_ids[b] : b;
+          const double u = dcd_oracle_accept_uniform(seed, offset, (uint32_t)(sb * N + c));
           ++out->n_tests;
           if (isfinite(ratio)) {
             const double d = fabs(u - ratio) / (ratio > 1.0 ? ratio : 1.0);
@@ -438,7 +441,10 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
           }
           residual_step(V, r, qr, tmp);
         }
-        if (out->acc_child < 0) out->term_token = race(V, r, seed, offset, (uint32_t)g, &out->gap_race);
+        if (out->acc_child < 0) {
+          const int64_t sb = seq_ids ? seq_ids[b] : b;
+          out->term_token = race(V, r, seed, offset, (uint32_t)(sb * N + n), &out->gap_race);
+        }
       }
     }
     free(lp);

@@ -1,0 +1,199 @@
+// dcd_api.cu -- the C ABI of include/dcd.h: argument checks, workspace layout and the
+// stream-ordered launches of the verification step.
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <climits>
+
+#include "dcd.h"
+#include "dcd_internal.h"
+
+namespace {
+
+constexpr int kVersion = 10000;  // 1.0.0
+
+bool shape_ok(const dcd_shape* s, bool need_q) {
+  if (!s) return false;
+  if (s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || s->reserved != 0) return false;
+  if (s->logits_dtype != DCD_F32 && s->logits_dtype != DCD_BF16) return false;
+  if (s->ld_logits < s->V) return false;
+  if (need_q && s->ld_q < s->V) return false;
+  if (static_cast<int64_t>(s->B) * s->N > INT_MAX / 16) return false;
+  return true;
+}
+
+size_t workspace_bytes_for(const dcd_shape* s) {
+  const size_t rows = static_cast<size_t>(s->B) * static_cast<size_t>(s->N);
+  const size_t raw = dcd::kWorkspaceHeader + rows * sizeof(dcd::RowRecord);
+  return (raw + 255) & ~static_cast<size_t>(255);
+}
+
+int check_workspace(const dcd_shape* s, const void* ws, size_t bytes) {
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return DCD_ERR_WORKSPACE;
+  if (bytes < workspace_bytes_for(s)) return DCD_ERR_WORKSPACE;
+  return DCD_OK;
+}
+
+dcd::RowRecord* records(void* ws) {
+  return reinterpret_cast<dcd::RowRecord*>(static_cast<char*>(ws) + dcd::kWorkspaceHeader);
+}
+
+uint32_t* error_word(void* ws) { return static_cast<uint32_t*>(ws); }
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? DCD_OK : DCD_ERR_CUDA; }
+
+dcd::ScoreArgs make_args(const dcd_shape* s, const void* z_exp, const void* z_ama, const float* q,
+                         const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                         const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
+                         int32_t* cd_argmax, float* cd_lse, void* ws) {
+  dcd::ScoreArgs a{};
+  a.zp = z_exp;
+  a.zq = z_ama;
+  a.q = q;
+  a.ld = s->ld_logits;
+  a.ldq = q ? s->ld_q : 0;
+  a.V = s->V;
+  a.tokens = tokens;
+  a.parents = parents;
+  a.alpha = alpha;
+  a.beta = beta;
+  a.temp = temperature;
+  a.B = s->B;
+  a.N = s->N;
+  a.dtype = s->logits_dtype;
+  a.seed = seed;
+  a.offset = offset;
+  a.cd_logprob = cd_logprob;
+  a.cd_argmax = cd_argmax;
+  a.cd_lse = cd_lse;
+  a.rec = records(ws);
+  a.err = error_word(ws);
+  a.force_cluster = 0;
+  a.force_plain = 0;
+  return a;
+}
+
+int score_rows_impl(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                    const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                    const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob, int32_t* cd_argmax,
+                    float* cd_lse, void* workspace, size_t workspace_bytes, cudaStream_t stream, int force_cluster,
+                    int force_plain) {
+  const bool sampled_call = temperature != nullptr;
+  if (!shape_ok(shape, sampled_call)) return DCD_ERR_INVALID_ARG;
+  if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
+  if (sampled_call && !q) return DCD_ERR_INVALID_ARG;
+  if (!sampled_call && q) return DCD_ERR_INVALID_ARG;
+  if (shape->B == 0) return DCD_OK;
+  if (!z_exp || !z_ama || !tokens || !parents || !alpha) return DCD_ERR_INVALID_ARG;
+  const int ws = check_workspace(shape, workspace, workspace_bytes);
+  if (ws != DCD_OK) return ws;
+  dcd::ScoreArgs a = make_args(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset,
+                               cd_logprob, cd_argmax, cd_lse, workspace);
+  a.force_cluster = force_cluster;
+  a.force_plain = force_plain;
+  const dcd::RowGeometry geo = dcd::row_geometry(a);
+  if (geo.smem > 227 * 1024) return DCD_ERR_UNSUPPORTED;
+  return cuda_status(dcd::launch_score_rows(a, stream));
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t dcd_workspace_bytes(const dcd_shape* shape) {
+  if (!shape_ok(shape, false)) return 0;
+  return workspace_bytes_for(shape);
+}
+
+int dcd_score_rows(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                   const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                   const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob, int32_t* cd_argmax,
+                   float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
+  return score_rows_impl(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset, cd_logprob,
+                         cd_argmax, cd_lse, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), 0, 0);
+}
+
+int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_path, int32_t* bonus,
+                  void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
+  if (!shape_ok(shape, false)) return DCD_ERR_INVALID_ARG;
+  if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
+  if (shape->B == 0) return DCD_OK;
+  if (!accept_len || !accept_path || !bonus) return DCD_ERR_INVALID_ARG;
+  const int ws = check_workspace(shape, workspace, workspace_bytes);
+  if (ws != DCD_OK) return ws;
+  return cuda_status(dcd::launch_tree_walk(shape->B, shape->N, records(workspace), error_word(workspace), accept_len,
+                                           accept_path, bonus, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dcd_verify_greedy(const dcd_shape* shape, const void* z_exp, const void* z_ama, const int32_t* tokens,
+                      const int32_t* parents, const float* alpha, const float* beta, int32_t* accept_len,
+                      int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax, float* cd_lse,
+                      void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
+  if (!shape_ok(shape, false)) return DCD_ERR_INVALID_ARG;
+  if (shape->B > 0 && (!accept_len || !accept_path || !bonus)) return DCD_ERR_INVALID_ARG;
+  int rc = dcd_score_rows(shape, z_exp, z_ama, nullptr, tokens, parents, alpha, beta, nullptr, 0, 0, cd_logprob,
+                          cd_argmax, cd_lse, workspace, workspace_bytes, stream);
+  if (rc != DCD_OK) return rc;
+  return dcd_tree_walk(shape, accept_len, accept_path, bonus, workspace, workspace_bytes, stream);
+}
+
+int dcd_verify_sample(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                      const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                      const float* temperature, uint64_t seed, uint64_t offset, int32_t* accept_len,
+                      int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax, float* cd_lse,
+                      float* residual, void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
+  if (!shape_ok(shape, true)) return DCD_ERR_INVALID_ARG;
+  if (!temperature || !q) return DCD_ERR_INVALID_ARG;
+  if (shape->B > 0 && (!accept_len || !accept_path || !bonus)) return DCD_ERR_INVALID_ARG;
+  int rc = dcd_score_rows(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset,
+                          cd_logprob, cd_argmax, cd_lse, workspace, workspace_bytes, stream);
+  if (rc != DCD_OK) return rc;
+  rc = dcd_tree_walk(shape, accept_len, accept_path, bonus, workspace, workspace_bytes, stream);
+  if (rc != DCD_OK || !residual || shape->B == 0) return rc;
+  dcd::ScoreArgs a = make_args(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset,
+                               cd_logprob, cd_argmax, cd_lse, workspace);
+  return cuda_status(dcd::launch_terminal_residual(a, accept_len, accept_path, bonus, residual,
+                                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dcd_get_device_error(const void* workspace, dcd_stream_t stream, uint32_t* bits) {
+  if (!workspace || !bits) return DCD_ERR_INVALID_ARG;
+  uint32_t host = 0;
+  cudaError_t e = cudaMemcpyAsync(&host, workspace, sizeof host, cudaMemcpyDeviceToHost,
+                                  reinterpret_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return DCD_ERR_CUDA;
+  *bits = host;
+  return host ? DCD_ERR_DEVICE_INPUT : DCD_OK;
+}
+
+const char* dcd_status_string(int status) {
+  switch (status) {
+    case DCD_OK: return "ok";
+    case DCD_ERR_INVALID_ARG: return "invalid argument";
+    case DCD_ERR_BAD_TREE: return "malformed draft tree";
+    case DCD_ERR_UNSUPPORTED: return "unsupported request";
+    case DCD_ERR_CUDA: return "CUDA error";
+    case DCD_ERR_TIMEOUT: return "device wait timed out";
+    case DCD_ERR_DEVICE_INPUT: return "device-side input error";
+    case DCD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    default: return "unknown status";
+  }
+}
+
+int dcd_version(void) { return kVersion; }
+
+// Test and tuning hook: dcd_score_rows with a forced cluster size and/or plain loads.
+int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                      const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
+                      const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
+                      int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
+                      int cluster, int plain_loads) {
+  if (cluster != 0 && (cluster < 1 || cluster > 16 || (cluster & (cluster - 1)) != 0)) return DCD_ERR_INVALID_ARG;
+  return score_rows_impl(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset, cd_logprob,
+                         cd_argmax, cd_lse, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream),
+                         cluster, plain_loads);
+}
+
+}  // extern "C"

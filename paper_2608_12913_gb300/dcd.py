@@ -1,0 +1,275 @@
+"""Thin ctypes binding of libdcd.so (include/dcd.h), same entry-point names.
+
+Argument marshalling only: every step of the verification runs in the CUDA
+library.  Tensors are torch CUDA tensors (torch provides device memory and
+streams); the library never sees a torch type.  There is no CPU fallback: if
+the library cannot be built or loaded, or no CUDA device is present, the calls
+raise.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+DCD_OK = 0
+DCD_F32, DCD_BF16 = 0, 1
+DEVERR_BITS = {0x1: "bad_parent", 0x2: "bad_token", 0x4: "nonfinite", 0x8: "timeout", 0x10: "bad_param"}
+MAX_NODES = 1024
+
+_lock = threading.Lock()
+_lib = None
+
+
+class DcdShape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("N", ctypes.c_int32), ("V", ctypes.c_int64),
+                ("logits_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("ld_logits", ctypes.c_int64), ("ld_q", ctypes.c_int64)]
+
+
+class DcdError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True):
+    """Loads (building first if needed) libdcd.so and declares its C signatures."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if build_if_missing:
+            path = _build.build()
+        if not os.path.exists(path):
+            raise RuntimeError(f"libdcd.so is not built ({path})")
+        lib = ctypes.CDLL(path)
+        P, I32, U64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint64, ctypes.c_size_t
+        SH = ctypes.POINTER(DcdShape)
+        lib.dcd_workspace_bytes.argtypes = [SH]
+        lib.dcd_workspace_bytes.restype = SZ
+        lib.dcd_verify_greedy.argtypes = [SH, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
+        lib.dcd_verify_sample.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, P, P, P, P, SZ, P]
+        lib.dcd_score_rows.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P]
+        lib.dcd_score_rows_ex.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P,
+                                          ctypes.c_int, ctypes.c_int]
+        lib.dcd_tree_walk.argtypes = [SH, P, P, P, P, SZ, P]
+        lib.dcd_get_device_error.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
+        lib.dcd_status_string.argtypes = [ctypes.c_int]
+        lib.dcd_status_string.restype = ctypes.c_char_p
+        lib.dcd_version.restype = ctypes.c_int
+        for name in ("dcd_verify_greedy", "dcd_verify_sample", "dcd_score_rows", "dcd_score_rows_ex",
+                     "dcd_tree_walk", "dcd_get_device_error"):
+            getattr(lib, name).restype = I32
+        _lib = lib
+        return lib
+
+
+def status_string(status: int) -> str:
+    return load().dcd_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != DCD_OK:
+        raise DcdError(status, where)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _require(t, name, dtype=None, device=None, shape=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor (the library has no CPU path)")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+
+
+def _logits_dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return DCD_BF16
+    if t.dtype == torch.float32:
+        return DCD_F32
+    raise TypeError(f"logits must be bfloat16 or float32, got {t.dtype}")
+
+
+def make_shape(B: int, N: int, V: int, dtype: int, ld: Optional[int] = None, ldq: Optional[int] = None) -> DcdShape:
+    return DcdShape(B, N, V, dtype, 0, V if ld is None else ld, (V if ldq is None else ldq))
+
+
+def workspace_bytes(B: int, N: int, V: int, dtype: int = DCD_BF16) -> int:
+    sh = make_shape(B, N, V, dtype)
+    n = load().dcd_workspace_bytes(ctypes.byref(sh))
+    if n == 0:
+        raise ValueError("invalid shape")
+    return int(n)
+
+
+def alloc_workspace(B: int, N: int, V: int, device, dtype: int = DCD_BF16) -> torch.Tensor:
+    ws = torch.zeros(workspace_bytes(B, N, V, dtype), dtype=torch.uint8, device=device)
+    assert ws.data_ptr() % 256 == 0
+    return ws
+
+
+def alloc_outputs(B: int, N: int, device, V: Optional[int] = None, residual: bool = False) -> dict:
+    out = dict(
+        accept_len=torch.empty(B, dtype=torch.int32, device=device),
+        accept_path=torch.empty((B, N), dtype=torch.int32, device=device),
+        bonus=torch.empty(B, dtype=torch.int32, device=device),
+        cd_logprob=torch.empty((B, N), dtype=torch.float32, device=device),
+        cd_argmax=torch.empty((B, N), dtype=torch.int32, device=device),
+        cd_lse=torch.empty((B, N), dtype=torch.float32, device=device),
+    )
+    if residual:
+        out["residual"] = torch.empty((B, V), dtype=torch.float32, device=device)
+    return out
+
+
+class _Call:
+    """Validated arguments of one verification call."""
+
+    def __init__(self, z_exp, z_ama, tokens, parents, alpha, beta, q=None, temperature=None):
+        _require(z_exp, "z_exp")
+        dev = z_exp.device
+        if z_exp.dim() != 2 or z_exp.stride(1) != 1:
+            raise ValueError("z_exp must be a 2-D tensor with unit stride along the vocabulary")
+        _require(z_ama, "z_ama", dtype=z_exp.dtype, device=dev, shape=z_exp.shape)
+        if z_ama.stride() != z_exp.stride():
+            raise ValueError("z_exp and z_ama must share one row stride")
+        _require(tokens, "tokens", dtype=torch.int32, device=dev)
+        if tokens.dim() != 2 or not tokens.is_contiguous():
+            raise ValueError("tokens must be a contiguous [B, N] int32 tensor")
+        B, N = tokens.shape
+        V = z_exp.shape[1]
+        if z_exp.shape[0] != B * N:
+            raise ValueError(f"z_exp has {z_exp.shape[0]} rows, expected B*N = {B * N}")
+        _require(parents, "parents", dtype=torch.int32, device=dev, shape=(B, N))
+        if not parents.is_contiguous():
+            raise ValueError("parents must be contiguous")
+        _require(alpha, "alpha", dtype=torch.float32, device=dev, shape=(B,))
+        if beta is not None:
+            _require(beta, "beta", dtype=torch.float32, device=dev, shape=(B,))
+        ldq = None
+        if q is not None:
+            _require(q, "q", dtype=torch.float32, device=dev)
+            if q.dim() != 2 or q.shape[0] != B * N or q.shape[1] != V or q.stride(1) != 1:
+                raise ValueError("q must be a [B*N, V] float32 tensor with unit stride along the vocabulary")
+            ldq = q.stride(0)
+        if temperature is not None:
+            _require(temperature, "temperature", dtype=torch.float32, device=dev, shape=(B,))
+        self.device = dev
+        self.B, self.N, self.V = B, N, V
+        self.shape = make_shape(B, N, V, _logits_dtype(z_exp), z_exp.stride(0), ldq)
+        self.args = (z_exp, z_ama, q, tokens, parents, alpha, beta, temperature)
+
+    def workspace(self, workspace):
+        need = load().dcd_workspace_bytes(ctypes.byref(self.shape))
+        if workspace is None:
+            return torch.empty(need, dtype=torch.uint8, device=self.device)
+        _require(workspace, "workspace", dtype=torch.uint8, device=self.device)
+        if workspace.numel() < need:
+            raise ValueError(f"workspace has {workspace.numel()} bytes, needs {need}")
+        return workspace
+
+    def outputs(self, out, residual=False):
+        if out is None:
+            return alloc_outputs(self.B, self.N, self.device, self.V, residual)
+        return out
+
+
+def dcd_verify_greedy(z_exp, z_ama, tokens, parents, alpha, beta=None, *, out=None, workspace=None,
+                      stream=None) -> dict:
+    """Greedy CD verification; returns accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse."""
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta)
+    ws = c.workspace(workspace)
+    o = c.outputs(out)
+    st = load().dcd_verify_greedy(
+        ctypes.byref(c.shape), _ptr(z_exp), _ptr(z_ama), _ptr(tokens), _ptr(parents), _ptr(alpha), _ptr(beta),
+        _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]), _ptr(o.get("cd_logprob")),
+        _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(ws), ws.numel(), _stream(stream))
+    _check(st, "dcd_verify_greedy")
+    o["workspace"] = ws
+    return o
+
+
+def dcd_verify_sample(z_exp, z_ama, q, tokens, parents, alpha, temperature, seed: int, offset: int, beta=None, *,
+                      residual: bool = False, out=None, workspace=None, stream=None) -> dict:
+    """Speculative-sampling CD verification (greedy for sequences with temperature 0)."""
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
+    ws = c.workspace(workspace)
+    o = c.outputs(out, residual=residual)
+    st = load().dcd_verify_sample(
+        ctypes.byref(c.shape), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(tokens), _ptr(parents), _ptr(alpha),
+        _ptr(beta), _ptr(temperature), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+        _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]), _ptr(o.get("cd_logprob")),
+        _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(o.get("residual") if residual else None), _ptr(ws),
+        ws.numel(), _stream(stream))
+    _check(st, "dcd_verify_sample")
+    o["workspace"] = ws
+    return o
+
+
+def dcd_score_rows(z_exp, z_ama, tokens, parents, alpha, beta=None, q=None, temperature=None, seed: int = 0,
+                   offset: int = 0, *, out=None, workspace=None, stream=None, cluster: int = 0,
+                   plain_loads: bool = False) -> dict:
+    """The per-row step alone (records stay in the workspace); see dcd_tree_walk."""
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
+    ws = c.workspace(workspace)
+    o = c.outputs(out)
+    lib = load()
+    common = (ctypes.byref(c.shape), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(tokens), _ptr(parents), _ptr(alpha),
+              _ptr(beta), _ptr(temperature), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+              _ptr(o.get("cd_logprob")), _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(ws), ws.numel(),
+              _stream(stream))
+    if cluster or plain_loads:
+        st = lib.dcd_score_rows_ex(*common, int(cluster), int(bool(plain_loads)))
+    else:
+        st = lib.dcd_score_rows(*common)
+    _check(st, "dcd_score_rows")
+    o["workspace"] = ws
+    return o
+
+
+def dcd_tree_walk(B: int, N: int, V: int, out: dict, workspace, stream=None) -> dict:
+    """Tree walk over the records a previous dcd_score_rows left in `workspace`."""
+    sh = make_shape(B, N, V, DCD_BF16)
+    st = load().dcd_tree_walk(ctypes.byref(sh), _ptr(out["accept_len"]), _ptr(out["accept_path"]),
+                              _ptr(out["bonus"]), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, "dcd_tree_walk")
+    return out
+
+
+def dcd_get_device_error(workspace: torch.Tensor, stream=None) -> int:
+    """Synchronises the stream and returns the device error bits of the last call on `workspace`."""
+    bits = ctypes.c_uint32(0)
+    st = load().dcd_get_device_error(_ptr(workspace), _stream(stream), ctypes.byref(bits))
+    if st not in (DCD_OK, -6):
+        raise DcdError(st, "dcd_get_device_error")
+    return int(bits.value)
+
+
+def version() -> int:
+    return int(load().dcd_version())

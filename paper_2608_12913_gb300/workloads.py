@@ -178,7 +178,7 @@ def generate(*, name: str, B: int, V: int, dtype: str, spikes=(1, 6),
              temperatures: Sequence[float] = (0.0,), levels: Optional[Sequence[int]] = None,
              chain_len: Optional[int] = None, seed: int = 0, offset: int = 0,
              margin_fn: Optional[Callable] = None, margin: float = 1e-3,
-             max_attempts: int = 100) -> Workload:
+             max_attempts: int = 100, max_children: int = MAX_CHILDREN) -> Workload:
     """Numpy generator (CPU tensors). Per-sequence alpha/T cycle through the given lists.
 
     ``margin_fn(zp_row, za_row, alpha, beta) -> float`` receives the rounded logits
@@ -189,7 +189,7 @@ def generate(*, name: str, B: int, V: int, dtype: str, spikes=(1, 6),
         tree = [chain_parents(chain_len) for _ in range(B)]
     else:
         lv = tuple(levels) if levels is not None else TREE_LEVELS_60
-        tree = [tree_parents(_rng(seed, _S_TREE, b), lv) for b in range(B)]
+        tree = [tree_parents(_rng(seed, _S_TREE, b), lv, max_children) for b in range(B)]
     N = len(tree[0])
     assert all(len(t) == N for t in tree)
     R = B * N

@@ -1,0 +1,130 @@
+"""Shared helpers of the GPU-versus-oracle parity tests.
+
+Bars (stated once, used by every parity test):
+* token ids, argmax, accepted lengths, accepted paths, bonus tokens and the per-row
+  acceptance records: bit-exact;
+* cd_logprob and cd_lse (the CD scores): within 1e-4 absolute (fp32 on the GPU
+  against the fp64 oracle);
+* the residual a bonus was drawn from: total variation within 1e-5.
+
+Where floating point decides an integer, the two sides decide in different
+precisions (fp32 kernel, fp64 oracle).  The oracle reports every decision's
+margin; a row whose margin is below what fp32 can resolve is "ambiguous": its
+decision is not compared, and a sequence whose oracle path crosses an ambiguous
+row is only checked for validity.  Inputs drawn with the margin rule have none.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2608_12913_gb300 import dcd
+
+SCORE_TOL = 1e-4
+TV_TOL = 1e-5
+# margins below which fp32 and fp64 may legitimately decide differently
+AMB_ARGMAX = 2e-5
+AMB_ACCEPT = 1e-5
+AMB_RACE = 1e-4
+AMB_MASK = 1e-5
+
+
+def records(ws: torch.Tensor, R: int):
+    """Per-row records the row kernel leaves after the 256-byte workspace header."""
+    raw = ws[256:256 + 16 * R].cpu().numpy().view(np.int32).reshape(R, 4)
+    return dict(acc_child=raw[:, 0].copy(), term_token=raw[:, 1].copy(), status=raw[:, 2].view(np.uint32).copy())
+
+
+def run_gpu(w, *, sampled: bool, residual: bool = False, cluster: int = 0, plain: bool = False, offset=None,
+            out=None, workspace=None):
+    dev = torch.device("cuda")
+    wd = w.to(dev)
+    off = w.offset if offset is None else offset
+    if cluster or plain:
+        q = None
+        temp = None
+        if sampled:
+            q = wd.q if wd.q is not None else torch.zeros_like(wd.z_exp, dtype=torch.float32)
+            temp = wd.temperature
+        o = dcd.dcd_score_rows(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta, q=q, temperature=temp,
+                               seed=w.seed, offset=off, cluster=cluster, plain_loads=plain, out=out,
+                               workspace=workspace)
+        dcd.dcd_tree_walk(w.B, w.N, w.V, o, o["workspace"])
+    elif sampled:
+        q = wd.q if wd.q is not None else torch.zeros_like(wd.z_exp, dtype=torch.float32)
+        o = dcd.dcd_verify_sample(wd.z_exp, wd.z_ama, q, wd.tokens, wd.parents, wd.alpha, wd.temperature, w.seed, off,
+                                  wd.beta, residual=residual, out=out, workspace=workspace)
+    else:
+        o = dcd.dcd_verify_greedy(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta, out=out,
+                                  workspace=workspace)
+    torch.cuda.synchronize()
+    res = {k: v.cpu().numpy() for k, v in o.items() if k != "workspace"}
+    res["records"] = records(o["workspace"], w.B * w.N)
+    res["error_bits"] = dcd.dcd_get_device_error(o["workspace"])
+    return res
+
+
+def compare(w, gpu: dict, ref: dict, seqs=None, check_residual: bool = False, max_amb_frac: float = 0.05):
+    """Asserts parity of GPU outputs (all sequences of `w`, or the subset `seqs`) with the oracle's."""
+    B, N = w.B, w.N
+    sel = np.arange(B) if seqs is None else np.asarray(seqs)
+    rows_ref = ref["rows"]  # [len(sel), N]
+    gsel = (sel[:, None] * N + np.arange(N)[None, :]).reshape(-1)
+    rr = rows_ref.reshape(-1)
+    amb = ((rr["gap_argmax"] < AMB_ARGMAX) | (rr["gap_accept"] < AMB_ACCEPT) | (rr["gap_race"] < AMB_RACE) |
+           (rr["gap_mask"] < AMB_MASK))
+    assert gpu["error_bits"] == 0, f"device error bits {gpu['error_bits']:#x}"
+    assert np.all(gpu["records"]["status"][gsel] == 0)
+
+    # Eq. 1 scores, within tolerance everywhere
+    lse_g = gpu["cd_lse"].reshape(-1)[gsel].astype(np.float64)
+    lse_err = np.abs(lse_g - rr["cd_lse"])
+    assert lse_err.max() <= SCORE_TOL, f"cd_lse max error {lse_err.max():.3g}"
+    lp_g = gpu["cd_logprob"][sel].astype(np.float64)
+    lp_r = ref["cd_logprob"]
+    both_inf = np.isneginf(lp_g) & np.isneginf(lp_r)
+    assert np.array_equal(np.isneginf(lp_g), np.isneginf(lp_r)), "plausibility masks differ"
+    with np.errstate(invalid="ignore"):
+        lp_err = np.where(both_inf, 0.0, np.abs(lp_g - lp_r))
+    assert lp_err.max() <= SCORE_TOL, f"cd_logprob max error {lp_err.max():.3g}"
+
+    # integer decisions per row: bit-exact where the margin is resolvable in fp32
+    arg_g = gpu["cd_argmax"].reshape(-1)[gsel]
+    ok_arg = rr["gap_argmax"] >= AMB_ARGMAX
+    assert np.array_equal(arg_g[ok_arg], rr["argmax"][ok_arg]), "cd_argmax mismatch"
+    acc_g = gpu["records"]["acc_child"][gsel]
+    term_g = gpu["records"]["term_token"][gsel]
+    bad = np.nonzero((acc_g != rr["acc_child"]) & ~amb)[0]
+    assert bad.size == 0, f"accepted-child mismatch at rows {gsel[bad][:8]}: gpu {acc_g[bad][:8]} " \
+                          f"oracle {rr['acc_child'][bad][:8]} gap_accept {rr['gap_accept'][bad][:8]}"
+    bad = np.nonzero((term_g != rr["term_token"]) & ~amb)[0]
+    assert bad.size == 0, f"terminal-token mismatch at rows {gsel[bad][:8]}: gpu {term_g[bad][:8]} " \
+                          f"oracle {rr['term_token'][bad][:8]} gap_race {rr['gap_race'][bad][:8]}"
+
+    # sequences
+    amb_rows = amb.reshape(len(sel), N)
+    n_amb = 0
+    for i, b in enumerate(sel):
+        path = ref["accept_path"][i]
+        on = path[path >= 0]
+        if amb_rows[i, on].any():
+            n_amb += 1
+            # validity only: a path of real parent-child links from the root
+            gp = gpu["accept_path"][b]
+            L = gpu["accept_len"][b]
+            assert gp[0] == 0 and np.all(gp[L + 1:] == -1)
+            par = w.parents[b].cpu().numpy()
+            for k in range(1, L + 1):
+                assert par[gp[k]] == gp[k - 1]
+            continue
+        assert gpu["accept_len"][b] == ref["accept_len"][i], f"accept_len mismatch in sequence {b}"
+        assert np.array_equal(gpu["accept_path"][b], ref["accept_path"][i]), f"path mismatch in sequence {b}"
+        assert gpu["bonus"][b] == ref["bonus"][i], f"bonus mismatch in sequence {b}"
+        if check_residual:
+            tv = 0.5 * np.abs(gpu["residual"][b].astype(np.float64) - ref["residual"][i]).sum()
+            assert tv <= TV_TOL, f"residual TV {tv:.3g} in sequence {b}"
+    assert n_amb <= max(1, int(max_amb_frac * len(sel))), f"{n_amb} ambiguous sequences"
+    return dict(ambiguous_rows=int(amb.sum()), ambiguous_seqs=n_amb, max_lse_err=float(lse_err.max()),
+                max_logprob_err=float(lp_err.max()))

@@ -1,0 +1,118 @@
+"""C-ABI checks that need no GPU: the library builds, loads and exports every symbol
+declared in include/*.h, and host-side argument checks reject bad calls before any
+launch (no compute call is made here)."""
+
+import ctypes
+import glob
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2608_12913_gb300 import build as dcd_build
+from paper_2608_12913_gb300 import dcd
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w\s\*]*?\b(dcd_\w+)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    dcd_build.build()
+    return dcd.load()
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for required in ("dcd_verify_greedy", "dcd_verify_sample", "dcd_workspace_bytes", "dcd_score_rows",
+                     "dcd_tree_walk", "dcd_get_device_error", "dcd_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    out = subprocess.run(["nm", "-D", "--defined-only", dcd_build.LIB], capture_output=True, text=True, check=True)
+    exported = {line.split()[-1] for line in out.stdout.splitlines() if line.strip()}
+    missing = [n for n in names if n not in exported]
+    assert not missing, f"declared but not exported: {missing}"
+    for n in names:
+        assert hasattr(lib, n)
+
+
+def test_library_is_built_for_sm_103a(lib):
+    out = subprocess.run(["cuobjdump", "--list-elf", dcd_build.LIB], capture_output=True, text=True)
+    if out.returncode != 0:
+        pytest.skip("cuobjdump unavailable")
+    assert "sm_103a" in out.stdout
+
+
+def test_status_strings_and_version(lib):
+    assert dcd.status_string(0) == "ok"
+    assert "argument" in dcd.status_string(-1)
+    assert "workspace" in dcd.status_string(-7)
+    assert dcd.version() >= 10000
+
+
+def test_workspace_bytes(lib):
+    n = dcd.workspace_bytes(32, 60, 128256)
+    assert n >= 256 + 32 * 60 * 16 and n % 256 == 0
+    bad = dcd.make_shape(1, 0, 10, 0)
+    assert lib.dcd_workspace_bytes(ctypes.byref(bad)) == 0
+    bad = dcd.make_shape(1, 4, 10, 5)
+    assert lib.dcd_workspace_bytes(ctypes.byref(bad)) == 0
+    bad = dcd.make_shape(1, 4, 10, 0, ld=9)
+    assert lib.dcd_workspace_bytes(ctypes.byref(bad)) == 0
+
+
+def _fake(addr):
+    return ctypes.c_void_p(addr)
+
+
+def test_host_checks_reject_before_launch(lib):
+    """Invalid calls return a negative status; the fake pointers are never dereferenced."""
+    P = _fake(0x10000)
+    sh = dcd.make_shape(2, 4, 100, dcd.DCD_BF16)
+    ws_ok = _fake(0x100000)
+    base = [P, P, P, P, P, None, P, P, P, None, None, None]
+    # null shape
+    assert lib.dcd_verify_greedy(None, *base, ws_ok, 1 << 20, None) == -1
+    # null logits
+    assert lib.dcd_verify_greedy(ctypes.byref(sh), None, *base[1:], ws_ok, 1 << 20, None) == -1
+    # misaligned workspace / too small
+    assert lib.dcd_verify_greedy(ctypes.byref(sh), *base, _fake(0x100010), 1 << 20, None) == -7
+    assert lib.dcd_verify_greedy(ctypes.byref(sh), *base, ws_ok, 64, None) == -7
+    # unsupported tree size
+    big = dcd.make_shape(1, 2000, 100, dcd.DCD_BF16)
+    assert lib.dcd_verify_greedy(ctypes.byref(big), *base, ws_ok, 1 << 30, None) == -3
+    # sampled call without q or temperature
+    assert lib.dcd_verify_sample(ctypes.byref(sh), P, P, None, P, P, P, None, P, 0, 0, P, P, P, None, None, None,
+                                 None, ws_ok, 1 << 20, None) == -1
+    assert lib.dcd_verify_sample(ctypes.byref(sh), P, P, P, P, P, P, None, None, 0, 0, P, P, P, None, None, None,
+                                 None, ws_ok, 1 << 20, None) == -1
+    # row stride shorter than the vocabulary
+    bad = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, ld=50)
+    assert lib.dcd_verify_greedy(ctypes.byref(bad), *base, ws_ok, 1 << 20, None) == -1
+    # invalid forced cluster size
+    assert lib.dcd_score_rows_ex(ctypes.byref(sh), P, P, None, P, P, P, None, None, 0, 0, None, None, None, ws_ok,
+                                 1 << 20, None, 3, 0) == -1
+    # empty batch is a no-op
+    empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
+    assert lib.dcd_verify_greedy(ctypes.byref(empty), *base, ws_ok, 1 << 20, None) == 0
+
+
+def test_binding_refuses_cpu_tensors():
+    import torch
+    z = torch.zeros((6, 10))
+    t = torch.zeros((1, 6), dtype=torch.int32)
+    with pytest.raises(ValueError, match="CUDA"):
+        dcd.dcd_verify_greedy(z, z, t, t, torch.zeros(1))

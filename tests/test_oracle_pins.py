@@ -413,3 +413,16 @@ def test_invalid_trees_rejected():
         oracle.verify(tokens=np.array([[0, 0, V]], np.int32), parents=np.array([[-1, 0, 1]], np.int32), **base)
     with pytest.raises(ValueError):
         oracle.verify(tokens=np.zeros((1, 3), np.int32), parents=np.array([[0, 0, 1]], np.int32), **base)
+
+
+def test_subset_of_a_batch_draws_the_batch_uniforms():
+    """Verifying a subset of sequences (with their batch indices) reproduces the batch's results."""
+    from paper_2608_12913_gb300 import workloads
+    w = workloads.make_config(3, B=6, V=300, seed=31)
+    full = oracle.verify_workload(w)
+    sub = oracle.verify_workload(w, seqs=[4, 1])
+    for i, b in enumerate([4, 1]):
+        assert full["accept_len"][b] == sub["accept_len"][i]
+        assert full["bonus"][b] == sub["bonus"][i]
+        assert np.array_equal(full["rows"][b]["acc_child"], sub["rows"][i]["acc_child"])
+        assert np.array_equal(full["rows"][b]["term_token"], sub["rows"][i]["term_token"])
