@@ -160,6 +160,37 @@ int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_p
                   void* workspace, size_t workspace_bytes, dcd_stream_t stream);
 
 /*
+ * Capacity of the scratch array inside the library used by dcd_verify_sample_noalloc:
+ * enough for dcd_workspace_bytes(shape) <= 512 KiB, i.e. B * N <= 32752 rows.
+ */
+#define DCD_STATIC_SCRATCH_BYTES (512u * 1024u)
+
+/*
+ * dcd_verify_sample without a workspace argument, for callers that cannot allocate
+ * device memory: for example a plugin inside an inference engine that reserves all
+ * device memory for its own allocator, or a hook that must not call cudaMalloc or
+ * cudaFree because they can synchronise the device or fail under a fixed budget.
+ * (The paper has no counterpart; this is a deployment convenience of the library.)
+ * The caller still passes every input and output; the scratch lives in one array of
+ * DCD_STATIC_SCRATCH_BYTES compiled into the library, which every GPU that loads the
+ * library holds until the process exits.  Shapes needing more scratch return
+ * DCD_ERR_UNSUPPORTED.  Nothing is allocated: no cudaMalloc, cudaFree or allocating
+ * library call.  The first call on a device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any stream capture.
+ * All calls share the one array and it keeps the last call's contents (each call resets
+ * the error word and rewrites every record it reads), so calls that overlap on the GPU,
+ * from any stream or thread, race and must be serialised by the caller.
+ * dcd_get_device_error cannot read this scratch; device-side input errors still show
+ * as accept_len = 0 and bonus = -1 for the affected sequences.
+ * Arguments and results otherwise as dcd_verify_sample.
+ */
+int dcd_verify_sample_noalloc(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                              const int32_t* tokens, const int32_t* parents, const float* alpha,
+                              const float* beta, const float* temperature, uint64_t seed, uint64_t offset,
+                              int32_t* accept_len, int32_t* accept_path, int32_t* bonus, float* cd_logprob,
+                              int32_t* cd_argmax, float* cd_lse, float* residual, dcd_stream_t stream);
+
+/*
  * dcd_score_rows with an explicit launch geometry, for tests and tuning: `cluster` is
  * the number of CTAs sharing one row (0 = automatic, else 1, 2, 4, 8 or 16) and
  * `plain_loads` = 1 stages rows with ordinary loads instead of bulk asynchronous

@@ -62,6 +62,8 @@ def load(build_if_missing: bool = True):
         lib.dcd_verify_greedy.argtypes = [SH, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
         lib.dcd_verify_sample.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, P, P, P, P, SZ, P]
         lib.dcd_score_rows.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P]
+        lib.dcd_verify_sample_noalloc.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, P, P, P, P]
+        lib.dcd_verify_sample_noalloc.restype = I32
         lib.dcd_score_rows_ex.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P,
                                           ctypes.c_int, ctypes.c_int]
         lib.dcd_tree_walk.argtypes = [SH, P, P, P, P, SZ, P]
@@ -229,6 +231,25 @@ def dcd_verify_sample(z_exp, z_ama, q, tokens, parents, alpha, temperature, seed
         ws.numel(), _stream(stream))
     _check(st, "dcd_verify_sample")
     o["workspace"] = ws
+    return o
+
+
+def dcd_verify_sample_noalloc(z_exp, z_ama, q, tokens, parents, alpha, temperature, seed: int, offset: int,
+                              beta=None, *, residual: bool = False, out=None, stream=None) -> dict:
+    """dcd_verify_sample with the library's built-in scratch instead of a caller workspace.
+
+    For callers that cannot allocate device memory (see include/dcd.h).  Calls that overlap on the
+    GPU share that scratch and race; the caller serialises them.
+    """
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
+    o = c.outputs(out, residual=residual)
+    st = load().dcd_verify_sample_noalloc(
+        ctypes.byref(c.shape), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(tokens), _ptr(parents), _ptr(alpha),
+        _ptr(beta), _ptr(temperature), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+        _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]), _ptr(o.get("cd_logprob")),
+        _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(o.get("residual") if residual else None),
+        _stream(stream))
+    _check(st, "dcd_verify_sample_noalloc")
     return o
 
 
