@@ -197,7 +197,7 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     # weak scaling: every rank verifies its own full batch
-    w = workloads.make_config_torch(3, device=dev, seed=3 + rank)
+    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch)
     B, N, V = w.B, w.N, w.V
     R = B * N
     out = dcd.alloc_outputs(B, N, dev)
@@ -222,7 +222,7 @@ def run_ours(args):
     # keep the GPU busy for a second so the clock samples describe the loaded state
     t_soak = time.time()
     i = args.warmup
-    while time.time() - t_soak < 1.0:
+    while not args.no_soak and time.time() - t_soak < 1.0:
         step(i)
         i += 1
         if i % 64 == 0:
@@ -269,7 +269,7 @@ def run_ours(args):
 
     # end to end through the public API: pinned host inputs -> device, verify, results -> host
     e2e = None
-    if rank == 0 or world > 1:
+    if not args.no_e2e:
         host = {k: getattr(w, k).cpu().pin_memory() for k in ("z_exp", "z_ama", "q", "tokens", "parents", "alpha",
                                                                "beta", "temperature")}
         dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
@@ -297,6 +297,10 @@ def run_ours(args):
         b2.record(stream)
         torch.cuda.synchronize()
         e_ms = a.elapsed_time(b2) / n_e2e
+        if world > 1:
+            t = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e_ms = float(t.item())
         e2e = {"value": world * R / (e_ms / 1e3), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
         del dst, host
@@ -306,7 +310,7 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "B": B, "N": N, "V": V, "rows": R, "logits": "bf16",
+            "config": {"workload": WORKLOAD if B == 32 else f"{WORKLOAD} (profiling case, B={B})", "B": B, "N": N, "V": V, "rows": R, "logits": "bf16",
                        "sampled_sequences": int((w.temperature > 0).sum().item()),
                        "bytes_per_step": alg, "l2": "inputs (1.48 GB per step) larger than L2; no flush",
                        "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
@@ -331,6 +335,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
+    ap.add_argument("--no-soak", action="store_true", help="skip the 1 s clock soak (profiling runs)")
+    ap.add_argument("--batch", type=int, default=32,
+                    help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

@@ -84,6 +84,8 @@ def _load():
             lib.dcd_oracle_accept_uniform.restype = D
             lib.dcd_oracle_race_uniform.argtypes = [U64, U64, ctypes.c_uint32, I64]
             lib.dcd_oracle_race_uniform.restype = D
+            lib.dcd_oracle_block_uniform.argtypes = [U64, U64, ctypes.c_uint32, I64]
+            lib.dcd_oracle_block_uniform.restype = D
             lib.dcd_oracle_row_logpi.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, P, P, P, P, P, P]
             lib.dcd_oracle_row_chain.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, ctypes.c_int, P, P, P]
             lib.dcd_oracle_verify.argtypes = [I32, I32, I64, ctypes.c_int, I64, P, P, P, P, P, P, P, P, I64,
@@ -137,6 +139,10 @@ def accept_uniform(seed: int, offset: int, G: int) -> float:
 
 def race_uniform(seed: int, offset: int, G: int, x: int) -> float:
     return float(_load().dcd_oracle_race_uniform(seed, offset, G, x))
+
+
+def block_uniform(seed: int, offset: int, G: int, k: int) -> float:
+    return float(_load().dcd_oracle_block_uniform(seed, offset, G, k))
 
 
 def row_logpi(zp, zq, alpha: float, beta: float = 0.0, T: float = 1.0, dtype: str = "f64") -> dict:

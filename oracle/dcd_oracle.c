@@ -33,10 +33,12 @@
  * as 1, 2, 3", SC'11), key = (seed_lo, seed_hi).  The acceptance uniform of
  * node c (global id G = b*N + c) uses counter (G, 0, off_lo, off_hi), word 0;
  * the race uniform of token x in row G uses counter (G, 1 + x/4, off_lo,
- * off_hi), word x%4.  A 32-bit word w becomes u = ((w >> 9) + 0.5) * 2^-23, a
- * value in (0, 1) that fp32 also holds exactly.  Terminal tokens are drawn by
- * an exponential race: argmax_x log r(x) - log(-log u_x), ties to the lowest
- * token id.
+ * off_hi), word x%4; the race uniform of token block k (ids 256k .. 256k+255)
+ * uses counter (G, 2^31 + k/4, off_lo, off_hi), word k%4.  A 32-bit word w
+ * becomes u = ((w >> 9) + 0.5) * 2^-23, a value in (0, 1) that fp32 also holds
+ * exactly.  Terminal tokens are drawn by a two-level exponential race: a block
+ * by argmax_k log R_k - log(-log u_k) over the blocks' masses R_k, then a token
+ * of that block by argmax_x log r(x) - log(-log u_x); ties to the lowest id.
  *
  * Besides the outputs, every row reports decision margins (top-2 score gap,
  * |u - ratio| of every acceptance test taken, top-2 race-key gap, distance of
@@ -105,6 +107,11 @@ double dcd_oracle_accept_uniform(uint64_t seed, uint64_t offset, uint32_t G) {
 /* Exponential-race uniform of token x in global row G. */
 double dcd_oracle_race_uniform(uint64_t seed, uint64_t offset, uint32_t G, int64_t x) {
   return dcd_oracle_u01(philox_word(seed, offset, G, (uint32_t)(1 + (x >> 2)), (int)(x & 3)));
+}
+
+/* Exponential-race uniform of token block k (tokens 256k .. 256k+255) in global row G. */
+double dcd_oracle_block_uniform(uint64_t seed, uint64_t offset, uint32_t G, int64_t k) {
+  return dcd_oracle_u01(philox_word(seed, offset, G, 0x80000000u | (uint32_t)(k >> 2), (int)(k & 3)));
 }
 
 /* ---------------------------------------------------------------- inputs */
@@ -238,23 +245,54 @@ static double accept_ratio(double rt, double qt) {
   return rt > 0.0 ? INFINITY : 0.0;
 }
 
-/* Exponential race over r; returns the winner and writes the top-2 key gap. */
+#define RACE_BLOCK 256
+
+/*
+ * Draw from r (unnormalised, r >= 0) by a two-level exponential race: first a block of
+ * RACE_BLOCK consecutive token ids, k* = argmax_k log R_k - log(-log u_k) with R_k the block's
+ * mass, then a token of that block, argmax_x log r(x) - log(-log u_x).  Each level is a
+ * Gumbel-max draw, so P(x) = (R_k / sum R) (r(x) / R_k) = r(x) / sum r, with k the block of x.
+ * Ties go to the lowest id.
+ * Writes the smaller of the two levels' top-2 key gaps.
+ */
 static int32_t race(int64_t V, const double* r, uint64_t seed, uint64_t offset, uint32_t G, double* gap) {
+  const int64_t nblk = (V + RACE_BLOCK - 1) / RACE_BLOCK;
   double best = -INFINITY, second = -INFINITY;
-  int32_t arg = -1;
-  for (int64_t x = 0; x < V; ++x) {
-    if (!(r[x] > 0.0)) continue;
-    const double u = dcd_oracle_race_uniform(seed, offset, G, x);
-    const double key = log(r[x]) - log(-log(u));
+  int64_t kbest = -1;
+  for (int64_t k = 0; k < nblk; ++k) {
+    double mass = 0.0;
+    for (int64_t x = k * RACE_BLOCK; x < V && x < (k + 1) * RACE_BLOCK; ++x) mass += r[x];
+    if (!(mass > 0.0)) continue;
+    const double u = dcd_oracle_block_uniform(seed, offset, G, k);
+    const double key = log(mass) - log(-log(u));
     if (key > best) {
       second = best;
       best = key;
-      arg = (int32_t)x;
+      kbest = k;
     } else if (key > second) {
       second = key;
     }
   }
-  *gap = best - second;
+  const double gap1 = best - second;
+  best = -INFINITY;
+  second = -INFINITY;
+  int32_t arg = -1;
+  if (kbest >= 0) {
+    for (int64_t x = kbest * RACE_BLOCK; x < V && x < (kbest + 1) * RACE_BLOCK; ++x) {
+      if (!(r[x] > 0.0)) continue;
+      const double u = dcd_oracle_race_uniform(seed, offset, G, x);
+      const double key = log(r[x]) - log(-log(u));
+      if (key > best) {
+        second = best;
+        best = key;
+        arg = (int32_t)x;
+      } else if (key > second) {
+        second = key;
+      }
+    }
+  }
+  const double gap2 = best - second;
+  *gap = gap1 < gap2 ? gap1 : gap2;
   return arg;
 }
 

@@ -227,6 +227,41 @@ def test_exponential_race_samples_target():
     assert np.all(res["accept_len"] == 0)
 
 
+@pytest.mark.parametrize("T", [1.0, 0.7])
+def test_two_level_race_samples_target_across_blocks(T):
+    """V spans several 256-token blocks (the last one ragged): the bonus is still drawn from pi_CD."""
+    rng = np.random.default_rng(78)
+    V, B = 600, 120000
+    zp = 0.6 * rng.standard_normal(V)
+    zp[[5, 300, 599]] += 2.5  # mass in every block
+    zq = 0.7 * zp + 0.5 * rng.standard_normal(V)
+    res = oracle.verify(B=B, N=1, V=V, dtype="f64", z_exp=zp, z_ama=zq, ld=0,
+                        tokens=np.zeros((B, 1), np.int32), parents=np.full((B, 1), -1, np.int32),
+                        alpha=np.full(B, 0.3), temperature=np.full(B, T), q=np.zeros(V, np.float32), ldq=0,
+                        seed=4, offset=2, nthreads=4)
+    pi = np.exp(oracle.row_logpi(zp, zq, 0.3, 0.0, T)["logpi"])
+    counts = np.bincount(res["bonus"], minlength=V)
+    # block marginals and the token-level fit
+    for lo, hi in ((0, 256), (256, 512), (512, 600)):
+        p = pi[lo:hi].sum()
+        assert abs(counts[lo:hi].sum() / B - p) < 4 * np.sqrt(p * (1 - p) / B)
+    assert stats.chisquare(counts, B * pi).pvalue > 1e-4
+
+
+def test_race_returns_a_point_mass_wherever_it_sits():
+    """A row whose whole mass is on one token (first, last or interior of a block, or in the ragged
+    last block) always yields that token, whatever the uniforms."""
+    V, B = 700, 400
+    for hot in (0, 255, 256, 511, 512, 640, 699):
+        zp = np.zeros(V)
+        zp[hot] = 200.0  # exp(-200) leaves every other token without representable mass
+        res = oracle.verify(B=B, N=1, V=V, dtype="f64", z_exp=zp, z_ama=zp, ld=0,
+                            tokens=np.zeros((B, 1), np.int32), parents=np.full((B, 1), -1, np.int32),
+                            alpha=np.full(B, 0.2), temperature=np.full(B, 1.0), q=np.zeros(V, np.float32), ldq=0,
+                            seed=hot, offset=1)
+        assert np.all(res["bonus"] == hot)
+
+
 # ----------------------------------------------------------------------------- Algorithm 1 on chains
 
 def _algorithm1_chain(zp_rows, zq_rows, q_rows, drafts, alpha, T, seed, offset, b, N):
@@ -250,9 +285,21 @@ def _algorithm1_chain(zp_rows, zq_rows, q_rows, drafts, alpha, T, seed, offset, 
     else:
         P = pis[gamma]
         row = gamma
-    keys = [np.log(P[x]) - np.log(-np.log(oracle.race_uniform(seed, offset, b * N + row, x))) if P[x] > 0 else -np.inf
-            for x in range(V)]
-    return k - 1, int(np.argmax(keys))
+    return k - 1, _two_level_race(P, seed, offset, b * N + row)
+
+
+def _two_level_race(P, seed, offset, G, block=256):
+    """Sample from P with the library's two-level exponential race (block, then token)."""
+    V = len(P)
+    nb = (V + block - 1) // block
+    mass = np.array([P[k * block:(k + 1) * block].sum() for k in range(nb)])
+    kk = [np.log(mass[k]) - np.log(-np.log(oracle.block_uniform(seed, offset, G, k))) if mass[k] > 0 else -np.inf
+          for k in range(nb)]
+    kb = int(np.argmax(kk))
+    xs = range(kb * block, min(V, (kb + 1) * block))
+    keys = [np.log(P[x]) - np.log(-np.log(oracle.race_uniform(seed, offset, G, x))) if P[x] > 0 else -np.inf
+            for x in xs]
+    return kb * block + int(np.argmax(keys))
 
 
 def test_chain_reduces_to_algorithm1():
