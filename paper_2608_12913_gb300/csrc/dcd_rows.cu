@@ -1,16 +1,17 @@
 // dcd_rows.cu -- the streaming kernels of the CD verification step on sm_103a.
 //
 // score_rows_kernel: one thread-block cluster per tree-node row g = b * N + n.  The
-//   row's vocabulary is split into `cluster` contiguous slices (multiples of 8
+//   row's vocabulary is split into `cluster` contiguous slices (whole blocks of 256
 //   tokens); each CTA stages its slice of z_p, z_q (and q for sampled non-leaf rows)
 //   in shared memory with bulk asynchronous copies, so HBM is read exactly once per
 //   row however many passes the row needs.  Passes over shared memory compute, in
 //   order: the expert max (only when beta > 0, for the plausibility set of Sec. 2.1),
-//   the CD score s' = (1 + alpha) z_p - alpha z_q and its argmax (Eq. 1; the two
-//   log-softmax shifts are constant per row and cancel in the normaliser), the
-//   normaliser sum exp((s' - max) / T), then for sampled rows the sibling-rejection
-//   chain of Algorithm 1 (one residual pass per rejected child, r_j = max(0, r_{j-1}
-//   - q) / Z_j, computed in place) and the exponential race of the terminal draw.
+//   the CD score s' = (1 + alpha) z_p - alpha z_q with its max and argmax (Eq. 1; the
+//   two log-softmax shifts are constant per row and cancel in the normaliser), stored
+//   in place; the normaliser sum exp((s' - max) / T); then for sampled rows the
+//   sibling-rejection chain of Algorithm 1 (one residual pass per rejected child,
+//   r_j = max(0, r_{j-1} - q) / Z_j, in place) and the terminal draw, a two-level
+//   exponential race (a 256-token block by its mass, then a token of that block).
 //   Per-CTA partials are combined across the cluster through distributed shared
 //   memory; every CTA combines them in the same order, so all CTAs take identical
 //   decisions and run the same number of cluster barriers.
@@ -38,9 +39,11 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxCluster = 16;
-constexpr size_t kSmemBudget = 64 * 1024;  // data bytes per CTA the automatic geometry aims for
+constexpr size_t kSmemBudget = 64 * 1024 + 1024;  // data bytes per CTA the automatic geometry aims for
 constexpr size_t kSmemMax = 227 * 1024;
 constexpr long long kWaitCycles = 4000000000ll;  // about two seconds at the boost clock
+constexpr int kRaceBlock = 256;                  // tokens per block of the two-level terminal race
+constexpr float kLog2e = 1.4426950408889634f;
 
 // ------------------------------------------------------------------------------------------
 // PTX wrappers: mbarrier and bulk asynchronous global->shared copies.
@@ -143,9 +146,6 @@ __device__ __forceinline__ void lds8(const __nv_bfloat16* p, float v[8]) {
   v[4] = __uint_as_float(a.z << 16); v[5] = __uint_as_float(a.z & 0xffff0000u);
   v[6] = __uint_as_float(a.w << 16); v[7] = __uint_as_float(a.w & 0xffff0000u);
 }
-
-__device__ __forceinline__ float lds1(const float* p, int i) { return p[i]; }
-__device__ __forceinline__ float lds1(const __nv_bfloat16* p, int i) { return __bfloat162float(p[i]); }
 
 __device__ __forceinline__ void st8_value(float* zp, float* /*zq*/, int i0, const float v[8]) {
   reinterpret_cast<float4*>(zp + i0)[0] = make_float4(v[0], v[1], v[2], v[3]);
@@ -275,10 +275,40 @@ __device__ __forceinline__ void cluster_exchange(cg::cluster_group& cl, Partial*
 struct KParams {
   ScoreArgs a;
   int32_t cluster;
-  int32_t chunk;   // tokens per CTA (multiple of 8)
+  int32_t chunk;   // tokens per CTA (multiple of kRaceBlock)
   int32_t bulk;    // 1: bulk asynchronous copies, 0: plain loads
   int32_t data_offset;
 };
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float lg2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(~0u, v, o);
+  return v;
+}
+
+// log2 of a Gumbel-race divisor: key = log2 r - log2(-log2 u) orders tokens exactly as
+// ln r - ln(-ln u) does (the two differ by a positive factor and a constant).
+__device__ __forceinline__ float race_key(float log2_mass, uint32_t word) {
+  return log2_mass - lg2(-lg2(u01(word)));
+}
+
+__device__ __forceinline__ uint32_t philox_word(uint64_t seed, uint64_t off, uint32_t c0, uint32_t c1, int word) {
+  const uint4 w = philox4x32_10(make_uint4(c0, c1, (uint32_t)off, (uint32_t)(off >> 32)), (uint32_t)seed,
+                                (uint32_t)(seed >> 32));
+  return word == 0 ? w.x : word == 1 ? w.y : word == 2 ? w.z : w.w;
+}
 
 // ------------------------------------------------------------------------------------------
 template <typename TIn>
@@ -302,6 +332,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   int* kids = meta + 8;
   int* ktok = kids + N;
   float* ksv = reinterpret_cast<float*>(ktok + N);
+  float* blk = ksv + N;  // per 256-token block masses of this slice
   TIn* zp_s = reinterpret_cast<TIn*>(smem + kp.data_offset);
   TIn* zq_s = zp_s + kp.chunk;
   float* q_s = reinterpret_cast<float*>(zq_s + kp.chunk);
@@ -317,6 +348,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   const float T = p.temp ? p.temp[b] : 0.f;
   const bool sampled = T > 0.f;
   const float invT = sampled ? 1.f / T : 1.f;
+  const float k2 = kLog2e * invT;  // exp(x / T) = 2^(x * k2)
 
   if (g == 0 && rank == 0 && tid == 0) *p.err = 0u;
 
@@ -390,7 +422,9 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   }
   __syncthreads();
 
-  const int ngroups = (len + 7) >> 3;
+  // Loops run over 8-token groups; a warp's 32 groups are one 256-token race block, and the
+  // group count is rounded up to whole warps so every branch on `grp < ngw` is warp-uniform.
+  const int ngw = (((len + 7) >> 3) + 31) & ~31;
   const bool masked = beta > 0.f;
   const float logb = masked ? logf(beta) : -INFINITY;
   const float c1 = 1.f + alpha;
@@ -402,7 +436,9 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   float Mp = 0.f;
   if (masked) {
     float lm = -INFINITY;
-    for (int grp = tid; grp < ngroups; grp += kThreads) {
+    for (int base = 0; base < ngw; base += kThreads) {
+      const int grp = base + tid;
+      if (grp >= ngw) continue;
       const int i0 = grp << 3;
       float zp[8];
       lds8(zp_s + i0, zp);
@@ -417,68 +453,78 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
     for (int k = 0; k < C; ++k) Mp = fmaxf(Mp, gath[k].m);
   }
 
-  // ---- pass B: CD score argmax over the slice
+  // ---- pass B: CD score s' = (1 + alpha) z_p - alpha z_q on P_beta (-inf elsewhere), its max and
+  // argmax; s' overwrites the slice in place as fp32
   float best = -INFINITY;
   int barg = INT_MAX;
-  for (int grp = tid; grp < ngroups; grp += kThreads) {
+  for (int base = 0; base < ngw; base += kThreads) {
+    const int grp = base + tid;
+    if (grp >= ngw) continue;
     const int i0 = grp << 3;
-    float zp[8], zq[8];
+    float zp[8], zq[8], sv[8];
     lds8(zp_s + i0, zp);
     lds8(zq_s + i0, zq);
+    float gm = -INFINITY;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-      if (i0 + e >= len) break;
-      if (masked && !(zp[e] - Mp >= logb)) continue;
-      const float s = fmaf(c1, zp[e], -alpha * zq[e]);
-      if (s > best) {
-        best = s;
-        barg = static_cast<int>(lo) + i0 + e;
-      }
+      const bool in = (i0 + e < len) && (!masked || (zp[e] - Mp >= logb));
+      sv[e] = in ? fmaf(c1, zp[e], -alpha * zq[e]) : -INFINITY;
+      gm = fmaxf(gm, sv[e]);
     }
+    if (gm > best) {
+      best = gm;
+#pragma unroll
+      for (int e = 7; e >= 0; --e)
+        if (sv[e] == gm) barg = static_cast<int>(lo) + i0 + e;
+    }
+    st8_value(zp_s, zq_s, i0, sv);
   }
-  // children's scores, captured by the CTA whose slice holds the token (before pass C may
-  // overwrite the slice)
+  block_argmax(best, barg, redf, redi);  // ends with __syncthreads: every s' is stored
+  const float m_cta = best;
+  // children's scores, read by the CTA whose slice holds the token
   for (int k = tid; k < m; k += kThreads) {
     const int t = ktok[k];
-    if (t >= lo && t < hi) {
-      const float z = lds1(zp_s, t - static_cast<int>(lo));
-      const float zz = lds1(zq_s, t - static_cast<int>(lo));
-      const bool in = !masked || (z - Mp >= logb);
-      ksv[k] = in ? fmaf(c1, z, -alpha * zz) : -INFINITY;
-    }
+    if (t >= lo && t < hi) ksv[k] = ld1_value(zp_s, zq_s, t - static_cast<int>(lo));
   }
-  block_argmax(best, barg, redf, redi);
-  const float m_cta = best;
+  __syncthreads();  // the captures above finish before pass C rewrites the slice
 
-  // ---- pass C: normaliser; sampled non-leaf rows keep e(x) = exp((s' - m_cta) / T) in place
-  const bool store_e = sampled && m > 0;
+  // ---- pass C: normaliser sum 2^((s' - m_cta) k2); sampled rows keep e(x) in place, and leaf rows
+  // (whose terminal draw races over pi_CD itself) keep the 256-token block masses
+  const bool leaf_race = sampled && m == 0;
   float ssum = 0.f;
   if (m_cta > -INFINITY) {
-    for (int grp = tid; grp < ngroups; grp += kThreads) {
+    const float mk2 = m_cta * k2;
+    for (int base = 0; base < ngw; base += kThreads) {
+      const int grp = base + tid;
+      if (grp >= ngw) continue;
       const int i0 = grp << 3;
-      float zp[8], zq[8], ev[8];
-      lds8(zp_s + i0, zp);
-      lds8(zq_s + i0, zq);
+      float sv[8];
+      ld8_value(zp_s, zq_s, i0, sv);
+      float part = 0.f;
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
-        const bool in = (i0 + e < len) && (!masked || (zp[e] - Mp >= logb));
-        const float s = fmaf(c1, zp[e], -alpha * zq[e]);
-        ev[e] = in ? __expf((s - m_cta) * invT) : 0.f;
-        ssum += ev[e];
+        sv[e] = ex2(fmaf(sv[e], k2, -mk2));
+        part += sv[e];
       }
-      if (store_e) st8_value(zp_s, zq_s, i0, ev);
+      ssum += part;
+      if (sampled) st8_value(zp_s, zq_s, i0, sv);
+      if (leaf_race) {
+        const float bs = warp_sum(part);
+        if (lane == 0) blk[grp >> 5] = bs;
+      }
     }
-  } else if (store_e) {
+  } else if (sampled) {
     const float zero[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int grp = tid; grp < ngroups; grp += kThreads) st8_value(zp_s, zq_s, grp << 3, zero);
+    for (int grp = tid; grp < ngw; grp += kThreads) st8_value(zp_s, zq_s, grp << 3, zero);
+    for (int t = tid; t < (ngw >> 5); t += kThreads) blk[t] = 0.f;
   }
-  const float s_cta = block_sum(ssum, redf);  // ends with __syncthreads: stored values visible
+  const float s_cta = block_sum(ssum, redf);  // ends with __syncthreads
 
   mine = neutral_partial();
   mine.m = m_cta;
   mine.s = s_cta;
   mine.arg = barg;
-  if (store_e && tid == 0) {
+  if (sampled && m > 0 && tid == 0) {
     const int t = ktok[0];
     if (t >= lo && t < hi) {
       mine.cap_own = 1;
@@ -497,12 +543,12 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   for (int k = 0; k < C; ++k) {
     status |= gath[k].status;
     if (gath[k].m == M && arg == INT_MAX) arg = gath[k].arg;
-    if (gath[k].m > -INFINITY) S += gath[k].s * expf((gath[k].m - M) * invT);
+    if (gath[k].m > -INFINITY) S += gath[k].s * exp2f((gath[k].m - M) * k2);
   }
   if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
   for (int k = 0; k < C; ++k)
     if (gath[k].cap_own) {
-      rt = gath[k].cap_r * (expf((gath[k].m - M) * invT) / S);
+      rt = gath[k].cap_r * (exp2f((gath[k].m - M) * k2) / S);
       qt = gath[k].cap_q;
     }
   const float logS = logf(S);
@@ -517,7 +563,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
     for (int k = tid; k < m; k += kThreads) {
       const int t = ktok[k];
       if (t >= lo && t < hi)
-        p.cd_logprob[static_cast<int64_t>(b) * N + kids[k]] = ksv[k] > -INFINITY ? (ksv[k] - M) * invT - logS : -INFINITY;
+        p.cd_logprob[static_cast<int64_t>(b) * N + kids[k]] =
+            ksv[k] > -INFINITY ? (ksv[k] - M) * invT - logS : -INFINITY;
     }
   }
 
@@ -531,8 +578,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       }
     if (acc < 0) term = arg;
   } else {
-    // ---- sampled rule: sibling-rejection chain, then the terminal race if needed
-    const float scale_me = m_cta > -INFINITY ? expf((m_cta - M) * invT) / S : 0.f;
+    // ---- sampled rule: sibling-rejection chain over the slice, then the terminal race if needed
+    const float scale_me = m_cta > -INFINITY ? exp2f((m_cta - M) * k2) / S : 0.f;
     float invZ = 0.f;
     bool degen = false;
     for (int j = 0; j < m; ++j) {
@@ -543,21 +590,31 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         acc = kids[j];
         break;
       }
-      // rejected: r_{j+1} = max(0, r_j - q) / Z, written over the slice
+      // rejected: r_{j+1} = max(0, r_j - q) / Z, written over the slice; the last residual also
+      // records its block masses for the terminal race
+      const bool last = j == m - 1;
       float zsum = 0.f;
-      for (int grp = tid; grp < ngroups; grp += kThreads) {
+      for (int base = 0; base < ngw; base += kThreads) {
+        const int grp = base + tid;
+        if (grp >= ngw) continue;
         const int i0 = grp << 3;
         float r[8], qv[8];
         ld8_value(zp_s, zq_s, i0, r);
         lds8(q_s + i0, qv);
+        float part = 0.f;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const float prev = j == 0 ? r[e] * scale_me : (degen ? qv[e] : r[e] * invZ);
           const float nv = (i0 + e < len) ? fmaxf(prev - qv[e], 0.f) : 0.f;
           r[e] = nv;
-          zsum += nv;
+          part += nv;
         }
         st8_value(zp_s, zq_s, i0, r);
+        zsum += part;
+        if (last) {
+          const float bs = warp_sum(part);
+          if (lane == 0) blk[grp >> 5] = bs;
+        }
       }
       zsum = block_sum(zsum, redf);
       mine = neutral_partial();
@@ -590,58 +647,87 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       qt = cq;
     }
     if (acc < 0) {
-      // exponential race: argmax_x log r(x) - log(-log u_x); constants common to all x dropped
-      const uint32_t k0 = static_cast<uint32_t>(p.seed), k1 = static_cast<uint32_t>(p.seed >> 32);
-      const uint32_t o0 = static_cast<uint32_t>(p.offset), o1 = static_cast<uint32_t>(p.offset >> 32);
-      const bool leaf = m == 0;
-      float bk = -INFINITY;
-      int ba = INT_MAX;
-      for (int grp = tid; grp < ngroups; grp += kThreads) {
-        const int i0 = grp << 3;
-        const uint32_t x0 = static_cast<uint32_t>(lo) + static_cast<uint32_t>(i0);
-        float val[8];
-        if (leaf) {
-          float zp[8], zq[8];
-          lds8(zp_s + i0, zp);
-          lds8(zq_s + i0, zq);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const bool in = (i0 + e < len) && (!masked || (zp[e] - Mp >= logb));
-            val[e] = in ? (fmaf(c1, zp[e], -alpha * zq[e]) - M) * invT : -INFINITY;
-          }
-        } else {
-          float r[8], qv[8];
-          ld8_value(zp_s, zq_s, i0, r);
+      // ---- terminal draw: two-level exponential race (block of 256 tokens, then a token)
+      if (degen) {  // the residual is q itself: its block masses
+        for (int base = 0; base < ngw; base += kThreads) {
+          const int grp = base + tid;
+          if (grp >= ngw) continue;
+          const int i0 = grp << 3;
+          float qv[8];
           lds8(q_s + i0, qv);
+          float part = 0.f;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float rv = degen ? qv[e] : r[e];
-            val[e] = (i0 + e < len && rv > 0.f) ? logf(rv) : -INFINITY;
-          }
+          for (int e = 0; e < 8; ++e) part += (i0 + e < len) ? qv[e] : 0.f;
+          const float bs = warp_sum(part);
+          if (lane == 0) blk[grp >> 5] = bs;
         }
-        const uint4 wa = philox4x32_10(make_uint4(static_cast<uint32_t>(g), 1u + (x0 >> 2), o0, o1), k0, k1);
-        const uint4 wb = philox4x32_10(make_uint4(static_cast<uint32_t>(g), 2u + (x0 >> 2), o0, o1), k0, k1);
-        const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          if (val[e] > -INFINITY) {
-            const float key = val[e] - logf(-logf(u01(w[e])));
-            if (key > bk) {
-              bk = key;
-              ba = static_cast<int>(x0) + e;
-            }
+        __syncthreads();
+      }
+      // leaf rows hold e(x) relative to this CTA's max; bring block masses to the common scale
+      const float offset2 = leaf_race ? (m_cta - M) * k2 : 0.f;
+      const int nblk = (len + kRaceBlock - 1) / kRaceBlock;
+      const int kbase = static_cast<int>(lo / kRaceBlock);
+      float bk = -INFINITY;
+      int bb = INT_MAX;
+      for (int t = tid; t < nblk; t += kThreads) {
+        const float R = blk[t];
+        if (R > 0.f) {
+          const uint32_t kabs = static_cast<uint32_t>(kbase + t);
+          const float key = race_key(lg2(R) + offset2,
+                                     philox_word(p.seed, p.offset, static_cast<uint32_t>(g),
+                                                 0x80000000u | (kabs >> 2), static_cast<int>(kabs & 3)));
+          if (key > bk) {
+            bk = key;
+            bb = static_cast<int>(kabs);
           }
         }
       }
-      block_argmax(bk, ba, redf, redi);
+      block_argmax(bk, bb, redf, redi);
       mine = neutral_partial();
       mine.m = bk;
-      mine.arg = ba;
+      mine.arg = bb;
       cluster_exchange(cl, part, gath, stage, mine, C);
       float K = -INFINITY;
-      int ka = INT_MAX;
-      for (int k = 0; k < C; ++k) argmax_merge(K, ka, gath[k].m, gath[k].arg);
-      term = ka;
+      int kstar = INT_MAX;
+      for (int k = 0; k < C; ++k) argmax_merge(K, kstar, gath[k].m, gath[k].arg);
+      // token race inside block kstar, by the CTA whose slice holds it (one warp, 8 tokens a lane)
+      mine = neutral_partial();
+      const int64_t x_first = static_cast<int64_t>(kstar) * kRaceBlock;
+      if (kstar != INT_MAX && x_first >= lo && x_first < hi && warp == 0) {
+        const int i0 = static_cast<int>(x_first - lo) + lane * 8;
+        float r[8], qv[8];
+        ld8_value(zp_s, zq_s, i0, r);
+        if (degen) lds8(q_s + i0, qv);
+        const uint32_t x0 = static_cast<uint32_t>(x_first) + static_cast<uint32_t>(lane * 8);
+        const uint32_t o0 = static_cast<uint32_t>(p.offset), o1 = static_cast<uint32_t>(p.offset >> 32);
+        const uint32_t s0 = static_cast<uint32_t>(p.seed), s1 = static_cast<uint32_t>(p.seed >> 32);
+        const uint4 wa = philox4x32_10(make_uint4(static_cast<uint32_t>(g), 1u + (x0 >> 2), o0, o1), s0, s1);
+        const uint4 wb = philox4x32_10(make_uint4(static_cast<uint32_t>(g), 2u + (x0 >> 2), o0, o1), s0, s1);
+        const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+        float tk = -INFINITY;
+        int tx = INT_MAX;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float v = degen ? qv[e] : r[e];
+          if (i0 + e < len && v > 0.f) {
+            const float key = race_key(lg2(v), w[e]);
+            if (key > tk) {
+              tk = key;
+              tx = static_cast<int>(x0) + e;
+            }
+          }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) argmax_merge(tk, tx, __shfl_xor_sync(~0u, tk, o), __shfl_xor_sync(~0u, tx, o));
+        if (lane == 0) {
+          mine.m = tk;
+          mine.arg = tx;
+          mine.cap_own = 1;
+        }
+      }
+      cluster_exchange(cl, part, gath, stage, mine, C);
+      for (int k = 0; k < C; ++k)
+        if (gath[k].cap_own) term = gath[k].arg;
     }
   }
 
@@ -780,9 +866,9 @@ cudaError_t prepare_kernel_attributes() {
   return result[dev];
 }
 
-size_t header_bytes(int N) {
+size_t header_bytes(int N, int64_t chunk) {
   const size_t h = 16 + 2 * sizeof(Partial) + kMaxCluster * sizeof(Partial) + 64 * sizeof(float) + 8 * sizeof(int) +
-                   static_cast<size_t>(N) * 12;
+                   static_cast<size_t>(N) * 12 + static_cast<size_t>(chunk / kRaceBlock) * sizeof(float);
   return (h + 127) & ~static_cast<size_t>(127);
 }
 
@@ -792,9 +878,9 @@ RowGeometry row_geometry(const ScoreArgs& a) {
   RowGeometry geo{};
   const size_t es = a.dtype == DCD_BF16 ? 2 : 4;
   const size_t bpe = 2 * es + (a.q ? 4 : 0);
-  auto chunk_for = [&](int c) {
+  auto chunk_for = [&](int c) {  // slices hold whole 256-token race blocks
     const int64_t per = (a.V + c - 1) / c;
-    return (per + 7) & ~static_cast<int64_t>(7);
+    return (per + kRaceBlock - 1) / kRaceBlock * kRaceBlock;
   };
   int C = a.force_cluster;
   if (C <= 0) {
@@ -807,7 +893,7 @@ RowGeometry row_geometry(const ScoreArgs& a) {
   }
   geo.cluster = C;
   geo.chunk = chunk_for(C);
-  geo.smem = header_bytes(a.N) + static_cast<size_t>(geo.chunk) * bpe;
+  geo.smem = header_bytes(a.N, geo.chunk) + static_cast<size_t>(geo.chunk) * bpe;
   auto al16 = [](const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; };
   geo.bulk = !a.force_plain && al16(a.zp) && al16(a.zq) && (a.ld * static_cast<int64_t>(es)) % 16 == 0 &&
              (!a.q || (al16(a.q) && (a.ldq * 4) % 16 == 0));
@@ -826,7 +912,7 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   kp.cluster = geo.cluster;
   kp.chunk = static_cast<int32_t>(geo.chunk);
   kp.bulk = geo.bulk;
-  kp.data_offset = static_cast<int32_t>(header_bytes(a.N));
+  kp.data_offset = static_cast<int32_t>(header_bytes(a.N, geo.chunk));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(R * geo.cluster));
   cfg.blockDim = dim3(kThreads);
