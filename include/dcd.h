@@ -191,16 +191,16 @@ int dcd_verify_sample_noalloc(const dcd_shape* shape, const void* z_exp, const v
                               int32_t* cd_argmax, float* cd_lse, float* residual, dcd_stream_t stream);
 
 /*
- * dcd_score_rows with an explicit launch geometry, for tests and tuning: `cluster` is
- * the number of CTAs sharing one row (0 = automatic, else 1, 2, 4, 8 or 16) and
- * `plain_loads` = 1 stages rows with ordinary loads instead of bulk asynchronous
+ * dcd_score_rows with an explicit launch geometry, for tests and tuning: `stages` is
+ * the depth of each CTA's ring of shared-memory stages (0 = automatic, else 2 .. 8)
+ * and `plain_loads` = 1 stages rows with ordinary loads instead of bulk asynchronous
  * copies.  Results equal dcd_score_rows up to fp32 summation order.
  */
 int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
                       const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                       const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
                       int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
-                      dcd_stream_t stream, int cluster, int plain_loads);
+                      dcd_stream_t stream, int stages, int plain_loads);
 
 /*
  * Synchronises `stream`, then copies the device error word of `workspace` (the OR of

@@ -69,7 +69,7 @@ dcd::ScoreArgs make_args(const dcd_shape* s, const void* z_exp, const void* z_am
   a.cd_lse = cd_lse;
   a.rec = records(ws);
   a.err = error_word(ws);
-  a.force_cluster = 0;
+  a.force_stages = 0;
   a.force_plain = 0;
   return a;
 }
@@ -77,7 +77,7 @@ dcd::ScoreArgs make_args(const dcd_shape* s, const void* z_exp, const void* z_am
 int score_rows_impl(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
                     const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                     const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob, int32_t* cd_argmax,
-                    float* cd_lse, void* workspace, size_t workspace_bytes, cudaStream_t stream, int force_cluster,
+                    float* cd_lse, void* workspace, size_t workspace_bytes, cudaStream_t stream, int force_stages,
                     int force_plain) {
   const bool sampled_call = temperature != nullptr;
   if (!shape_ok(shape, sampled_call)) return DCD_ERR_INVALID_ARG;
@@ -90,10 +90,10 @@ int score_rows_impl(const dcd_shape* shape, const void* z_exp, const void* z_ama
   if (ws != DCD_OK) return ws;
   dcd::ScoreArgs a = make_args(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset,
                                cd_logprob, cd_argmax, cd_lse, workspace);
-  a.force_cluster = force_cluster;
+  a.force_stages = force_stages;
   a.force_plain = force_plain;
   const dcd::RowGeometry geo = dcd::row_geometry(a);
-  if (geo.smem > 227 * 1024) return DCD_ERR_UNSUPPORTED;
+  if (geo.smem > 227 * 1024 || geo.ctas_per_sm < 1) return DCD_ERR_UNSUPPORTED;
   return cuda_status(dcd::launch_score_rows(a, stream));
 }
 
@@ -184,16 +184,16 @@ const char* dcd_status_string(int status) {
 
 int dcd_version(void) { return kVersion; }
 
-// Test and tuning hook: dcd_score_rows with a forced cluster size and/or plain loads.
+// Test and tuning hook: dcd_score_rows with a forced ring depth and/or plain loads.
 int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
                       const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                       const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
                       int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
-                      int cluster, int plain_loads) {
-  if (cluster != 0 && (cluster < 1 || cluster > 16 || (cluster & (cluster - 1)) != 0)) return DCD_ERR_INVALID_ARG;
+                      int stages, int plain_loads) {
+  if (stages != 0 && (stages < 2 || stages > 8)) return DCD_ERR_INVALID_ARG;
   return score_rows_impl(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset, cd_logprob,
                          cd_argmax, cd_lse, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream),
-                         cluster, plain_loads);
+                         stages, plain_loads);
 }
 
 }  // extern "C"

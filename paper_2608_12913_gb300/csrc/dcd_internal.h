@@ -6,8 +6,9 @@
 
 namespace dcd {
 
-// Workspace layout: a 256-byte header (word 0 = device error bits), then one
-// RowRecord per row g = b * N + n.
+// Workspace layout: a 256-byte header (word 0 = device error bits, word 1 = the row
+// kernel's work counter, both zeroed at the start of every call), then one RowRecord per
+// row g = b * N + n.
 constexpr size_t kWorkspaceHeader = 256;
 
 struct RowRecord {
@@ -36,7 +37,7 @@ struct ScoreArgs {
   float* cd_lse;      // may be null
   RowRecord* rec;
   uint32_t* err;
-  int32_t force_cluster;  // 0 = automatic, else the cluster size to use (tests / tuning)
+  int32_t force_stages;   // 0 = automatic, else the ring depth to use (tests / tuning)
   int32_t force_plain;    // 1 = plain loads instead of bulk async copies
 };
 
@@ -48,12 +49,13 @@ cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_
 cudaError_t launch_terminal_residual(const ScoreArgs& a, const int32_t* accept_len, const int32_t* accept_path,
                                      const int32_t* bonus, float* residual, cudaStream_t stream);
 
-// Launch geometry the row kernel would use for a shape (exposed for diagnostics).
+// Launch geometry the row kernel would use for a call (exposed for diagnostics).
 struct RowGeometry {
-  int cluster;      // CTAs per row
-  int64_t chunk;    // vocabulary elements per CTA (multiple of 8)
-  size_t smem;      // dynamic shared memory per CTA
-  int bulk;         // 1 when rows are staged with bulk asynchronous copies
+  int stages;        // ring depth per CTA
+  int stage_tokens;  // vocabulary tokens per ring stage
+  size_t smem;       // dynamic shared memory per CTA
+  int ctas_per_sm;   // resident CTAs per SM
+  int bulk;          // 1 when rows are staged with bulk asynchronous copies
 };
 RowGeometry row_geometry(const ScoreArgs& a);
 

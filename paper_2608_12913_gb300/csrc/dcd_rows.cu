@@ -1,25 +1,33 @@
 // dcd_rows.cu -- the streaming kernels of the CD verification step on sm_103a.
 //
-// score_rows_kernel: one thread-block cluster per tree-node row g = b * N + n.  The
-//   row's vocabulary is split into `cluster` contiguous slices (whole blocks of 256
-//   tokens); each CTA stages its slice of z_p, z_q (and q for sampled non-leaf rows)
-//   in shared memory with bulk asynchronous copies, so HBM is read exactly once per
-//   row however many passes the row needs.  Passes over shared memory compute, in
-//   order: the expert max (only when beta > 0, for the plausibility set of Sec. 2.1),
-//   the CD score s' = (1 + alpha) z_p - alpha z_q with its max and argmax (Eq. 1; the
-//   two log-softmax shifts are constant per row and cancel in the normaliser), stored
-//   in place; the normaliser sum exp((s' - max) / T); then for sampled rows the
-//   sibling-rejection chain of Algorithm 1 (one residual pass per rejected child,
-//   r_j = max(0, r_{j-1} - q) / Z_j, in place) and the terminal draw, a two-level
-//   exponential race (a 256-token block by its mass, then a token of that block).
-//   Per-CTA partials are combined across the cluster through distributed shared
-//   memory; every CTA combines them in the same order, so all CTAs take identical
-//   decisions and run the same number of cluster barriers.
+// score_rows_kernel: a persistent grid (a few CTAs per SM).  Each CTA claims whole
+//   tree-node rows g = b * N + n from a work counter, in node-major order (every
+//   sequence's node 0, then every node 1, ...), so internal nodes -- the rows that
+//   may need extra passes -- come first and leaves last.  A row is streamed through
+//   a ring of 32 KB shared-memory stages filled by bulk
+//   asynchronous copies that complete on one mbarrier per stage; thread 0 refills a
+//   stage as soon as the block has consumed it, so a ring's worth of the row is
+//   always in flight.
+//   The "stats" pass computes the CD score s' = (1 + alpha) z_p - alpha z_q (Eq. 1;
+//   the two log-softmax shifts are constant per row and cancel in the normaliser)
+//   on the plausibility set P_beta of Sec. 2.1; every lane keeps an online max, a
+//   sum of 2^((s' - max) k2) (k2 = log2(e) / T) rescaled when its max grows, and
+//   its argmax, reduced over the block at the end of the row.  Rows whose terminal
+//   draw races over pi_CD itself (sampled leaves) also keep, per 256-token block,
+//   the block max and sum, i.e. the block masses of pi_CD.  With beta > 0 a "max"
+//   pass over z_p comes first.  Sampled rows then test their children in ascending node id (Algorithm 1
+//   on sibling lists); each rejection streams the row once more (z_p, z_q and q) to
+//   get the next residual's mass Z_j, recomputing r_j(x) = max(0, r_{j-1}(x) - q(x))
+//   / Z_j token by token from pi_CD(x), q(x) and the earlier Z's, so nothing per
+//   token is stored between passes.  Rows that take more than one pass are read with
+//   an L2 evict-last policy, so their later passes hit L2 and HBM is read once.  A
+//   node without an accepted child draws its terminal token by a two-level
+//   exponential race: a 256-token block by its mass, then a token of that block,
+//   whose 256 values are re-read directly.
 // tree_walk_kernel: one thread per sequence follows the accepted children.
 // terminal_residual_kernel: one block per sequence rebuilds the distribution its
 //   bonus token was drawn from (test output only).
 
-#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -31,22 +39,23 @@
 #include "dcd.h"
 #include "dcd_internal.h"
 
-namespace cg = cooperative_groups;
-
 namespace dcd {
 namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kMaxCluster = 16;
-constexpr size_t kSmemBudget = 64 * 1024 + 1024;  // data bytes per CTA the automatic geometry aims for
+constexpr int kStageBytes = 32 * 1024;            // bytes per ring stage
+constexpr int kRaceBlock = 256;                   // tokens per block of the two-level terminal race
+constexpr int kMaxStages = 8;
 constexpr size_t kSmemMax = 227 * 1024;
+constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr long long kWaitCycles = 4000000000ll;  // about two seconds at the boost clock
-constexpr int kRaceBlock = 256;                  // tokens per block of the two-level terminal race
 constexpr float kLog2e = 1.4426950408889634f;
 
+enum PassKind { kPassMax = 0, kPassStats = 1, kPassRes = 2 };
+
 // ------------------------------------------------------------------------------------------
-// PTX wrappers: mbarrier and bulk asynchronous global->shared copies.
+// PTX wrappers: mbarrier, L2 cache policies and bulk asynchronous global->shared copies.
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -60,15 +69,11 @@ __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile(
       "{\n\t.reg .b64 st;\n\t"
-      "mbarrier.arrive.shared::cta.b64 st, [%0];\n\t}" ::"r"(smem_addr(bar))
+      "mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}" ::"r"(smem_addr(bar)),
+      "r"(bytes)
       : "memory");
 }
 
@@ -93,12 +98,36 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
   return true;
 }
 
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
   asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_addr(dst)),
-      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], "
+      "%4;" ::"r"(smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
       : "memory");
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float lg2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -116,30 +145,36 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1
   return c;
 }
 
+__device__ __forceinline__ uint4 philox_block(uint64_t seed, uint64_t off, uint32_t c0, uint32_t c1) {
+  return philox4x32_10(make_uint4(c0, c1, static_cast<uint32_t>(off), static_cast<uint32_t>(off >> 32)),
+                       static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
+}
+
+__device__ __forceinline__ uint32_t word_of(const uint4& w, int i) {
+  return i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w;
+}
+
 // 32-bit word -> uniform in (0, 1): ((w >> 9) + 1/2) 2^-23, exact in fp32.
 __device__ __forceinline__ float u01(uint32_t w) {
   return (__uint2float_rn(w >> 9) + 0.5f) * 1.1920928955078125e-07f;
 }
 
-__device__ __forceinline__ float accept_uniform(uint64_t seed, uint64_t off, uint32_t G) {
-  const uint4 w = philox4x32_10(make_uint4(G, 0u, (uint32_t)off, (uint32_t)(off >> 32)), (uint32_t)seed,
-                                (uint32_t)(seed >> 32));
-  return u01(w.x);
+// Race key in log2 units: log2 r - log2(-log2 u) orders tokens exactly as ln r - ln(-ln u)
+// (the two differ by a positive factor and a constant).
+__device__ __forceinline__ float race_key(float log2_mass, uint32_t word) {
+  return log2_mass - lg2(-lg2(u01(word)));
 }
 
 // ------------------------------------------------------------------------------------------
-// Shared-memory element access.  Slices are read 8 tokens at a time (16 B of bf16 or 32 B of
-// fp32).  Sampled rows overwrite their logits in place with fp32 values: for fp32 input the
-// value takes the z_p slot; for bf16 input its low half goes to the z_p slot and its high
-// half to the z_q slot of the same token, so no token's slots are shared with another's.
-__device__ __forceinline__ void lds8(const float* p, float v[8]) {
+// Element access: 8 consecutive tokens as fp32 (16 B of bf16 or 32 B of fp32).
+__device__ __forceinline__ void ld8(const float* p, float v[8]) {
   const float4 a = reinterpret_cast<const float4*>(p)[0];
   const float4 b = reinterpret_cast<const float4*>(p)[1];
   v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
   v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
 }
 
-__device__ __forceinline__ void lds8(const __nv_bfloat16* p, float v[8]) {
+__device__ __forceinline__ void ld8(const __nv_bfloat16* p, float v[8]) {
   const uint4 a = *reinterpret_cast<const uint4*>(p);
   v[0] = __uint_as_float(a.x << 16); v[1] = __uint_as_float(a.x & 0xffff0000u);
   v[2] = __uint_as_float(a.y << 16); v[3] = __uint_as_float(a.y & 0xffff0000u);
@@ -147,46 +182,11 @@ __device__ __forceinline__ void lds8(const __nv_bfloat16* p, float v[8]) {
   v[6] = __uint_as_float(a.w << 16); v[7] = __uint_as_float(a.w & 0xffff0000u);
 }
 
-__device__ __forceinline__ void st8_value(float* zp, float* /*zq*/, int i0, const float v[8]) {
-  reinterpret_cast<float4*>(zp + i0)[0] = make_float4(v[0], v[1], v[2], v[3]);
-  reinterpret_cast<float4*>(zp + i0)[1] = make_float4(v[4], v[5], v[6], v[7]);
-}
-
-__device__ __forceinline__ void st8_value(__nv_bfloat16* zp, __nv_bfloat16* zq, int i0, const float v[8]) {
-  uint32_t w[8];
-#pragma unroll
-  for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(v[e]);
-  *reinterpret_cast<uint4*>(zp + i0) = make_uint4(__byte_perm(w[0], w[1], 0x5410), __byte_perm(w[2], w[3], 0x5410),
-                                                 __byte_perm(w[4], w[5], 0x5410), __byte_perm(w[6], w[7], 0x5410));
-  *reinterpret_cast<uint4*>(zq + i0) = make_uint4(__byte_perm(w[0], w[1], 0x7632), __byte_perm(w[2], w[3], 0x7632),
-                                                 __byte_perm(w[4], w[5], 0x7632), __byte_perm(w[6], w[7], 0x7632));
-}
-
-__device__ __forceinline__ void ld8_value(const float* zp, const float* /*zq*/, int i0, float v[8]) {
-  lds8(zp + i0, v);
-}
-
-__device__ __forceinline__ void ld8_value(const __nv_bfloat16* zp, const __nv_bfloat16* zq, int i0, float v[8]) {
-  const uint4 lo = *reinterpret_cast<const uint4*>(zp + i0);
-  const uint4 hi = *reinterpret_cast<const uint4*>(zq + i0);
-  const uint32_t l[4] = {lo.x, lo.y, lo.z, lo.w}, h[4] = {hi.x, hi.y, hi.z, hi.w};
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    v[2 * k] = __uint_as_float(__byte_perm(l[k], h[k], 0x5410));
-    v[2 * k + 1] = __uint_as_float(__byte_perm(l[k], h[k], 0x7632));
-  }
-}
-
-__device__ __forceinline__ float ld1_value(const float* zp, const float* /*zq*/, int i) { return zp[i]; }
-
-__device__ __forceinline__ float ld1_value(const __nv_bfloat16* zp, const __nv_bfloat16* zq, int i) {
-  const uint32_t lo = reinterpret_cast<const uint16_t*>(zp)[i];
-  const uint32_t hi = reinterpret_cast<const uint16_t*>(zq)[i];
-  return __uint_as_float((hi << 16) | lo);
-}
+__device__ __forceinline__ float ld1(const float* p, int64_t i) { return p[i]; }
+__device__ __forceinline__ float ld1(const __nv_bfloat16* p, int64_t i) { return __bfloat162float(p[i]); }
 
 // ------------------------------------------------------------------------------------------
-// Block reductions (every thread gets the result).
+// Reductions.
 __device__ __forceinline__ void argmax_merge(float& v, int& i, float v2, int i2) {
   if (v2 > v || (v2 == v && i2 < i)) {
     v = v2;
@@ -194,9 +194,26 @@ __device__ __forceinline__ void argmax_merge(float& v, int& i, float v2, int i2)
   }
 }
 
-__device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int* redi) {
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(~0u, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(~0u, v, o));
+  return v;
+}
+
+__device__ __forceinline__ void warp_argmax(float& v, int& i) {
 #pragma unroll
   for (int o = 16; o; o >>= 1) argmax_merge(v, i, __shfl_xor_sync(~0u, v, o), __shfl_xor_sync(~0u, i, o));
+}
+
+// Block reductions: every thread gets the result; the scratch is free again on return.
+__device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int* redi) {
+  warp_argmax(v, i);
   if ((threadIdx.x & 31) == 0) {
     redf[threadIdx.x >> 5] = v;
     redi[threadIdx.x >> 5] = i;
@@ -210,8 +227,7 @@ __device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int*
 }
 
 __device__ __forceinline__ float block_sum(float v, float* redf) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(~0u, v, o);
+  v = warp_sum(v);
   if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
   __syncthreads();
   float s = 0.f;
@@ -222,8 +238,7 @@ __device__ __forceinline__ float block_sum(float v, float* redf) {
 }
 
 __device__ __forceinline__ float block_max(float v, float* redf) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(~0u, v, o));
+  v = warp_max(v);
   if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
   __syncthreads();
   float s = -INFINITY;
@@ -234,512 +249,492 @@ __device__ __forceinline__ float block_max(float v, float* redf) {
 }
 
 // ------------------------------------------------------------------------------------------
-// Cluster exchange: each CTA publishes one Partial; after the cluster barrier every CTA
-// gathers all of them from distributed shared memory.  Partial slots alternate between two
-// buffers: a CTA rewrites a buffer only after the next barrier, which its peers pass only
-// once they have finished reading it.
-struct Partial {
-  float m;          // max (score or race key)
-  float s;          // sum
-  int32_t arg;      // token id attaining m
-  float cap_r;      // value captured at the next candidate token (owner CTA only)
-  float cap_q;      // q at that token (owner CTA only)
-  int32_t cap_own;  // 1 in the CTA whose slice holds the candidate token
-  uint32_t status;  // DCD_DEVERR_* bits
-  int32_t pad;
-};
-
-__device__ __forceinline__ Partial neutral_partial() {
-  Partial p;
-  p.m = -INFINITY;
-  p.s = 0.f;
-  p.arg = INT_MAX;
-  p.cap_r = 0.f;
-  p.cap_q = 0.f;
-  p.cap_own = 0;
-  p.status = 0u;
-  p.pad = 0;
-  return p;
-}
-
-__device__ __forceinline__ void cluster_exchange(cg::cluster_group& cl, Partial* part, Partial* gath, int& stage,
-                                                 const Partial& mine, int C) {
-  Partial* slot = &part[stage & 1];
-  ++stage;
-  if (threadIdx.x == 0) *slot = mine;
-  cl.sync();
-  if (threadIdx.x < C) gath[threadIdx.x] = *cl.map_shared_rank(slot, threadIdx.x);
-  __syncthreads();
-}
-
-struct KParams {
+struct SParams {
   ScoreArgs a;
-  int32_t cluster;
-  int32_t chunk;   // tokens per CTA (multiple of kRaceBlock)
-  int32_t bulk;    // 1: bulk asynchronous copies, 0: plain loads
-  int32_t data_offset;
+  int32_t nst;           // ring depth (stages of kStageBytes)
+  int32_t tok_a;         // tokens per stage in the max and stats passes (z_p, z_q)
+  int32_t tok_r;         // tokens per stage in residual passes (z_p, z_q, q)
+  int32_t bulk;          // 1: bulk asynchronous copies, 0: plain loads
+  int32_t nblk;          // race blocks per row, ceil(V / 256)
+  int32_t meta_offset;   // byte offsets into dynamic shared memory
+  int32_t blk_offset;
+  int32_t stage_offset;
+  uint32_t* work;        // row counter, zeroed before the launch
 };
 
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
+// Row state shared by the block (written by one thread, read after a barrier).
+struct RowShared {
+  int32_t next;      // the next claimed work item
+  int32_t m;         // children of the row's node
+  uint32_t status;   // DCD_DEVERR_* bits
+  int32_t accept;    // outcome of the current sibling test
+  int32_t term;      // terminal token
+  int32_t pad[3];
+};
 
-__device__ __forceinline__ float lg2(float x) {
-  float y;
-  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
+template <typename TIn>
+struct Stage {
+  TIn* zp;
+  TIn* zq;
+  float* q;
+};
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(~0u, v, o);
-  return v;
-}
-
-// log2 of a Gumbel-race divisor: key = log2 r - log2(-log2 u) orders tokens exactly as
-// ln r - ln(-ln u) does (the two differ by a positive factor and a constant).
-__device__ __forceinline__ float race_key(float log2_mass, uint32_t word) {
-  return log2_mass - lg2(-lg2(u01(word)));
-}
-
-__device__ __forceinline__ uint32_t philox_word(uint64_t seed, uint64_t off, uint32_t c0, uint32_t c1, int word) {
-  const uint4 w = philox4x32_10(make_uint4(c0, c1, (uint32_t)off, (uint32_t)(off >> 32)), (uint32_t)seed,
-                                (uint32_t)(seed >> 32));
-  return word == 0 ? w.x : word == 1 ? w.y : word == 2 ? w.z : w.w;
+// A stage holds `tok` tokens of z_p, then of z_q, then (residual passes) of q.
+template <typename TIn>
+__device__ __forceinline__ Stage<TIn> stage_at(unsigned char* base, int s, int tok) {
+  Stage<TIn> st;
+  st.zp = reinterpret_cast<TIn*>(base + static_cast<size_t>(s) * kStageBytes);
+  st.zq = st.zp + tok;
+  st.q = reinterpret_cast<float*>(st.zq + tok);
+  return st;
 }
 
 // ------------------------------------------------------------------------------------------
 template <typename TIn>
-__global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_constant__ KParams kp) {
-  const ScoreArgs& p = kp.a;
-  cg::cluster_group cl = cg::this_cluster();
-  const int C = kp.cluster;
-  const int rank = static_cast<int>(cl.block_rank());
-  const int64_t g = static_cast<int64_t>(blockIdx.x) / C;
-  const int N = p.N;
-  const int b = static_cast<int>(g / N), n = static_cast<int>(g % N);
+__global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_constant__ SParams sp) {
+  const ScoreArgs& p = sp.a;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int N = p.N;
+  const int64_t V = p.V;
+  const int R = p.B * N;
+  const int nch_a = static_cast<int>((V + sp.tok_a - 1) / sp.tok_a);  // chunks of a max / stats pass
+  const int nch_r = static_cast<int>((V + sp.tok_r - 1) / sp.tok_r);  // chunks of a residual pass
 
   extern __shared__ __align__(128) unsigned char smem[];
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
-  Partial* part = reinterpret_cast<Partial*>(smem + 16);
-  Partial* gath = part + 2;
-  float* redf = reinterpret_cast<float*>(gath + kMaxCluster);
-  int* redi = reinterpret_cast<int*>(redf + 32);
-  int* meta = redi + 32;  // [0] child count, [1] status bits
-  int* kids = meta + 8;
-  int* ktok = kids + N;
-  float* ksv = reinterpret_cast<float*>(ktok + N);
-  float* blk = ksv + N;  // per 256-token block masses of this slice
-  TIn* zp_s = reinterpret_cast<TIn*>(smem + kp.data_offset);
-  TIn* zq_s = zp_s + kp.chunk;
-  float* q_s = reinterpret_cast<float*>(zq_s + kp.chunk);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem);             // [kMaxStages]
+  float* redf = reinterpret_cast<float*>(smem + 8 * kMaxStages);  // [32]
+  int* redi = reinterpret_cast<int*>(redf + 32);                  // [32]
+  RowShared* rs = reinterpret_cast<RowShared*>(smem + sp.meta_offset);
+  int* kids = reinterpret_cast<int*>(rs + 1);                     // [N] children, ascending id
+  int* ktok = kids + N;                                           // [N] their tokens
+  float* czp = reinterpret_cast<float*>(ktok + N);                // [N] z_p at those tokens
+  float* czq = czp + N;                                           // [N] z_q at those tokens
+  float* cq = czq + N;                                            // [N] q at those tokens
+  float* invZ = cq + N;                                           // [N] 1/Z_j (0 marks Z_j = 0)
+  float* bmax = reinterpret_cast<float*>(smem + sp.blk_offset);   // [nblk] block max of s'
+  float* bsum = bmax + sp.nblk;                                   // [nblk] block sums
+  float* bres = bsum + sp.nblk;                                   // [nblk] final residual block masses
+  float* bq = bres + sp.nblk;                                     // [nblk] block masses of q
+  unsigned char* ring = smem + sp.stage_offset;
 
-  const int64_t lo = static_cast<int64_t>(rank) * kp.chunk;
-  const int64_t hi = lo + kp.chunk < p.V ? lo + kp.chunk : p.V;
-  const int len = hi > lo ? static_cast<int>(hi - lo) : 0;
-  const TIn* zp_g = static_cast<const TIn*>(p.zp) + g * p.ld + lo;
-  const TIn* zq_g = static_cast<const TIn*>(p.zq) + g * p.ld + lo;
-
-  const float alpha = p.alpha[b];
-  const float beta = p.beta ? p.beta[b] : 0.f;
-  const float T = p.temp ? p.temp[b] : 0.f;
-  const bool sampled = T > 0.f;
-  const float invT = sampled ? 1.f / T : 1.f;
-  const float k2 = kLog2e * invT;  // exp(x / T) = 2^(x * k2)
-
-  if (g == 0 && rank == 0 && tid == 0) *p.err = 0u;
-
-  // ---- stage the slice: bulk copies of z_p / z_q first, q once the children are known
-  const uint32_t zbulk = kp.bulk ? static_cast<uint32_t>((len * static_cast<int>(sizeof(TIn))) & ~15) : 0u;
   if (tid == 0) {
-    mbar_init(bar, 1);
+    for (int s = 0; s < sp.nst; ++s) mbar_init(&full[s], 1);
     fence_mbar_init();
-    if (zbulk) {
-      mbar_expect_tx(bar, 2u * zbulk);
-      bulk_g2s(zp_s, zp_g, zbulk, bar);
-      bulk_g2s(zq_s, zq_g, zbulk, bar);
-    }
-  }
-  if (warp == 0) {
-    // children of node n in ascending id, and the checks of this row's own node
-    const int32_t* par = p.parents + static_cast<int64_t>(b) * N;
-    const int32_t* tok = p.tokens + static_cast<int64_t>(b) * N;
-    int count = 0;
-    for (int base = n + 1; base < N; base += 32) {
-      const int c = base + lane;
-      const bool is = c < N && par[c] == n;
-      const unsigned msk = __ballot_sync(~0u, is);
-      if (is) {
-        const int pos = count + __popc(msk & ((1u << lane) - 1u));
-        kids[pos] = c;
-        ktok[pos] = tok[c];
-      }
-      count += __popc(msk);
-    }
-    if (lane == 0) {
-      uint32_t st = 0u;
-      const int pp = par[n];
-      if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
-      if (n > 0) {
-        const int t = tok[n];
-        if (t < 0 || t >= p.V) st |= DCD_DEVERR_BAD_TOKEN;
-      }
-      if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
-        st |= DCD_DEVERR_BAD_PARAM;
-      meta[0] = count;
-      meta[1] = static_cast<int>(st);
-    }
+    rs->next = static_cast<int32_t>(atomicAdd(sp.work, 1u));
   }
   __syncthreads();
-  const int m = meta[0];
-  const bool need_q = sampled && m > 0 && p.q != nullptr;
-  const float* q_g = need_q ? p.q + g * p.ldq + lo : nullptr;
-  const uint32_t qbulk = (kp.bulk && need_q) ? static_cast<uint32_t>((len * 4) & ~15) : 0u;
-  if (tid == 0) {
-    if (qbulk) {
-      mbar_expect_tx(bar, qbulk);
-      bulk_g2s(q_s, q_g, qbulk, bar);
-    }
-    mbar_arrive(bar);
-  }
-  {  // plain loads: the whole slice without bulk copies, else only the ragged tail
-    const int zfirst = static_cast<int>(zbulk / sizeof(TIn));
-    for (int i = zfirst + tid; i < len; i += kThreads) {
-      zp_s[i] = zp_g[i];
-      zq_s[i] = zq_g[i];
-    }
-    if (need_q) {
-      const int qfirst = static_cast<int>(qbulk / 4);
-      for (int i = qfirst + tid; i < len; i += kThreads) q_s[i] = q_g[i];
-    }
-  }
-  if (!mbar_wait_bounded(bar, 0)) {
-    atomicOr(reinterpret_cast<unsigned*>(&meta[1]), DCD_DEVERR_TIMEOUT);
-    mbar_wait_bounded(bar, 0);  // give copies still in flight a second bounded chance
-  }
-  __syncthreads();
+  const uint64_t pol_last = l2_policy_evict_last();
+  const uint64_t pol_first = l2_policy_evict_first();
+  uint32_t seq = 0;  // ring items consumed by this CTA so far (identical in every thread)
 
-  // Loops run over 8-token groups; a warp's 32 groups are one 256-token race block, and the
-  // group count is rounded up to whole warps so every branch on `grp < ngw` is warp-uniform.
-  const int ngw = (((len + 7) >> 3) + 31) & ~31;
-  const bool masked = beta > 0.f;
-  const float logb = masked ? logf(beta) : -INFINITY;
-  const float c1 = 1.f + alpha;
-  int stage = 0;
-  Partial mine = neutral_partial();
-  uint32_t status = 0u;
+  for (;;) {
+    const int item = rs->next;
+    __syncthreads();  // every thread has read the claim before thread 0 replaces it
+    if (item >= R) break;
+    if (tid == 0) rs->next = static_cast<int32_t>(atomicAdd(sp.work, 1u));  // used by the next row
+    const int b = item % p.B, n = item / p.B;  // node-major order
+    const int64_t g = static_cast<int64_t>(b) * N + n;
+    const float alpha = p.alpha[b];
+    const float beta = p.beta ? p.beta[b] : 0.f;
+    const float T = p.temp ? p.temp[b] : 0.f;
+    const bool sampled = T > 0.f && p.q != nullptr;
+    const bool masked = beta > 0.f;
+    const float invT = T > 0.f ? 1.f / T : 1.f;
+    const float k2 = kLog2e * invT;  // exp(x / T) = 2^(x * k2)
+    const float c1 = 1.f + alpha;
+    const float logb = masked ? logf(beta) : -INFINITY;
+    const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
+    const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
+    const float* q_row = sampled ? p.q + g * p.ldq : nullptr;
 
-  // ---- pass A (beta > 0): the expert max, for P_beta = {x : z_p(x) - max z_p >= log beta}
-  float Mp = 0.f;
-  if (masked) {
-    float lm = -INFINITY;
-    for (int base = 0; base < ngw; base += kThreads) {
-      const int grp = base + tid;
-      if (grp >= ngw) continue;
-      const int i0 = grp << 3;
-      float zp[8];
-      lds8(zp_s + i0, zp);
-#pragma unroll
-      for (int e = 0; e < 8; ++e)
-        if (i0 + e < len) lm = fmaxf(lm, zp[e]);
-    }
-    lm = block_max(lm, redf);
-    mine.m = lm;
-    cluster_exchange(cl, part, gath, stage, mine, C);
-    Mp = -INFINITY;
-    for (int k = 0; k < C; ++k) Mp = fmaxf(Mp, gath[k].m);
-  }
-
-  // ---- pass B: CD score s' = (1 + alpha) z_p - alpha z_q on P_beta (-inf elsewhere), its max and
-  // argmax; s' overwrites the slice in place as fp32
-  float best = -INFINITY;
-  int barg = INT_MAX;
-  for (int base = 0; base < ngw; base += kThreads) {
-    const int grp = base + tid;
-    if (grp >= ngw) continue;
-    const int i0 = grp << 3;
-    float zp[8], zq[8], sv[8];
-    lds8(zp_s + i0, zp);
-    lds8(zq_s + i0, zq);
-    float gm = -INFINITY;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const bool in = (i0 + e < len) && (!masked || (zp[e] - Mp >= logb));
-      sv[e] = in ? fmaf(c1, zp[e], -alpha * zq[e]) : -INFINITY;
-      gm = fmaxf(gm, sv[e]);
-    }
-    if (gm > best) {
-      best = gm;
-#pragma unroll
-      for (int e = 7; e >= 0; --e)
-        if (sv[e] == gm) barg = static_cast<int>(lo) + i0 + e;
-    }
-    st8_value(zp_s, zq_s, i0, sv);
-  }
-  block_argmax(best, barg, redf, redi);  // ends with __syncthreads: every s' is stored
-  const float m_cta = best;
-  // children's scores, read by the CTA whose slice holds the token
-  for (int k = tid; k < m; k += kThreads) {
-    const int t = ktok[k];
-    if (t >= lo && t < hi) ksv[k] = ld1_value(zp_s, zq_s, t - static_cast<int>(lo));
-  }
-  __syncthreads();  // the captures above finish before pass C rewrites the slice
-
-  // ---- pass C: normaliser sum 2^((s' - m_cta) k2); sampled rows keep e(x) in place, and leaf rows
-  // (whose terminal draw races over pi_CD itself) keep the 256-token block masses
-  const bool leaf_race = sampled && m == 0;
-  float ssum = 0.f;
-  if (m_cta > -INFINITY) {
-    const float mk2 = m_cta * k2;
-    for (int base = 0; base < ngw; base += kThreads) {
-      const int grp = base + tid;
-      if (grp >= ngw) continue;
-      const int i0 = grp << 3;
-      float sv[8];
-      ld8_value(zp_s, zq_s, i0, sv);
-      float part = 0.f;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        sv[e] = ex2(fmaf(sv[e], k2, -mk2));
-        part += sv[e];
+    // ---- ring items of this row: [max pass if beta > 0] [stats pass] [a residual pass per
+    // rejected child]; thread 0 keeps up to nst items in flight, never past `limit`
+    const int nknown = (masked ? 2 : 1) * nch_a;
+    const uint32_t seq0 = seq;
+    auto pass_of = [&](int L) -> int {
+      if (L < nknown) return (masked && L < nch_a) ? kPassMax : kPassStats;
+      return kPassRes;
+    };
+    // token range and stage layout of item L
+    auto chunk_of = [&](int L, int64_t& x0, int& clen, int& tok) {
+      const bool res = L >= nknown;
+      tok = res ? sp.tok_r : sp.tok_a;
+      const int c = res ? (L - nknown) % nch_r : L % nch_a;
+      x0 = static_cast<int64_t>(c) * tok;
+      clen = static_cast<int>((V - x0) < tok ? (V - x0) : tok);
+    };
+    auto issue = [&](int L, uint64_t pol) {  // thread 0 only
+      const uint32_t sq = seq0 + static_cast<uint32_t>(L);
+      const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
+      int64_t x0;
+      int clen, tok;
+      chunk_of(L, x0, clen, tok);
+      const Stage<TIn> st = stage_at<TIn>(ring, s, tok);
+      const int kind = pass_of(L);
+      uint32_t zb = 0, qb = 0;
+      if (sp.bulk) {
+        zb = static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u;
+        qb = kind == kPassRes ? static_cast<uint32_t>(clen * 4) & ~15u : 0u;
       }
-      ssum += part;
-      if (sampled) st8_value(zp_s, zq_s, i0, sv);
-      if (leaf_race) {
-        const float bs = warp_sum(part);
-        if (lane == 0) blk[grp >> 5] = bs;
+      mbar_arrive_expect_tx(&full[s], (kind == kPassMax ? zb : 2u * zb) + qb);
+      if (zb) {
+        bulk_g2s(st.zp, zp_row + x0, zb, &full[s], pol);
+        if (kind != kPassMax) bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pol);
+      }
+      if (qb) bulk_g2s(st.q, q_row + x0, qb, &full[s], pol);
+    };
+
+    // thread 0 starts the row's stream at once (rows that may take more than one pass are
+    // kept in L2); warp 1 meanwhile finds the children of node n and checks this row's node
+    uint64_t pol = (masked || sampled) ? pol_last : pol_first;
+    if (tid == 0) {
+      const int first = nknown < sp.nst ? nknown : sp.nst;
+      for (int L = 0; L < first; ++L) issue(L, pol);
+    }
+    if (warp == 1) {
+      const int32_t* par = p.parents + static_cast<int64_t>(b) * N;
+      const int32_t* tok = p.tokens + static_cast<int64_t>(b) * N;
+      int count = 0;
+      for (int base = n + 1; base < N; base += 32) {
+        const int c = base + lane;
+        const bool is = c < N && par[c] == n;
+        const unsigned msk = __ballot_sync(~0u, is);
+        if (is) {
+          const int pos = count + __popc(msk & ((1u << lane) - 1u));
+          kids[pos] = c;
+          ktok[pos] = tok[c];
+        }
+        count += __popc(msk);
+      }
+      if (lane == 0) {
+        uint32_t st = 0u;
+        const int pp = par[n];
+        if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
+        if (n > 0) {
+          const int t = tok[n];
+          if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
+        }
+        if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
+          st |= DCD_DEVERR_BAD_PARAM;
+        rs->m = count;
+        rs->status = st;
       }
     }
-  } else if (sampled) {
-    const float zero[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int grp = tid; grp < ngw; grp += kThreads) st8_value(zp_s, zq_s, grp << 3, zero);
-    for (int t = tid; t < (ngw >> 5); t += kThreads) blk[t] = 0.f;
-  }
-  const float s_cta = block_sum(ssum, redf);  // ends with __syncthreads
-
-  mine = neutral_partial();
-  mine.m = m_cta;
-  mine.s = s_cta;
-  mine.arg = barg;
-  if (sampled && m > 0 && tid == 0) {
-    const int t = ktok[0];
-    if (t >= lo && t < hi) {
-      mine.cap_own = 1;
-      mine.cap_r = ld1_value(zp_s, zq_s, t - static_cast<int>(lo));
-      mine.cap_q = q_s[t - static_cast<int>(lo)];
-    }
-  }
-  if (tid == 0) mine.status = static_cast<uint32_t>(meta[1]);
-  cluster_exchange(cl, part, gath, stage, mine, C);
-
-  float M = -INFINITY;
-  for (int k = 0; k < C; ++k) M = fmaxf(M, gath[k].m);
-  int arg = INT_MAX;
-  float S = 0.f;
-  float rt = 0.f, qt = 0.f;
-  for (int k = 0; k < C; ++k) {
-    status |= gath[k].status;
-    if (gath[k].m == M && arg == INT_MAX) arg = gath[k].arg;
-    if (gath[k].m > -INFINITY) S += gath[k].s * exp2f((gath[k].m - M) * k2);
-  }
-  if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
-  for (int k = 0; k < C; ++k)
-    if (gath[k].cap_own) {
-      rt = gath[k].cap_r * (exp2f((gath[k].m - M) * k2) / S);
-      qt = gath[k].cap_q;
-    }
-  const float logS = logf(S);
-
-  // ---- outputs of the Eq. 1 target
-  if (rank == 0 && tid == 0) {
-    if (p.cd_argmax) p.cd_argmax[g] = arg;
-    if (p.cd_lse) p.cd_lse[g] = M * invT + logS;
-    if (n == 0 && p.cd_logprob) p.cd_logprob[g] = 0.f;
-  }
-  if (p.cd_logprob) {
-    for (int k = tid; k < m; k += kThreads) {
-      const int t = ktok[k];
-      if (t >= lo && t < hi)
-        p.cd_logprob[static_cast<int64_t>(b) * N + kids[k]] =
-            ksv[k] > -INFINITY ? (ksv[k] - M) * invT - logS : -INFINITY;
-    }
-  }
-
-  int acc = -1, term = -1;
-  if (!sampled) {
-    // ---- greedy rule
-    for (int k = 0; k < m; ++k)
-      if (ktok[k] == arg) {
-        acc = kids[k];
-        break;
+    __syncthreads();
+    const int m = rs->m;
+    pol = (masked || (sampled && m > 0)) ? pol_last : pol_first;
+    // values at the children's tokens: the loads are issued now and consumed after the stats pass
+    float pzp = 0.f, pzq = 0.f, pq = 0.f;
+    if (tid < m) {
+      const int t = ktok[tid];
+      if (t >= 0 && t < V) {
+        pzp = ld1(zp_row, t);
+        pzq = ld1(zq_row, t);
+        if (sampled) pq = q_row[t];
       }
-    if (acc < 0) term = arg;
-  } else {
-    // ---- sampled rule: sibling-rejection chain over the slice, then the terminal race if needed
-    const float scale_me = m_cta > -INFINITY ? exp2f((m_cta - M) * k2) / S : 0.f;
-    float invZ = 0.f;
-    bool degen = false;
-    for (int j = 0; j < m; ++j) {
-      const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[j]);
-      const float u = accept_uniform(p.seed, p.offset, G);
-      const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
-      if (u <= ratio) {
-        acc = kids[j];
-        break;
+    }
+
+    int limit = nknown;  // items planned so far
+    int L = 0;           // next item to consume
+    bool timed_out = false;
+
+    // Consumes `count` items: waits for each stage, fills a ragged or unaligned remainder with
+    // plain loads, hands the stage to `body`, releases the stage and refills it.
+    auto run_items = [&](int count, auto&& body) {
+      for (int it = 0; it < count; ++it, ++L) {
+        const uint32_t sq = seq0 + static_cast<uint32_t>(L);
+        const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
+        const uint32_t parity = (sq / static_cast<uint32_t>(sp.nst)) & 1u;
+        int64_t x0;
+        int clen, tok;
+        chunk_of(L, x0, clen, tok);
+        const Stage<TIn> st = stage_at<TIn>(ring, s, tok);
+        const int kind = pass_of(L);
+        if (!mbar_wait_bounded(&full[s], parity)) timed_out = true;
+        const int zfirst =
+            sp.bulk ? ((clen * static_cast<int>(sizeof(TIn))) & ~15) / static_cast<int>(sizeof(TIn)) : 0;
+        const int qfirst = sp.bulk ? ((clen * 4) & ~15) / 4 : 0;
+        if (zfirst < clen || (kind == kPassRes && qfirst < clen)) {
+          for (int i = zfirst + tid; i < clen; i += kThreads) {
+            st.zp[i] = zp_row[x0 + i];
+            if (kind != kPassMax) st.zq[i] = zq_row[x0 + i];
+          }
+          if (kind == kPassRes)
+            for (int i = qfirst + tid; i < clen; i += kThreads) st.q[i] = q_row[x0 + i];
+          __syncthreads();
+        }
+        body(st, x0, clen);
+        __syncthreads();
+        if (tid == 0 && L + sp.nst < limit) issue(L + sp.nst, pol);
       }
-      // rejected: r_{j+1} = max(0, r_j - q) / Z, written over the slice; the last residual also
-      // records its block masses for the terminal race
-      const bool last = j == m - 1;
-      float zsum = 0.f;
-      for (int base = 0; base < ngw; base += kThreads) {
-        const int grp = base + tid;
-        if (grp >= ngw) continue;
-        const int i0 = grp << 3;
-        float r[8], qv[8];
-        ld8_value(zp_s, zq_s, i0, r);
-        lds8(q_s + i0, qv);
-        float part = 0.f;
+    };
+
+    // ---- pass A (beta > 0): the expert max, for P_beta = {x : z_p(x) - max z_p >= log beta}
+    float Mp = 0.f;
+    if (masked) {
+      float lm = -INFINITY;
+      run_items(nch_a, [&](const Stage<TIn>& st, int64_t, int clen) {
+        for (int i0 = tid * 8; i0 < clen; i0 += kThreads * 8) {
+          float zp[8];
+          ld8(st.zp + i0, zp);
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            if (i0 + e < clen) lm = fmaxf(lm, zp[e]);
+        }
+      });
+      Mp = block_max(lm, redf);
+    }
+
+    // ---- pass B: the CD score s' on P_beta.  Each lane keeps an online max, a sum of
+    // 2^((s' - max) k2) rescaled whenever its max grows, and its argmax.  Rows that end in a
+    // race over pi_CD itself (sampled leaves) also record, per 256-token block (one warp, 8
+    // tokens a lane), the block's max and its sum relative to that max.
+    const bool leaf_race = sampled && m == 0;
+    float lmax = -INFINITY, lsum = 0.f;
+    int larg = INT_MAX;
+    run_items(nch_a, [&](const Stage<TIn>& st, int64_t x0, int clen) {
+      for (int kb = warp; kb * kRaceBlock < sp.tok_a; kb += kWarps) {
+        if (kb * kRaceBlock >= clen) break;  // warp-uniform
+        const int i0 = kb * kRaceBlock + lane * 8;
+        float zp[8], zq[8], sv[8];
+        ld8(st.zp + i0, zp);
+        ld8(st.zq + i0, zq);
+        float gm = -INFINITY;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float prev = j == 0 ? r[e] * scale_me : (degen ? qv[e] : r[e] * invZ);
-          const float nv = (i0 + e < len) ? fmaxf(prev - qv[e], 0.f) : 0.f;
-          r[e] = nv;
-          part += nv;
+          const bool in = (i0 + e < clen) && (!masked || (zp[e] - Mp >= logb));
+          sv[e] = in ? fmaf(c1, zp[e], -alpha * zq[e]) : -INFINITY;
+          gm = fmaxf(gm, sv[e]);
         }
-        st8_value(zp_s, zq_s, i0, r);
-        zsum += part;
-        if (last) {
-          const float bs = warp_sum(part);
-          if (lane == 0) blk[grp >> 5] = bs;
-        }
-      }
-      zsum = block_sum(zsum, redf);
-      mine = neutral_partial();
-      mine.s = zsum;
-      if (tid == 0 && j + 1 < m) {
-        const int t = ktok[j + 1];
-        if (t >= lo && t < hi) {
-          mine.cap_own = 1;
-          mine.cap_r = ld1_value(zp_s, zq_s, t - static_cast<int>(lo));
-          mine.cap_q = q_s[t - static_cast<int>(lo)];
-        }
-      }
-      cluster_exchange(cl, part, gath, stage, mine, C);
-      float Z = 0.f, cr = 0.f, cq = 0.f;
-      for (int k = 0; k < C; ++k) {
-        Z += gath[k].s;
-        if (gath[k].cap_own) {
-          cr = gath[k].cap_r;
-          cq = gath[k].cap_q;
-        }
-      }
-      if (Z > 0.f) {
-        degen = false;
-        invZ = 1.f / Z;
-        rt = cr * invZ;
-      } else {
-        degen = true;  // r_j == q in exact arithmetic when nothing is left
-        rt = cq;
-      }
-      qt = cq;
-    }
-    if (acc < 0) {
-      // ---- terminal draw: two-level exponential race (block of 256 tokens, then a token)
-      if (degen) {  // the residual is q itself: its block masses
-        for (int base = 0; base < ngw; base += kThreads) {
-          const int grp = base + tid;
-          if (grp >= ngw) continue;
-          const int i0 = grp << 3;
-          float qv[8];
-          lds8(q_s + i0, qv);
-          float part = 0.f;
+        if (gm > lmax) {
+          lsum *= ex2((lmax - gm) * k2);  // 0 while lmax is -inf
+          lmax = gm;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) part += (i0 + e < len) ? qv[e] : 0.f;
-          const float bs = warp_sum(part);
-          if (lane == 0) blk[grp >> 5] = bs;
+          for (int e = 7; e >= 0; --e)
+            if (sv[e] == gm) larg = static_cast<int>(x0) + i0 + e;
         }
-        __syncthreads();
-      }
-      // leaf rows hold e(x) relative to this CTA's max; bring block masses to the common scale
-      const float offset2 = leaf_race ? (m_cta - M) * k2 : 0.f;
-      const int nblk = (len + kRaceBlock - 1) / kRaceBlock;
-      const int kbase = static_cast<int>(lo / kRaceBlock);
-      float bk = -INFINITY;
-      int bb = INT_MAX;
-      for (int t = tid; t < nblk; t += kThreads) {
-        const float R = blk[t];
-        if (R > 0.f) {
-          const uint32_t kabs = static_cast<uint32_t>(kbase + t);
-          const float key = race_key(lg2(R) + offset2,
-                                     philox_word(p.seed, p.offset, static_cast<uint32_t>(g),
-                                                 0x80000000u | (kabs >> 2), static_cast<int>(kabs & 3)));
-          if (key > bk) {
-            bk = key;
-            bb = static_cast<int>(kabs);
+        if (lmax > -INFINITY) {
+          const float mk = lmax * k2;
+          float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; e += 2) {
+            s0 += ex2(fmaf(sv[e], k2, -mk));
+            s1 += ex2(fmaf(sv[e + 1], k2, -mk));
+          }
+          lsum += s0 + s1;
+        }
+        if (leaf_race) {
+          const float bm = warp_max(gm);
+          float part = 0.f;
+          if (bm > -INFINITY) {
+            const float mk = bm * k2;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) part += ex2(fmaf(sv[e], k2, -mk));
+          }
+          const float bs = warp_sum(part);
+          if (lane == 0) {
+            const int kabs = static_cast<int>(x0 / kRaceBlock) + kb;
+            bmax[kabs] = bm;
+            bsum[kabs] = bs;
           }
         }
       }
-      block_argmax(bk, bb, redf, redi);
-      mine = neutral_partial();
-      mine.m = bk;
-      mine.arg = bb;
-      cluster_exchange(cl, part, gath, stage, mine, C);
-      float K = -INFINITY;
-      int kstar = INT_MAX;
-      for (int k = 0; k < C; ++k) argmax_merge(K, kstar, gath[k].m, gath[k].arg);
-      // token race inside block kstar, by the CTA whose slice holds it (one warp, 8 tokens a lane)
-      mine = neutral_partial();
-      const int64_t x_first = static_cast<int64_t>(kstar) * kRaceBlock;
-      if (kstar != INT_MAX && x_first >= lo && x_first < hi && warp == 0) {
-        const int i0 = static_cast<int>(x_first - lo) + lane * 8;
-        float r[8], qv[8];
-        ld8_value(zp_s, zq_s, i0, r);
-        if (degen) lds8(q_s + i0, qv);
-        const uint32_t x0 = static_cast<uint32_t>(x_first) + static_cast<uint32_t>(lane * 8);
-        const uint32_t o0 = static_cast<uint32_t>(p.offset), o1 = static_cast<uint32_t>(p.offset >> 32);
-        const uint32_t s0 = static_cast<uint32_t>(p.seed), s1 = static_cast<uint32_t>(p.seed >> 32);
-        const uint4 wa = philox4x32_10(make_uint4(static_cast<uint32_t>(g), 1u + (x0 >> 2), o0, o1), s0, s1);
-        const uint4 wb = philox4x32_10(make_uint4(static_cast<uint32_t>(g), 2u + (x0 >> 2), o0, o1), s0, s1);
-        const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
-        float tk = -INFINITY;
-        int tx = INT_MAX;
+    });
+    if (tid < m) {
+      czp[tid] = pzp;
+      czq[tid] = pzq;
+      cq[tid] = pq;
+    }
+    for (int k = kThreads + tid; k < m; k += kThreads) {  // rows with more children than threads
+      const int t = ktok[k];
+      const bool ok = t >= 0 && t < V;
+      czp[k] = ok ? ld1(zp_row, t) : 0.f;
+      czq[k] = ok ? ld1(zq_row, t) : 0.f;
+      cq[k] = (ok && sampled) ? q_row[t] : 0.f;
+    }
+    // row statistics from the lanes' (max, sum, argmax) (the reductions below also publish
+    // czp/czq/cq)
+    const float M = block_max(lmax, redf);
+    const float S = block_sum(lmax > -INFINITY ? lsum * ex2((lmax - M) * k2) : 0.f, redf);
+    float lbest = lmax;
+    block_argmax(lbest, larg, redf, redi);
+    const int arg = larg;
+    uint32_t status = rs->status;
+    if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
+    const float logS = logf(S);
+    const float invS = 1.f / S;
+    const float Mk2 = M * k2;
+
+    // ---- outputs of the Eq. 1 target
+    if (tid == 0) {
+      if (p.cd_argmax) p.cd_argmax[g] = arg;
+      if (p.cd_lse) p.cd_lse[g] = M * invT + logS;
+      if (n == 0 && p.cd_logprob) p.cd_logprob[g] = 0.f;
+    }
+    if (p.cd_logprob) {
+      for (int k = tid; k < m; k += kThreads) {
+        const bool in = !masked || (czp[k] - Mp >= logb);
+        p.cd_logprob[static_cast<int64_t>(b) * N + kids[k]] =
+            in ? (fmaf(c1, czp[k], -alpha * czq[k]) - M) * invT - logS : -INFINITY;
+      }
+    }
+
+    int acc = -1, term = -1;
+    if (!sampled) {
+      // ---- greedy rule: the first child whose token is the argmax
+      for (int k = 0; k < m; ++k)
+        if (ktok[k] == arg) {
+          acc = kids[k];
+          break;
+        }
+      if (acc < 0) term = arg;
+    } else {
+      // ---- sampled rule: test the children in order; each rejection streams one residual pass.
+      // r_j(x) = max(0, r_{j-1}(x) - q(x)) / Z_j with r_0 = pi_CD,T; invZ[j] = 0 marks Z_j = 0,
+      // where r_{j-1} equals q exactly and r_j is taken as q.
+      auto residual_at = [&](float s, bool in, float qv, int levels) -> float {
+        float r = in ? ex2(fmaf(s, k2, -Mk2)) * invS : 0.f;
+        for (int i = 1; i <= levels; ++i) {
+          const float iz = invZ[i];
+          r = iz > 0.f ? fmaxf(r - qv, 0.f) * iz : qv;
+        }
+        return r;
+      };
+      for (int j = 0; j < m; ++j) {
+        if (tid == 0) {
+          const bool in = !masked || (czp[j] - Mp >= logb);
+          const float rt = residual_at(fmaf(c1, czp[j], -alpha * czq[j]), in, cq[j], j);
+          const float qt = cq[j];
+          const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
+          const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[j]);
+          const float u = u01(philox_block(p.seed, p.offset, G, 0u).x);
+          rs->accept = u <= ratio;
+        }
+        __syncthreads();
+        if (rs->accept) {
+          acc = kids[j];
+          break;
+        }
+        // rejected: one more pass gives Z_{j+1}; after the last child it also keeps the block
+        // masses of the final residual and of q for the terminal race
+        const bool last = j + 1 == m;
+        const int first = limit;
+        limit += nch_r;
+        if (tid == 0)
+          for (int Li = first; Li < limit && Li < first + sp.nst; ++Li) issue(Li, pol);
+        float zl = 0.f;
+        run_items(nch_r, [&](const Stage<TIn>& st, int64_t x0, int clen) {
+          for (int kb = warp; kb * kRaceBlock < sp.tok_r; kb += kWarps) {
+            if (kb * kRaceBlock >= clen) break;  // warp-uniform
+            const int i0 = kb * kRaceBlock + lane * 8;
+            float zp[8], zq[8], qv[8];
+            ld8(st.zp + i0, zp);
+            ld8(st.zq + i0, zq);
+            ld8(st.q + i0, qv);
+            float part = 0.f, partq = 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float v = degen ? qv[e] : r[e];
-          if (i0 + e < len && v > 0.f) {
-            const float key = race_key(lg2(v), w[e]);
-            if (key > tk) {
-              tk = key;
-              tx = static_cast<int>(x0) + e;
+            for (int e = 0; e < 8; ++e) {
+              const bool valid = i0 + e < clen;
+              const float qe = valid ? qv[e] : 0.f;
+              const bool in = valid && (!masked || (zp[e] - Mp >= logb));
+              const float r = residual_at(fmaf(c1, zp[e], -alpha * zq[e]), in, qe, j);
+              part += valid ? fmaxf(r - qe, 0.f) : 0.f;
+              partq += qe;
+            }
+            zl += part;
+            if (last) {
+              const float br = warp_sum(part);
+              const float bqq = warp_sum(partq);
+              if (lane == 0) {
+                const int kabs = static_cast<int>(x0 / kRaceBlock) + kb;
+                bres[kabs] = br;
+                bq[kabs] = bqq;
+              }
+            }
+          }
+        });
+        const float Z = block_sum(zl, redf);
+        if (tid == 0) invZ[j + 1] = Z > 0.f ? 1.f / Z : 0.f;
+        __syncthreads();
+      }
+      if (acc < 0) {
+        // ---- terminal draw, two-level exponential race: a 256-token block by its mass ...
+        const bool leaf = m == 0;
+        const bool degen = !leaf && !(invZ[m] > 0.f);
+        float bk = -INFINITY;
+        int bb = INT_MAX;
+        for (int k = tid; k < sp.nblk; k += kThreads) {
+          float lm = -INFINITY;
+          if (leaf) {
+            if (bmax[k] > -INFINITY && bsum[k] > 0.f) lm = lg2(bsum[k]) + (bmax[k] - M) * k2;
+          } else {
+            const float Rk = degen ? bq[k] : bres[k];
+            if (Rk > 0.f) lm = lg2(Rk);
+          }
+          if (lm > -INFINITY) {
+            const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
+                                         0x80000000u | (static_cast<uint32_t>(k) >> 2));
+            const float key = race_key(lm, word_of(w, k & 3));
+            if (key > bk) {
+              bk = key;
+              bb = k;
             }
           }
         }
+        block_argmax(bk, bb, redf, redi);
+        // ... then a token of that block (warp 0 re-reads the block's 256 tokens)
+        if (warp == 0) {
+          float tk = -INFINITY;
+          int tx = INT_MAX;
+          if (bb != INT_MAX) {
+            const int64_t xb = static_cast<int64_t>(bb) * kRaceBlock + lane * 8;
+            const uint4 wa = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
+                                          1u + static_cast<uint32_t>(xb >> 2));
+            const uint4 wb = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
+                                          2u + static_cast<uint32_t>(xb >> 2));
+            const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
 #pragma unroll
-        for (int o = 16; o; o >>= 1) argmax_merge(tk, tx, __shfl_xor_sync(~0u, tk, o), __shfl_xor_sync(~0u, tx, o));
-        if (lane == 0) {
-          mine.m = tk;
-          mine.arg = tx;
-          mine.cap_own = 1;
+            for (int e = 0; e < 8; ++e) {
+              const int64_t x = xb + e;
+              if (x < V) {
+                const float z = ld1(zp_row, x);
+                const bool in = !masked || (z - Mp >= logb);
+                const float s = fmaf(c1, z, -alpha * ld1(zq_row, x));
+                float v;
+                if (leaf) {
+                  v = in ? ex2(fmaf(s, k2, -Mk2)) : 0.f;
+                } else {
+                  const float qe = q_row[x];
+                  v = degen ? qe : fmaxf(residual_at(s, in, qe, m - 1) - qe, 0.f);
+                }
+                if (v > 0.f) {
+                  const float key = race_key(lg2(v), w[e]);
+                  if (key > tk) {
+                    tk = key;
+                    tx = static_cast<int>(x);
+                  }
+                }
+              }
+            }
+          }
+          warp_argmax(tk, tx);
+          if (lane == 0) rs->term = tx;
         }
+        __syncthreads();
+        term = rs->term;
       }
-      cluster_exchange(cl, part, gath, stage, mine, C);
-      for (int k = 0; k < C; ++k)
-        if (gath[k].cap_own) term = gath[k].arg;
     }
+    if (tid == 0) {
+      RowRecord r;
+      r.acc_child = acc;
+      r.term_token = acc < 0 ? term : -1;
+      r.status = status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
+      r.reserved = 0;
+      p.rec[g] = r;
+    }
+    seq = seq0 + static_cast<uint32_t>(L);
+    __syncthreads();  // row state in shared memory is rewritten by the next row
   }
-
-  if (rank == 0 && tid == 0) {
-    RowRecord r;
-    r.acc_child = acc;
-    r.term_token = acc < 0 ? term : -1;
-    r.status = status;
-    r.reserved = 0;
-    p.rec[g] = r;
-  }
-  cl.sync();  // no CTA leaves while a peer may still read its partial slots
 }
 
 // ------------------------------------------------------------------------------------------
@@ -799,29 +794,22 @@ __global__ void __launch_bounds__(kThreads) terminal_residual_kernel(const Score
   const bool masked = beta > 0.f;
   const float logb = masked ? logf(beta) : -INFINITY;
   const float c1 = 1.f + alpha, invT = 1.f / T;
-  auto ld = [](const TIn* a, int64_t i) -> float {
-    if constexpr (sizeof(TIn) == 2) {
-      return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(a)[i]);
-    } else {
-      return static_cast<float>(reinterpret_cast<const float*>(a)[i]);
-    }
-  };
   float Mp = 0.f;
   if (masked) {
     float v = -INFINITY;
-    for (int64_t x = threadIdx.x; x < V; x += kThreads) v = fmaxf(v, ld(zp, x));
+    for (int64_t x = threadIdx.x; x < V; x += kThreads) v = fmaxf(v, ld1(zp, x));
     Mp = block_max(v, redf);
   }
   float M = -INFINITY;
   for (int64_t x = threadIdx.x; x < V; x += kThreads) {
-    const float z = ld(zp, x);
-    if (!masked || z - Mp >= logb) M = fmaxf(M, fmaf(c1, z, -alpha * ld(zq, x)));
+    const float z = ld1(zp, x);
+    if (!masked || z - Mp >= logb) M = fmaxf(M, fmaf(c1, z, -alpha * ld1(zq, x)));
   }
   M = block_max(M, redf);
   float s = 0.f;
   for (int64_t x = threadIdx.x; x < V; x += kThreads) {
-    const float z = ld(zp, x);
-    const float e = (!masked || z - Mp >= logb) ? expf((fmaf(c1, z, -alpha * ld(zq, x)) - M) * invT) : 0.f;
+    const float z = ld1(zp, x);
+    const float e = (!masked || z - Mp >= logb) ? expf((fmaf(c1, z, -alpha * ld1(zq, x)) - M) * invT) : 0.f;
     out[x] = e;
     s += e;
   }
@@ -849,53 +837,75 @@ __global__ void __launch_bounds__(kThreads) terminal_residual_kernel(const Score
 }
 
 // ------------------------------------------------------------------------------------------
+struct DeviceInfo {
+  int sms = 0;
+  cudaError_t err = cudaSuccess;
+};
+
 template <typename TIn>
-cudaError_t prepare_kernel_attributes() {
+cudaError_t prepare_kernel(int* sms) {
   static std::once_flag once[64];
-  static cudaError_t result[64];
+  static DeviceInfo info[64];
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   std::call_once(once[dev], [&] {
-    cudaError_t r = cudaFuncSetAttribute(score_rows_kernel<TIn>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kSmemMax));
-    if (r == cudaSuccess) r = cudaFuncSetAttribute(score_rows_kernel<TIn>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    result[dev] = r;
+    DeviceInfo d;
+    d.err = cudaFuncSetAttribute(score_rows_kernel<TIn>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kSmemMax));
+    if (d.err == cudaSuccess) d.err = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
+    info[dev] = d;
   });
-  return result[dev];
+  *sms = info[dev].sms;
+  return info[dev].err;
 }
 
-size_t header_bytes(int N, int64_t chunk) {
-  const size_t h = 16 + 2 * sizeof(Partial) + kMaxCluster * sizeof(Partial) + 64 * sizeof(float) + 8 * sizeof(int) +
-                   static_cast<size_t>(N) * 12 + static_cast<size_t>(chunk / kRaceBlock) * sizeof(float);
-  return (h + 127) & ~static_cast<size_t>(127);
+struct Layout {
+  int meta_offset, blk_offset, stage_offset;
+  size_t total;
+};
+
+Layout layout_for(int N, int nblk, int nst, int stage_bytes) {
+  Layout l;
+  l.meta_offset = 8 * kMaxStages + 64 * 4;
+  const size_t meta_end = static_cast<size_t>(l.meta_offset) + sizeof(RowShared) + static_cast<size_t>(N) * 4 * 6;
+  l.blk_offset = static_cast<int>((meta_end + 15) & ~static_cast<size_t>(15));
+  const size_t blk_end = static_cast<size_t>(l.blk_offset) + static_cast<size_t>(nblk) * 4 * 4;
+  l.stage_offset = static_cast<int>((blk_end + 127) & ~static_cast<size_t>(127));
+  l.total = static_cast<size_t>(l.stage_offset) + static_cast<size_t>(nst) * stage_bytes;
+  return l;
 }
+
+// Tokens per stage: z_p and z_q fill a stage in the max / stats passes; z_p, z_q and q share
+// it in residual passes (whole race blocks of 256 tokens either way).
+int tokens_a(int es) { return kStageBytes / (2 * es); }
+int tokens_r(int es) { return kStageBytes / (2 * es + 4) / kRaceBlock * kRaceBlock; }
 
 }  // namespace
 
 RowGeometry row_geometry(const ScoreArgs& a) {
   RowGeometry geo{};
-  const size_t es = a.dtype == DCD_BF16 ? 2 : 4;
-  const size_t bpe = 2 * es + (a.q ? 4 : 0);
-  auto chunk_for = [&](int c) {  // slices hold whole 256-token race blocks
-    const int64_t per = (a.V + c - 1) / c;
-    return (per + kRaceBlock - 1) / kRaceBlock * kRaceBlock;
-  };
-  int C = a.force_cluster;
-  if (C <= 0) {
-    C = kMaxCluster;
-    for (int c = 1; c <= kMaxCluster; c *= 2)
-      if (static_cast<size_t>(chunk_for(c)) * bpe <= kSmemBudget) {
-        C = c;
+  const int es = a.dtype == DCD_BF16 ? 2 : 4;
+  const int nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
+  int nst = a.force_stages;
+  if (nst <= 0) {
+    // the deepest ring (up to 3 stages) that still lets two CTAs share an SM
+    nst = 2;
+    for (int s = 3; s >= 2; --s)
+      if (2 * (layout_for(a.N, nblk, s, kStageBytes).total + 1024) <= kSmemPerSm) {
+        nst = s;
         break;
       }
   }
-  geo.cluster = C;
-  geo.chunk = chunk_for(C);
-  geo.smem = header_bytes(a.N, geo.chunk) + static_cast<size_t>(geo.chunk) * bpe;
+  const Layout l = layout_for(a.N, nblk, nst, kStageBytes);
+  const int per_sm = static_cast<int>(kSmemPerSm / (l.total + 1024));
+  geo.stages = nst;
+  geo.stage_tokens = tokens_a(es);
+  geo.smem = l.total;
+  geo.ctas_per_sm = per_sm > 4 ? 4 : per_sm;
   auto al16 = [](const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; };
-  geo.bulk = !a.force_plain && al16(a.zp) && al16(a.zq) && (a.ld * static_cast<int64_t>(es)) % 16 == 0 &&
+  geo.bulk = !a.force_plain && al16(a.zp) && al16(a.zq) && (a.ld * es) % 16 == 0 &&
              (!a.q || (al16(a.q) && (a.ldq * 4) % 16 == 0));
   return geo;
 }
@@ -904,38 +914,35 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   const int64_t R = static_cast<int64_t>(a.B) * a.N;
   if (R == 0) return cudaSuccess;
   const RowGeometry geo = row_geometry(a);
-  if (geo.smem > kSmemMax || geo.cluster < 1 || geo.cluster > kMaxCluster ||
-      (geo.cluster & (geo.cluster - 1)) != 0 || R * geo.cluster > INT_MAX)
+  if (geo.smem > kSmemMax || geo.stages < 1 || geo.stages > kMaxStages || geo.ctas_per_sm < 1)
     return cudaErrorInvalidConfiguration;
-  KParams kp;
-  kp.a = a;
-  kp.cluster = geo.cluster;
-  kp.chunk = static_cast<int32_t>(geo.chunk);
-  kp.bulk = geo.bulk;
-  kp.data_offset = static_cast<int32_t>(header_bytes(a.N, geo.chunk));
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(R * geo.cluster));
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = geo.smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = geo.cluster;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaError_t e;
-  if (a.dtype == DCD_BF16) {
-    e = prepare_kernel_attributes<__nv_bfloat16>();
-    if (e != cudaSuccess) return e;
-    e = cudaLaunchKernelEx(&cfg, score_rows_kernel<__nv_bfloat16>, kp);
-  } else {
-    e = prepare_kernel_attributes<float>();
-    if (e != cudaSuccess) return e;
-    e = cudaLaunchKernelEx(&cfg, score_rows_kernel<float>, kp);
-  }
-  return e;
+  int sms = 0;
+  cudaError_t e = a.dtype == DCD_BF16 ? prepare_kernel<__nv_bfloat16>(&sms) : prepare_kernel<float>(&sms);
+  if (e != cudaSuccess) return e;
+  const int es = a.dtype == DCD_BF16 ? 2 : 4;
+  SParams sp;
+  sp.a = a;
+  sp.nst = geo.stages;
+  sp.tok_a = tokens_a(es);
+  sp.tok_r = tokens_r(es);
+  sp.bulk = geo.bulk;
+  sp.nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
+  const Layout l = layout_for(a.N, sp.nblk, sp.nst, kStageBytes);
+  sp.meta_offset = l.meta_offset;
+  sp.blk_offset = l.blk_offset;
+  sp.stage_offset = l.stage_offset;
+  sp.work = a.err + 1;  // header word 1
+  // the device error word and the work counter start every call at zero
+  e = cudaMemsetAsync(a.err, 0, 2 * sizeof(uint32_t), stream);
+  if (e != cudaSuccess) return e;
+  int64_t grid = static_cast<int64_t>(sms) * geo.ctas_per_sm;
+  if (grid > R) grid = R;
+  if (grid < 1) grid = 1;
+  if (a.dtype == DCD_BF16)
+    score_rows_kernel<__nv_bfloat16><<<static_cast<unsigned>(grid), kThreads, geo.smem, stream>>>(sp);
+  else
+    score_rows_kernel<float><<<static_cast<unsigned>(grid), kThreads, geo.smem, stream>>>(sp);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_t* err, int32_t* accept_len,

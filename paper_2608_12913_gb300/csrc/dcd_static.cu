@@ -56,8 +56,8 @@ extern "C" int dcd_verify_sample_noalloc(const dcd_shape* shape, const void* z_e
   void* scratch = nullptr;
   const int rc = scratch_address(&scratch);
   if (rc != DCD_OK) return rc;
-  // The error word is reset by the row kernel at the start of every call and every row record
-  // is rewritten, so nothing left by an earlier call leaks into this one.
+  // Every call zeroes the error word and the work counter with a stream-ordered memset before
+  // its kernels run, and rewrites every row record, so nothing left by an earlier call leaks in.
   return dcd_verify_sample(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset,
                            accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse, residual, scratch,
                            DCD_STATIC_SCRATCH_BYTES, stream);

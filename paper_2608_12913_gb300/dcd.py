@@ -254,7 +254,7 @@ def dcd_verify_sample_noalloc(z_exp, z_ama, q, tokens, parents, alpha, temperatu
 
 
 def dcd_score_rows(z_exp, z_ama, tokens, parents, alpha, beta=None, q=None, temperature=None, seed: int = 0,
-                   offset: int = 0, *, out=None, workspace=None, stream=None, cluster: int = 0,
+                   offset: int = 0, *, out=None, workspace=None, stream=None, stages: int = 0,
                    plain_loads: bool = False) -> dict:
     """The per-row step alone (records stay in the workspace); see dcd_tree_walk."""
     c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
@@ -265,8 +265,8 @@ def dcd_score_rows(z_exp, z_ama, tokens, parents, alpha, beta=None, q=None, temp
               _ptr(beta), _ptr(temperature), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
               _ptr(o.get("cd_logprob")), _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(ws), ws.numel(),
               _stream(stream))
-    if cluster or plain_loads:
-        st = lib.dcd_score_rows_ex(*common, int(cluster), int(bool(plain_loads)))
+    if stages or plain_loads:
+        st = lib.dcd_score_rows_ex(*common, int(stages), int(bool(plain_loads)))
     else:
         st = lib.dcd_score_rows(*common)
     _check(st, "dcd_score_rows")

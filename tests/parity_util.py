@@ -37,19 +37,19 @@ def records(ws: torch.Tensor, R: int):
     return dict(acc_child=raw[:, 0].copy(), term_token=raw[:, 1].copy(), status=raw[:, 2].view(np.uint32).copy())
 
 
-def run_gpu(w, *, sampled: bool, residual: bool = False, cluster: int = 0, plain: bool = False, offset=None,
+def run_gpu(w, *, sampled: bool, residual: bool = False, stages: int = 0, plain: bool = False, offset=None,
             out=None, workspace=None):
     dev = torch.device("cuda")
     wd = w.to(dev)
     off = w.offset if offset is None else offset
-    if cluster or plain:
+    if stages or plain:
         q = None
         temp = None
         if sampled:
             q = wd.q if wd.q is not None else torch.zeros_like(wd.z_exp, dtype=torch.float32)
             temp = wd.temperature
         o = dcd.dcd_score_rows(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta, q=q, temperature=temp,
-                               seed=w.seed, offset=off, cluster=cluster, plain_loads=plain, out=out,
+                               seed=w.seed, offset=off, stages=stages, plain_loads=plain, out=out,
                                workspace=workspace)
         dcd.dcd_tree_walk(w.B, w.N, w.V, o, o["workspace"])
     elif sampled:

@@ -102,9 +102,9 @@ def test_host_checks_reject_before_launch(lib):
     # row stride shorter than the vocabulary
     bad = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, ld=50)
     assert lib.dcd_verify_greedy(ctypes.byref(bad), *base, ws_ok, 1 << 20, None) == -1
-    # invalid forced cluster size
+    # invalid forced ring depth
     assert lib.dcd_score_rows_ex(ctypes.byref(sh), P, P, None, P, P, P, None, None, 0, 0, None, None, None, ws_ok,
-                                 1 << 20, None, 3, 0) == -1
+                                 1 << 20, None, 1, 0) == -1
     # empty batch is a no-op
     empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
     assert lib.dcd_verify_greedy(ctypes.byref(empty), *base, ws_ok, 1 << 20, None) == 0

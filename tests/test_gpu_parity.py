@@ -2,7 +2,7 @@
 
 Covers the four streaming workloads (tiny fp32 chain; 60-node tree greedy; the same
 tree sampled at T = 1; the 32-sequence mixed batch, reduced and at full size), the
-plausibility mask, every cluster geometry and the plain-load path, ragged and tiny
+plausibility mask, every ring depth and the plain-load path, ragged and tiny
 vocabularies, degenerate trees, device-side input errors, determinism and offsets.
 Bars and the ambiguity rule are in parity_util.
 """
@@ -72,11 +72,11 @@ def test_plausibility_mask(beta, sampled):
     compare(w, g, r, check_residual=sampled)
 
 
-@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
+@pytest.mark.parametrize("stages", [2, 3, 4, 6])
 @pytest.mark.parametrize("plain", [False, True])
-def test_every_cluster_geometry(cluster, plain):
+def test_every_ring_depth(stages, plain):
     w = workloads.make_config(3, B=4, V=12347, seed=7, margin_fn=oracle.margin_fn)
-    g = run_gpu(w, sampled=True, cluster=cluster, plain=plain)
+    g = run_gpu(w, sampled=True, stages=stages, plain=plain)
     r = _oracle(w)
     compare(w, g, r)
 
@@ -148,7 +148,7 @@ def _greedy(w):
 def test_split_steps_equal_verify_and_determinism():
     w = workloads.make_config(3, B=6, V=4001, seed=17)
     a = run_gpu(w, sampled=True)
-    b = run_gpu(w, sampled=True, cluster=0)
+    b = run_gpu(w, sampled=True, stages=0)
     wd = w.to("cuda")
     o = dcd.dcd_score_rows(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta, q=wd.q,
                            temperature=wd.temperature, seed=w.seed, offset=w.offset)
