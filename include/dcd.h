@@ -46,7 +46,8 @@
  *   s'(x) / T_eff - cd_lse[g]); T_eff = T, or 1 for greedy sequences.
  * - Memory: every array pointer is a DEVICE pointer owned by the caller.  The
  *   library allocates nothing per call; scratch lives in the caller's workspace
- *   (dcd_workspace_bytes).  Calls are asynchronous and ordered on `stream`; host-side
+ *   (dcd_workspace_bytes: 256 bytes plus, per row, 96 bytes and 16 bytes per 4096
+ *   vocabulary tokens (bf16 logits); its contents need no initialisation).  Calls are asynchronous and ordered on `stream`; host-side
  *   argument checks return a negative status before anything is launched.  Two
  *   calls that share a workspace must not overlap on the device.
  * - Thread safety: entry points may be called from several host threads, each with
@@ -161,9 +162,10 @@ int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_p
 
 /*
  * Capacity of the scratch array inside the library used by dcd_verify_sample_noalloc:
- * enough for dcd_workspace_bytes(shape) <= 512 KiB, i.e. B * N <= 32752 rows.
+ * enough for dcd_workspace_bytes(shape) <= 4 MiB, e.g. B * N up to about 6900 rows at
+ * V = 128256 with bf16 logits.
  */
-#define DCD_STATIC_SCRATCH_BYTES (512u * 1024u)
+#define DCD_STATIC_SCRATCH_BYTES (4u * 1024u * 1024u)
 
 /*
  * dcd_verify_sample without a workspace argument, for callers that cannot allocate

@@ -25,7 +25,8 @@ bool shape_ok(const dcd_shape* s, bool need_q) {
 
 size_t workspace_bytes_for(const dcd_shape* s) {
   const size_t rows = static_cast<size_t>(s->B) * static_cast<size_t>(s->N);
-  const size_t raw = dcd::kWorkspaceHeader + rows * sizeof(dcd::RowRecord);
+  const size_t raw = dcd::kWorkspaceHeader +
+                     rows * (sizeof(dcd::Job) + sizeof(dcd::RowRecord) + dcd::slot_bytes(s->V, s->logits_dtype));
   return (raw + 255) & ~static_cast<size_t>(255);
 }
 
@@ -35,11 +36,24 @@ int check_workspace(const dcd_shape* s, const void* ws, size_t bytes) {
   return DCD_OK;
 }
 
-dcd::RowRecord* records(void* ws) {
-  return reinterpret_cast<dcd::RowRecord*>(static_cast<char*>(ws) + dcd::kWorkspaceHeader);
-}
+struct WsView {
+  dcd::WsHeader* hdr;
+  dcd::Job* jobs;
+  dcd::RowRecord* rec;
+  unsigned char* slots;
+};
 
-uint32_t* error_word(void* ws) { return static_cast<uint32_t*>(ws); }
+WsView view(void* ws, const dcd_shape* s) {
+  const size_t rows = static_cast<size_t>(s->B) * static_cast<size_t>(s->N);
+  char* base = static_cast<char*>(ws);
+  WsView v;
+  v.hdr = reinterpret_cast<dcd::WsHeader*>(base);
+  v.jobs = reinterpret_cast<dcd::Job*>(base + dcd::kWorkspaceHeader);
+  v.rec = reinterpret_cast<dcd::RowRecord*>(base + dcd::kWorkspaceHeader + rows * sizeof(dcd::Job));
+  v.slots = reinterpret_cast<unsigned char*>(base + dcd::kWorkspaceHeader +
+                                             rows * (sizeof(dcd::Job) + sizeof(dcd::RowRecord)));
+  return v;
+}
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? DCD_OK : DCD_ERR_CUDA; }
 
@@ -67,8 +81,11 @@ dcd::ScoreArgs make_args(const dcd_shape* s, const void* z_exp, const void* z_am
   a.cd_logprob = cd_logprob;
   a.cd_argmax = cd_argmax;
   a.cd_lse = cd_lse;
-  a.rec = records(ws);
-  a.err = error_word(ws);
+  const WsView v = view(ws, s);
+  a.hdr = v.hdr;
+  a.jobs = v.jobs;
+  a.rec = v.rec;
+  a.slots = v.slots;
   a.force_stages = 0;
   a.force_plain = 0;
   return a;
@@ -122,8 +139,9 @@ int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_p
   if (!accept_len || !accept_path || !bonus) return DCD_ERR_INVALID_ARG;
   const int ws = check_workspace(shape, workspace, workspace_bytes);
   if (ws != DCD_OK) return ws;
-  return cuda_status(dcd::launch_tree_walk(shape->B, shape->N, records(workspace), error_word(workspace), accept_len,
-                                           accept_path, bonus, reinterpret_cast<cudaStream_t>(stream)));
+  const WsView v = view(workspace, shape);
+  return cuda_status(dcd::launch_tree_walk(shape->B, shape->N, v.rec, &v.hdr->err, accept_len, accept_path, bonus,
+                                           reinterpret_cast<cudaStream_t>(stream)));
 }
 
 int dcd_verify_greedy(const dcd_shape* shape, const void* z_exp, const void* z_ama, const int32_t* tokens,

@@ -1,0 +1,278 @@
+// dcd_device.cuh -- device helpers shared by the library's CUDA kernels (not by the oracle):
+// PTX wrappers for mbarriers, L2 cache policies and bulk asynchronous copies; fast exp2/log2;
+// Philox4x32-10; shared-memory element access; warp and block reductions.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <climits>
+
+namespace dcd {
+namespace dev {
+
+constexpr int kThreads = 256;  // threads per CTA of every row kernel
+constexpr int kWarps = kThreads / 32;
+constexpr int kRaceBlock = 256;                   // tokens per block of the two-level terminal race
+constexpr long long kWaitCycles = 4000000000ll;  // bounded waits: about two seconds at the boost clock
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ------------------------------------------------------------------------------------------
+// PTX wrappers: mbarrier, L2 cache policies and bulk asynchronous global->shared copies.
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile(
+      "{\n\t.reg .b64 st;\n\t"
+      "mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}" ::"r"(smem_addr(bar)),
+      "r"(bytes)
+      : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile(
+      "{\n\t.reg .b64 st;\n\t"
+      "mbarrier.arrive.shared::cta.b64 st, [%0];\n\t}" ::"r"(smem_addr(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.b32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// Bounded wait: gives up after kWaitCycles and reports false.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
+  const long long start = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - start > kWaitCycles) return false;
+  }
+  return true;
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], "
+      "%4;" ::"r"(smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
+      : "memory");
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float lg2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// ------------------------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32->64 products
+// with the published multipliers, the key advanced by the published Weyl increments.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return c;
+}
+
+__device__ __forceinline__ uint4 philox_block(uint64_t seed, uint64_t off, uint32_t c0, uint32_t c1) {
+  return philox4x32_10(make_uint4(c0, c1, static_cast<uint32_t>(off), static_cast<uint32_t>(off >> 32)),
+                       static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
+}
+
+__device__ __forceinline__ uint32_t word_of(const uint4& w, int i) {
+  return i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w;
+}
+
+// 32-bit word -> uniform in (0, 1): ((w >> 9) + 1/2) 2^-23, exact in fp32.
+__device__ __forceinline__ float u01(uint32_t w) {
+  return (__uint2float_rn(w >> 9) + 0.5f) * 1.1920928955078125e-07f;
+}
+
+// Race key in log2 units: log2 r - log2(-log2 u) orders tokens exactly as ln r - ln(-ln u)
+// (the two differ by a positive factor and a constant).
+__device__ __forceinline__ float race_key(float log2_mass, uint32_t word) {
+  return log2_mass - lg2(-lg2(u01(word)));
+}
+
+// ------------------------------------------------------------------------------------------
+// Element access: 8 consecutive tokens as fp32 (16 B of bf16 or 32 B of fp32).
+__device__ __forceinline__ void ld8(const float* p, float v[8]) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0];
+  const float4 b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+__device__ __forceinline__ void ld8(const __nv_bfloat16* p, float v[8]) {
+  const uint4 a = *reinterpret_cast<const uint4*>(p);
+  v[0] = __uint_as_float(a.x << 16); v[1] = __uint_as_float(a.x & 0xffff0000u);
+  v[2] = __uint_as_float(a.y << 16); v[3] = __uint_as_float(a.y & 0xffff0000u);
+  v[4] = __uint_as_float(a.z << 16); v[5] = __uint_as_float(a.z & 0xffff0000u);
+  v[6] = __uint_as_float(a.w << 16); v[7] = __uint_as_float(a.w & 0xffff0000u);
+}
+
+__device__ __forceinline__ float ld1(const float* p, int64_t i) { return p[i]; }
+__device__ __forceinline__ float ld1(const __nv_bfloat16* p, int64_t i) { return __bfloat162float(p[i]); }
+
+// ------------------------------------------------------------------------------------------
+// Reductions.
+__device__ __forceinline__ void argmax_merge(float& v, int& i, float v2, int i2) {
+  if (v2 > v || (v2 == v && i2 < i)) {
+    v = v2;
+    i = i2;
+  }
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(~0u, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(~0u, v, o));
+  return v;
+}
+
+__device__ __forceinline__ void warp_argmax(float& v, int& i) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) argmax_merge(v, i, __shfl_xor_sync(~0u, v, o), __shfl_xor_sync(~0u, i, o));
+}
+
+// Block reductions: every thread gets the result; the scratch is free again on return.
+__device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int* redi) {
+  warp_argmax(v, i);
+  if ((threadIdx.x & 31) == 0) {
+    redf[threadIdx.x >> 5] = v;
+    redi[threadIdx.x >> 5] = i;
+  }
+  __syncthreads();
+  v = redf[0];
+  i = redi[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) argmax_merge(v, i, redf[w], redi[w]);
+  __syncthreads();
+}
+
+__device__ __forceinline__ float block_sum(float v, float* redf) {
+  v = warp_sum(v);
+  if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float s = 0.f;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) s += redf[w];
+  __syncthreads();
+  return s;
+}
+
+__device__ __forceinline__ float block_max(float v, float* redf) {
+  v = warp_max(v);
+  if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float s = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) s = fmaxf(s, redf[w]);
+  __syncthreads();
+  return s;
+}
+
+
+// ------------------------------------------------------------------------------------------
+// In-place fp32 values over a staged (z_p, z_q) slice: for fp32 input a token's value takes its
+// z_p slot; for bf16 input its low half goes to the token's z_p slot and its high half to its z_q
+// slot, so no token's slots are shared with another's.
+__device__ __forceinline__ void st8_value(float* zp, float* /*zq*/, int i0, const float v[8]) {
+  reinterpret_cast<float4*>(zp + i0)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(zp + i0)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+__device__ __forceinline__ void st8_value(__nv_bfloat16* zp, __nv_bfloat16* zq, int i0, const float v[8]) {
+  uint32_t w[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(v[e]);
+  *reinterpret_cast<uint4*>(zp + i0) = make_uint4(__byte_perm(w[0], w[1], 0x5410), __byte_perm(w[2], w[3], 0x5410),
+                                                 __byte_perm(w[4], w[5], 0x5410), __byte_perm(w[6], w[7], 0x5410));
+  *reinterpret_cast<uint4*>(zq + i0) = make_uint4(__byte_perm(w[0], w[1], 0x7632), __byte_perm(w[2], w[3], 0x7632),
+                                                 __byte_perm(w[4], w[5], 0x7632), __byte_perm(w[6], w[7], 0x7632));
+}
+
+__device__ __forceinline__ void ld8_value(const float* zp, const float* /*zq*/, int i0, float v[8]) { ld8(zp + i0, v); }
+
+__device__ __forceinline__ void ld8_value(const __nv_bfloat16* zp, const __nv_bfloat16* zq, int i0, float v[8]) {
+  const uint4 lo = *reinterpret_cast<const uint4*>(zp + i0);
+  const uint4 hi = *reinterpret_cast<const uint4*>(zq + i0);
+  const uint32_t l[4] = {lo.x, lo.y, lo.z, lo.w}, h[4] = {hi.x, hi.y, hi.z, hi.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    v[2 * k] = __uint_as_float(__byte_perm(l[k], h[k], 0x5410));
+    v[2 * k + 1] = __uint_as_float(__byte_perm(l[k], h[k], 0x7632));
+  }
+}
+
+__device__ __forceinline__ float ld1_value(const float* zp, const float* /*zq*/, int i) { return zp[i]; }
+
+__device__ __forceinline__ float ld1_value(const __nv_bfloat16* zp, const __nv_bfloat16* zq, int i) {
+  const uint32_t lo = reinterpret_cast<const uint16_t*>(zp)[i];
+  const uint32_t hi = reinterpret_cast<const uint16_t*>(zq)[i];
+  return __uint_as_float((hi << 16) | lo);
+}
+
+}  // namespace dev
+}  // namespace dcd

@@ -6,10 +6,30 @@
 
 namespace dcd {
 
-// Workspace layout: a 256-byte header (word 0 = device error bits, word 1 = the row
-// kernel's work counter, both zeroed at the start of every call), then one RowRecord per
-// row g = b * N + n.
+// Workspace layout, all in the caller's buffer:
+//   [WsHeader, 256 B][Job x R][RowRecord x R][slot x R]
+// The header and the job list are zeroed at the start of every call; records and slots are
+// written before they are read.  R = B * N rows; a slot (SlotHead + one PiecePart per residual
+// piece) holds the chain state of a row whose first sibling was rejected.
 constexpr size_t kWorkspaceHeader = 256;
+
+struct WsHeader {
+  uint32_t err;        // DCD_DEVERR_* bits of the call (read by dcd_get_device_error)
+  uint32_t work;       // rows claimed by the streaming kernel
+  uint32_t job_alloc;  // residual passes created
+  uint32_t job_head;   // first pass that may still have unclaimed pieces
+  uint32_t nslots;     // rows handed to residual passes
+  uint32_t reserved[59];
+};
+static_assert(sizeof(WsHeader) == kWorkspaceHeader, "WsHeader layout");
+
+struct Job {            // one residual pass of one row
+  int32_t slot;         // the row's slot
+  int32_t J;            // the pass (rejections so far, >= 1); 0 until published
+  uint32_t next_piece;  // pieces claimed
+  uint32_t done;        // pieces finished
+};
+static_assert(sizeof(Job) == 16, "Job layout");
 
 struct RowRecord {
   int32_t acc_child;   // accepted child node id, -1 if none
@@ -18,6 +38,24 @@ struct RowRecord {
   int32_t reserved;
 };
 static_assert(sizeof(RowRecord) == 16, "RowRecord layout");
+
+struct SlotHead {  // chain state of a handed-over row
+  int32_t g, m;    // row, children of its node
+  float M, S, Mp;  // max CD score, normaliser sum 2^((s' - M) k2), expert max
+  float c, D;      // c_J and D_J of the residual r_J = max(0, pi - c_J q) / D_J last computed
+  int32_t degen;   // a pass found no residual mass
+  uint32_t status;
+  int32_t pad[7];
+};
+static_assert(sizeof(SlotHead) == 64, "SlotHead layout");
+
+struct PiecePart {  // one piece's share of a residual pass
+  float z;          // sum of max(0, pi - c_J q) over the piece
+  float key;        // best race key of the piece's blocks (last pass only)
+  int32_t blk;      // its block
+  int32_t timed_out;
+};
+static_assert(sizeof(PiecePart) == 16, "PiecePart layout");
 
 struct ScoreArgs {
   const void* zp;
@@ -35,11 +73,17 @@ struct ScoreArgs {
   float* cd_logprob;  // may be null
   int32_t* cd_argmax; // may be null
   float* cd_lse;      // may be null
+  WsHeader* hdr;
+  Job* jobs;
   RowRecord* rec;
-  uint32_t* err;
+  unsigned char* slots;
   int32_t force_stages;   // 0 = automatic, else the ring depth to use (tests / tuning)
   int32_t force_plain;    // 1 = plain loads instead of bulk async copies
 };
+
+// Residual pieces per pass and slot bytes per row for a vocabulary of V tokens.
+int residual_pieces(int64_t V, int dtype);
+size_t slot_bytes(int64_t V, int dtype);
 
 cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream);
 

@@ -1,32 +1,41 @@
 // dcd_rows.cu -- the streaming kernels of the CD verification step on sm_103a.
 //
-// score_rows_kernel: a persistent grid (a few CTAs per SM).  Each CTA claims whole
-//   tree-node rows g = b * N + n from a work counter, in node-major order (every
-//   sequence's node 0, then every node 1, ...), so internal nodes -- the rows that
-//   may need extra passes -- come first and leaves last.  A row is streamed through
-//   a ring of 32 KB shared-memory stages filled by bulk
-//   asynchronous copies that complete on one mbarrier per stage; thread 0 refills a
-//   stage as soon as the block has consumed it, so a ring's worth of the row is
-//   always in flight.
-//   The "stats" pass computes the CD score s' = (1 + alpha) z_p - alpha z_q (Eq. 1;
-//   the two log-softmax shifts are constant per row and cancel in the normaliser)
-//   on the plausibility set P_beta of Sec. 2.1; every lane keeps an online max, a
-//   sum of 2^((s' - max) k2) (k2 = log2(e) / T) rescaled when its max grows, and
-//   its argmax, reduced over the block at the end of the row.  Rows whose terminal
-//   draw races over pi_CD itself (sampled leaves) also keep, per 256-token block,
-//   the block max and sum, i.e. the block masses of pi_CD.  With beta > 0 a "max"
-//   pass over z_p comes first.  Sampled rows then test their children in ascending node id (Algorithm 1
-//   on sibling lists); each rejection streams the row once more (z_p, z_q and q) to
-//   get the next residual's mass Z_j, recomputing r_j(x) = max(0, r_{j-1}(x) - q(x))
-//   / Z_j token by token from pi_CD(x), q(x) and the earlier Z's, so nothing per
-//   token is stored between passes.  Rows that take more than one pass are read with
-//   an L2 evict-last policy, so their later passes hit L2 and HBM is read once.  A
-//   node without an accepted child draws its terminal token by a two-level
-//   exponential race: a 256-token block by its mass, then a token of that block,
-//   whose 256 values are re-read directly.
+// score_rows_kernel: a persistent grid (a few CTAs per SM) with two kinds of work.
+//
+//  * Rows.  A CTA claims whole tree-node rows g = b * N + n from a work counter, in
+//    node-major order (every sequence's node 0, then every node 1, ...), so internal
+//    nodes -- the rows that may start residual work -- come first and leaves last.  A
+//    row is streamed through a ring of 32 KB shared-memory stages filled by bulk
+//    asynchronous copies that complete on one mbarrier per stage; thread 0 refills a
+//    stage as soon as the block has consumed it.  The "stats" pass computes the CD score
+//    s' = (1 + alpha) z_p - alpha z_q (Eq. 1; the two log-softmax shifts are constant per
+//    row and cancel in the normaliser) on the plausibility set P_beta of Sec. 2.1; every
+//    lane keeps an online max, a sum of 2^((s' - max) k2) (k2 = log2(e) / T) rescaled when
+//    its max grows, and its argmax, reduced over the block at the end of the row.  With
+//    beta > 0 a "max" pass over z_p comes first.  Rows whose terminal draw races over
+//    pi_CD itself (sampled leaves) also keep per-256-token block maxima and sums, i.e. the
+//    block masses of pi_CD.  The greedy rule, the first sibling test of the sampled rule
+//    and the leaf race then finish the row.
+//
+//  * Residual pieces.  After a rejected sibling, Algorithm 1 (generalised to sibling
+//    lists) needs the next residual over the whole vocabulary.  With c_0 = 0, D_0 = 1 the
+//    j-th residual is r_j = max(0, pi - c_j q) / D_j, where c_j = c_{j-1} + D_{j-1} and
+//    D_j = sum_x max(0, pi(x) - c_j q(x)) (induction on j from r_j = normalise(max(0,
+//    r_{j-1} - q))), so a pass needs only two scalars from the one before.  A row that
+//    needs a pass is handed to a job list; the pass is split into pieces of 4096 tokens
+//    that any CTA claims before taking a new row.  Each piece writes its partial sum (and,
+//    in the pass after the last sibling, its best race key) to its own slot; the CTA that
+//    finishes a pass's last piece (an atomic ticket, no waiting) sums the slots in a fixed
+//    order, tests the next sibling, and either queues the next pass or runs the terminal
+//    race.  Nothing waits on another CTA, so a CTA leaves when no piece is claimable and no
+//    row is left: work queued later belongs to a CTA that is still running.
+//
+//  A node without an accepted child draws its terminal token by a two-level exponential
+//  race: a 256-token block by its mass, then a token of that block, whose 256 values are
+//  re-read directly.
 // tree_walk_kernel: one thread per sequence follows the accepted children.
-// terminal_residual_kernel: one block per sequence rebuilds the distribution its
-//   bonus token was drawn from (test output only).
+// terminal_residual_kernel: one block per sequence rebuilds the distribution its bonus
+//   token was drawn from (test output only).
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -37,239 +46,60 @@
 #include <mutex>
 
 #include "dcd.h"
+#include "dcd_device.cuh"
 #include "dcd_internal.h"
 
 namespace dcd {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kWarps = kThreads / 32;
-constexpr int kStageBytes = 32 * 1024;            // bytes per ring stage
-constexpr int kRaceBlock = 256;                   // tokens per block of the two-level terminal race
+using namespace dev;
+
+#ifndef DCD_STAGE_KIB
+#define DCD_STAGE_KIB 32
+#endif
+constexpr int kStageBytes = DCD_STAGE_KIB * 1024;  // bytes per ring stage
 constexpr int kMaxStages = 8;
 constexpr size_t kSmemMax = 227 * 1024;
 constexpr size_t kSmemPerSm = 228 * 1024;
-constexpr long long kWaitCycles = 4000000000ll;  // about two seconds at the boost clock
-constexpr float kLog2e = 1.4426950408889634f;
 
-enum PassKind { kPassMax = 0, kPassStats = 1, kPassRes = 2 };
-
-// ------------------------------------------------------------------------------------------
-// PTX wrappers: mbarrier, L2 cache policies and bulk asynchronous global->shared copies.
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void fence_mbar_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile(
-      "{\n\t.reg .b64 st;\n\t"
-      "mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}" ::"r"(smem_addr(bar)),
-      "r"(bytes)
-      : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.b32 %0, 1, 0, p;\n\t}"
-      : "=r"(done)
-      : "r"(smem_addr(bar)), "r"(parity)
-      : "memory");
-  return done != 0;
-}
-
-// Bounded wait: gives up after kWaitCycles and reports false.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
-  const long long start = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - start > kWaitCycles) return false;
-  }
-  return true;
-}
-
-__device__ __forceinline__ uint64_t l2_policy_evict_last() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-
-__device__ __forceinline__ uint64_t l2_policy_evict_first() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], "
-      "%4;" ::"r"(smem_addr(dst)),
-      "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
-      : "memory");
-}
-
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ float lg2(float x) {
-  float y;
-  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-// ------------------------------------------------------------------------------------------
-// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32->64 products
-// with the published multipliers, the key advanced by the published Weyl increments.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
-    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-    k0 += 0x9E3779B9u;
-    k1 += 0xBB67AE85u;
-  }
-  return c;
-}
-
-__device__ __forceinline__ uint4 philox_block(uint64_t seed, uint64_t off, uint32_t c0, uint32_t c1) {
-  return philox4x32_10(make_uint4(c0, c1, static_cast<uint32_t>(off), static_cast<uint32_t>(off >> 32)),
-                       static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
-}
-
-__device__ __forceinline__ uint32_t word_of(const uint4& w, int i) {
-  return i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w;
-}
-
-// 32-bit word -> uniform in (0, 1): ((w >> 9) + 1/2) 2^-23, exact in fp32.
-__device__ __forceinline__ float u01(uint32_t w) {
-  return (__uint2float_rn(w >> 9) + 0.5f) * 1.1920928955078125e-07f;
-}
-
-// Race key in log2 units: log2 r - log2(-log2 u) orders tokens exactly as ln r - ln(-ln u)
-// (the two differ by a positive factor and a constant).
-__device__ __forceinline__ float race_key(float log2_mass, uint32_t word) {
-  return log2_mass - lg2(-lg2(u01(word)));
-}
-
-// ------------------------------------------------------------------------------------------
-// Element access: 8 consecutive tokens as fp32 (16 B of bf16 or 32 B of fp32).
-__device__ __forceinline__ void ld8(const float* p, float v[8]) {
-  const float4 a = reinterpret_cast<const float4*>(p)[0];
-  const float4 b = reinterpret_cast<const float4*>(p)[1];
-  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-}
-
-__device__ __forceinline__ void ld8(const __nv_bfloat16* p, float v[8]) {
-  const uint4 a = *reinterpret_cast<const uint4*>(p);
-  v[0] = __uint_as_float(a.x << 16); v[1] = __uint_as_float(a.x & 0xffff0000u);
-  v[2] = __uint_as_float(a.y << 16); v[3] = __uint_as_float(a.y & 0xffff0000u);
-  v[4] = __uint_as_float(a.z << 16); v[5] = __uint_as_float(a.z & 0xffff0000u);
-  v[6] = __uint_as_float(a.w << 16); v[7] = __uint_as_float(a.w & 0xffff0000u);
-}
-
-__device__ __forceinline__ float ld1(const float* p, int64_t i) { return p[i]; }
-__device__ __forceinline__ float ld1(const __nv_bfloat16* p, int64_t i) { return __bfloat162float(p[i]); }
-
-// ------------------------------------------------------------------------------------------
-// Reductions.
-__device__ __forceinline__ void argmax_merge(float& v, int& i, float v2, int i2) {
-  if (v2 > v || (v2 == v && i2 < i)) {
-    v = v2;
-    i = i2;
-  }
-}
-
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(~0u, v, o);
-  return v;
-}
-
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(~0u, v, o));
-  return v;
-}
-
-__device__ __forceinline__ void warp_argmax(float& v, int& i) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) argmax_merge(v, i, __shfl_xor_sync(~0u, v, o), __shfl_xor_sync(~0u, i, o));
-}
-
-// Block reductions: every thread gets the result; the scratch is free again on return.
-__device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int* redi) {
-  warp_argmax(v, i);
-  if ((threadIdx.x & 31) == 0) {
-    redf[threadIdx.x >> 5] = v;
-    redi[threadIdx.x >> 5] = i;
-  }
-  __syncthreads();
-  v = redf[0];
-  i = redi[0];
-#pragma unroll
-  for (int w = 1; w < kWarps; ++w) argmax_merge(v, i, redf[w], redi[w]);
-  __syncthreads();
-}
-
-__device__ __forceinline__ float block_sum(float v, float* redf) {
-  v = warp_sum(v);
-  if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
-  __syncthreads();
-  float s = 0.f;
-#pragma unroll
-  for (int w = 0; w < kWarps; ++w) s += redf[w];
-  __syncthreads();
-  return s;
-}
-
-__device__ __forceinline__ float block_max(float v, float* redf) {
-  v = warp_max(v);
-  if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
-  __syncthreads();
-  float s = -INFINITY;
-#pragma unroll
-  for (int w = 0; w < kWarps; ++w) s = fmaxf(s, redf[w]);
-  __syncthreads();
-  return s;
-}
+enum PassKind { kPassMax = 0, kPassStats = 1 };
+enum WorkKind { kWorkNone = 0, kWorkRow = 1, kWorkPiece = 2 };
 
 // ------------------------------------------------------------------------------------------
 struct SParams {
   ScoreArgs a;
   int32_t nst;           // ring depth (stages of kStageBytes)
-  int32_t tok_a;         // tokens per stage in the max and stats passes (z_p, z_q)
-  int32_t tok_r;         // tokens per stage in residual passes (z_p, z_q, q)
+  int32_t tok_a;         // tokens per stage in row passes (z_p, then z_q)
+  int32_t tok_r;         // tokens per residual piece (z_p, z_q, then q)
+  int32_t npieces;       // pieces per residual pass
   int32_t bulk;          // 1: bulk asynchronous copies, 0: plain loads
   int32_t nblk;          // race blocks per row, ceil(V / 256)
   int32_t meta_offset;   // byte offsets into dynamic shared memory
   int32_t blk_offset;
   int32_t stage_offset;
-  uint32_t* work;        // row counter, zeroed before the launch
+  int32_t slot_bytes;
+  WsHeader* hdr;         // counters, zeroed before the launch
+  Job* jobs;             // residual passes (zeroed before the launch)
+  unsigned char* slots;  // per handed-over row: SlotHead + npieces PieceParts
 };
 
-// Row state shared by the block (written by one thread, read after a barrier).
+// Row / piece state shared by the block (written by one thread, read after a barrier).
 struct RowShared {
-  int32_t next;      // the next claimed work item
+  int32_t next;      // the next claimed row item
+  int32_t kind;      // WorkKind of the current work
+  int32_t item;      // row item or job index
+  int32_t piece;     // piece index
   int32_t m;         // children of the row's node
   uint32_t status;   // DCD_DEVERR_* bits
-  int32_t accept;    // outcome of the current sibling test
-  int32_t term;      // terminal token
-  int32_t pad[3];
+  int32_t accept;    // outcome of a sibling test
+  int32_t term;      // terminal token, or winning race block
+  int32_t last;      // this CTA finished a pass's last piece
+  int32_t degen;     // a pass found no residual mass left
+  int32_t slot;      // slot of the handed-over row
+  int32_t J;         // residual pass index (rejections so far)
+  int32_t g;         // row of the piece
+  float M, S, Mp, c, D;
+  int32_t pad[2];
 };
 
 template <typename TIn>
@@ -279,7 +109,7 @@ struct Stage {
   float* q;
 };
 
-// A stage holds `tok` tokens of z_p, then of z_q, then (residual passes) of q.
+// A stage holds `tok` tokens of z_p, then of z_q, then (residual pieces) of q.
 template <typename TIn>
 __device__ __forceinline__ Stage<TIn> stage_at(unsigned char* base, int s, int tok) {
   Stage<TIn> st;
@@ -287,6 +117,51 @@ __device__ __forceinline__ Stage<TIn> stage_at(unsigned char* base, int s, int t
   st.zq = st.zp + tok;
   st.q = reinterpret_cast<float*>(st.zq + tok);
   return st;
+}
+
+__device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
+  return *reinterpret_cast<const volatile uint32_t*>(p);
+}
+__device__ __forceinline__ int32_t ld_volatile(const int32_t* p) {
+  return *reinterpret_cast<const volatile int32_t*>(p);
+}
+
+__device__ __forceinline__ SlotHead* slot_head(const SParams& sp, int s) {
+  return reinterpret_cast<SlotHead*>(sp.slots + static_cast<size_t>(s) * sp.slot_bytes);
+}
+
+__device__ __forceinline__ PiecePart* slot_parts(const SParams& sp, int s) {
+  return reinterpret_cast<PiecePart*>(sp.slots + static_cast<size_t>(s) * sp.slot_bytes + sizeof(SlotHead));
+}
+
+// Publishes residual pass J of slot s (thread 0 of the creating CTA).
+__device__ __forceinline__ void create_job(const SParams& sp, int s, int J) {
+  const uint32_t k = atomicAdd(&sp.hdr->job_alloc, 1u);
+  Job* job = &sp.jobs[k];
+  job->slot = s;
+  job->next_piece = 0u;
+  job->done = 0u;
+  __threadfence();
+  *reinterpret_cast<volatile int32_t*>(&job->J) = J;
+}
+
+// The sibling test of child `node` (token t): accept iff u <= r(t) / q(t) with
+// r = max(0, pi - c q) / D, or r = q once a pass found no residual mass (`degen`).  One thread.
+template <typename TIn>
+__device__ bool sibling_test(const ScoreArgs& p, int b, int node, int t, const TIn* zp_row, const TIn* zq_row,
+                             const float* q_row, float c1, float alpha, bool masked, float Mp, float logb, float k2,
+                             float Mk2, float invS, float c, float D, bool degen) {
+  const bool ok = t >= 0 && t < p.V;
+  const float z = ok ? ld1(zp_row, t) : 0.f;
+  const float zz = ok ? ld1(zq_row, t) : 0.f;
+  const float qt = ok ? q_row[t] : 0.f;
+  const bool in = ok && (!masked || (z - Mp >= logb));
+  const float pit = in ? ex2(fmaf(fmaf(c1, z, -alpha * zz), k2, -Mk2)) * invS : 0.f;
+  const float rt = degen ? qt : fmaxf(pit - c * qt, 0.f) / D;
+  const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
+  const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * p.N + node);
+  const float u = u01(philox_block(p.seed, p.offset, G, 0u).x);
+  return u <= ratio;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -298,7 +173,6 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   const int64_t V = p.V;
   const int R = p.B * N;
   const int nch_a = static_cast<int>((V + sp.tok_a - 1) / sp.tok_a);  // chunks of a max / stats pass
-  const int nch_r = static_cast<int>((V + sp.tok_r - 1) / sp.tok_r);  // chunks of a residual pass
 
   extern __shared__ __align__(128) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);             // [kMaxStages]
@@ -310,28 +184,327 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   float* czp = reinterpret_cast<float*>(ktok + N);                // [N] z_p at those tokens
   float* czq = czp + N;                                           // [N] z_q at those tokens
   float* cq = czq + N;                                            // [N] q at those tokens
-  float* invZ = cq + N;                                           // [N] 1/Z_j (0 marks Z_j = 0)
   float* bmax = reinterpret_cast<float*>(smem + sp.blk_offset);   // [nblk] block max of s'
   float* bsum = bmax + sp.nblk;                                   // [nblk] block sums
-  float* bres = bsum + sp.nblk;                                   // [nblk] final residual block masses
-  float* bq = bres + sp.nblk;                                     // [nblk] block masses of q
   unsigned char* ring = smem + sp.stage_offset;
 
   if (tid == 0) {
     for (int s = 0; s < sp.nst; ++s) mbar_init(&full[s], 1);
     fence_mbar_init();
-    rs->next = static_cast<int32_t>(atomicAdd(sp.work, 1u));
+    rs->next = static_cast<int32_t>(atomicAdd(&sp.hdr->work, 1u));
   }
   __syncthreads();
   const uint64_t pol_last = l2_policy_evict_last();
   const uint64_t pol_first = l2_policy_evict_first();
   uint32_t seq = 0;  // ring items consumed by this CTA so far (identical in every thread)
 
+  // Lists the children of node n of sequence b (warp `w`), ascending id, and their count.
+  auto scan_children = [&](int b, int n, int w) {
+    if (warp == w) {
+      const int32_t* par = p.parents + static_cast<int64_t>(b) * N;
+      const int32_t* tok = p.tokens + static_cast<int64_t>(b) * N;
+      int count = 0;
+      for (int base = n + 1; base < N; base += 32) {
+        const int c = base + lane;
+        const bool is = c < N && par[c] == n;
+        const unsigned msk = __ballot_sync(~0u, is);
+        if (is) {
+          const int pos = count + __popc(msk & ((1u << lane) - 1u));
+          kids[pos] = c;
+          ktok[pos] = tok[c];
+        }
+        count += __popc(msk);
+      }
+      if (lane == 0) rs->m = count;
+    }
+  };
+
+  // Waits for ring item `sq`, then fills a ragged or unaligned remainder with plain loads.
+  auto wait_stage = [&](uint32_t sq, const Stage<TIn>& st, const TIn* zp_row, const TIn* zq_row,
+                        const float* q_row, int64_t x0, int clen, bool with_zq, bool with_q, bool& timed_out) {
+    const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
+    const uint32_t parity = (sq / static_cast<uint32_t>(sp.nst)) & 1u;
+    if (!mbar_wait_bounded(&full[s], parity)) timed_out = true;
+    const int zfirst =
+        sp.bulk ? ((clen * static_cast<int>(sizeof(TIn))) & ~15) / static_cast<int>(sizeof(TIn)) : 0;
+    const int qfirst = sp.bulk ? ((clen * 4) & ~15) / 4 : 0;
+    if (zfirst < clen || (with_q && qfirst < clen)) {
+      for (int i = zfirst + tid; i < clen; i += kThreads) {
+        st.zp[i] = zp_row[x0 + i];
+        if (with_zq) st.zq[i] = zq_row[x0 + i];
+      }
+      if (with_q)
+        for (int i = qfirst + tid; i < clen; i += kThreads) st.q[i] = q_row[x0 + i];
+      __syncthreads();
+    }
+  };
+
   for (;;) {
-    const int item = rs->next;
-    __syncthreads();  // every thread has read the claim before thread 0 replaces it
-    if (item >= R) break;
-    if (tid == 0) rs->next = static_cast<int32_t>(atomicAdd(sp.work, 1u));  // used by the next row
+    // ---- next work: a residual piece if one can be claimed, else the next row
+    if (tid == 0) {
+      int kind = kWorkNone, job = -1, piece = 0;
+      const uint32_t alloc = ld_volatile(&sp.hdr->job_alloc);
+      for (uint32_t k = ld_volatile(&sp.hdr->job_head); k < alloc; ++k) {
+        if (ld_volatile(&sp.jobs[k].J) == 0) break;  // not yet published
+        const uint32_t pc = atomicAdd(&sp.jobs[k].next_piece, 1u);
+        if (pc < static_cast<uint32_t>(sp.npieces)) {
+          job = static_cast<int>(k);
+          piece = static_cast<int>(pc);
+          break;
+        }
+        atomicMax(&sp.hdr->job_head, k + 1u);
+      }
+      if (job >= 0) {
+        kind = kWorkPiece;
+        rs->item = job;
+        rs->piece = piece;
+      } else if (rs->next < R) {
+        kind = kWorkRow;
+        rs->item = rs->next;
+        rs->next = static_cast<int32_t>(atomicAdd(&sp.hdr->work, 1u));
+      }
+      rs->kind = kind;
+    }
+    __syncthreads();
+    const int kind = rs->kind;
+    if (kind == kWorkNone) break;
+
+    if (kind == kWorkPiece) {
+      // ================= one piece of residual pass J of a handed-over row
+      if (tid == 0) {
+        __threadfence();  // the job and its slot were written before J was published
+        const Job* job = &sp.jobs[rs->item];
+        const int s = ld_volatile(&job->slot);
+        const SlotHead* sh = slot_head(sp, s);
+        rs->slot = s;
+        rs->J = ld_volatile(&job->J);
+        rs->g = sh->g;
+        rs->m = sh->m;
+        rs->M = sh->M;
+        rs->S = sh->S;
+        rs->Mp = sh->Mp;
+        rs->c = sh->c + sh->D;  // c_J = c_{J-1} + D_{J-1}
+        rs->status = sh->status;
+      }
+      __syncthreads();
+      const int64_t g = rs->g;
+      const int J = rs->J, m = rs->m, piece = rs->piece;
+      const int b = static_cast<int>(g / N);
+      const float alpha = p.alpha[b];
+      const float beta = p.beta ? p.beta[b] : 0.f;
+      const float T = p.temp[b];
+      const bool masked = beta > 0.f;
+      const float k2 = kLog2e / T;
+      const float c1 = 1.f + alpha;
+      const float logb = masked ? logf(beta) : -INFINITY;
+      const float M = rs->M, invS = 1.f / rs->S, Mp = rs->Mp, cJ = rs->c;
+      const float Mk2 = M * k2;
+      const bool race = J == m;  // the pass after the last sibling also ranks race blocks
+      const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
+      const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
+      const float* q_row = p.q + g * p.ldq;
+      const int64_t x0 = static_cast<int64_t>(piece) * sp.tok_r;
+      const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
+      const uint32_t sq = seq;
+      const int s_idx = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
+      const Stage<TIn> st = stage_at<TIn>(ring, s_idx, sp.tok_r);
+      if (tid == 0) {
+        uint64_t* bar = &full[s_idx];
+        const uint32_t zb = sp.bulk ? static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u : 0u;
+        const uint32_t qb = sp.bulk ? static_cast<uint32_t>(clen * 4) & ~15u : 0u;
+        mbar_arrive_expect_tx(bar, 2u * zb + qb);
+        if (zb) {
+          bulk_g2s(st.zp, zp_row + x0, zb, bar, pol_last);
+          bulk_g2s(st.zq, zq_row + x0, zb, bar, pol_last);
+        }
+        if (qb) bulk_g2s(st.q, q_row + x0, qb, bar, pol_last);
+      }
+      bool timed_out = false;
+      wait_stage(sq, st, zp_row, zq_row, q_row, x0, clen, true, true, timed_out);
+      float zl = 0.f, bk = -INFINITY;
+      int bb = INT_MAX;
+      for (int kb = warp; kb * kRaceBlock < sp.tok_r; kb += kWarps) {
+        if (kb * kRaceBlock >= clen) break;  // warp-uniform
+        const int i0 = kb * kRaceBlock + lane * 8;
+        float zp[8], zq[8], qv[8];
+        ld8(st.zp + i0, zp);
+        ld8(st.zq + i0, zq);
+        ld8(st.q + i0, qv);
+        float part = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const bool valid = i0 + e < clen;
+          const bool in = valid && (!masked || (zp[e] - Mp >= logb));
+          const float pit = in ? ex2(fmaf(fmaf(c1, zp[e], -alpha * zq[e]), k2, -Mk2)) * invS : 0.f;
+          part += valid ? fmaxf(pit - cJ * qv[e], 0.f) : 0.f;
+        }
+        zl += part;
+        if (race) {
+          const float R_b = warp_sum(part);
+          if (lane == 0 && R_b > 0.f) {
+            const uint32_t kabs = static_cast<uint32_t>(x0 / kRaceBlock) + static_cast<uint32_t>(kb);
+            const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (kabs >> 2));
+            const float key = race_key(lg2(R_b), word_of(w, static_cast<int>(kabs & 3)));
+            if (key > bk) {
+              bk = key;
+              bb = static_cast<int>(kabs);
+            }
+          }
+        }
+      }
+      seq = sq + 1;
+      const float zsum = block_sum(zl, redf);  // also frees the stage (all reads are done)
+      block_argmax(bk, bb, redf, redi);
+      if (tid == 0) {
+        PiecePart pp;
+        pp.z = zsum;
+        pp.key = bk;
+        pp.blk = bb;
+        pp.timed_out = timed_out ? 1 : 0;
+        slot_parts(sp, rs->slot)[piece] = pp;
+        __threadfence();
+        const uint32_t t = atomicAdd(&sp.jobs[rs->item].done, 1u);
+        rs->last = t + 1u == static_cast<uint32_t>(sp.npieces) ? 1 : 0;
+      }
+      __syncthreads();
+      if (!rs->last) continue;
+
+      // ================= the pass is complete: next sibling test, next pass or terminal race
+      const int n = static_cast<int>(g % N);
+      scan_children(b, n, 0);
+      if (tid == 0) {
+        __threadfence();  // every piece's part was written before its ticket
+        SlotHead* sh = slot_head(sp, rs->slot);
+        const PiecePart* parts = slot_parts(sp, rs->slot);
+        float DJ = 0.f, K = -INFINITY;
+        int kstar = INT_MAX;
+        uint32_t st2 = sh->status;
+        for (int k = 0; k < sp.npieces; ++k) {
+          DJ += parts[k].z;
+          argmax_merge(K, kstar, parts[k].key, parts[k].blk);
+          if (parts[k].timed_out) st2 |= DCD_DEVERR_TIMEOUT;
+        }
+        bool degen = sh->degen != 0;
+        float c = sh->c, D = sh->D;
+        if (DJ > 0.f) {
+          c = cJ;
+          D = DJ;
+        } else {
+          degen = true;  // r_{J-1} == q in exact arithmetic: r_J is taken as q from here on
+        }
+        // test the remaining siblings; after a pass without residual mass no pass is needed
+        int acc = -1;
+        bool queued = false;
+        for (int j = J; j < m; ++j) {
+          if (sibling_test<TIn>(p, b, kids[j], ktok[j], zp_row, zq_row, q_row, c1, alpha, masked, Mp, logb, k2, Mk2,
+                                invS, c, D, degen)) {
+            acc = kids[j];
+            break;
+          }
+          if (!degen) {
+            sh->c = c;
+            sh->D = D;
+            sh->degen = 0;
+            sh->status = st2;
+            create_job(sp, rs->slot, j + 1);
+            queued = true;
+            break;
+          }
+        }
+        rs->accept = queued ? -2 : acc;
+        rs->term = kstar;  // the winning race block when this pass ranked them
+        rs->status = st2;
+        rs->c = c;
+        rs->D = D;
+        rs->degen = degen ? 1 : 0;
+      }
+      __syncthreads();
+      if (rs->accept == -2) continue;  // the next pass is queued
+      const int acc = rs->accept;
+      int term = -1;
+      if (acc < 0) {
+        // every sibling rejected: terminal draw from r_m, or from q after a pass without mass
+        const bool degen = rs->degen != 0;
+        const float c = rs->c, D = rs->D;
+        int kstar = rs->term;
+        if (degen) {
+          // block masses of q, streamed by this CTA alone (rare: a residual without mass)
+          float bk2 = -INFINITY;
+          int bb2 = INT_MAX;
+          for (int kb = warp; kb < sp.nblk; kb += kWarps) {
+            const int64_t xb = static_cast<int64_t>(kb) * kRaceBlock + lane * 8;
+            float part = 0.f;
+            for (int e = 0; e < 8; ++e)
+              if (xb + e < V) part += q_row[xb + e];
+            const float R_b = warp_sum(part);
+            if (lane == 0 && R_b > 0.f) {
+              const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
+                                           0x80000000u | (static_cast<uint32_t>(kb) >> 2));
+              const float key = race_key(lg2(R_b), word_of(w, kb & 3));
+              if (key > bk2) {
+                bk2 = key;
+                bb2 = kb;
+              }
+            }
+          }
+          block_argmax(bk2, bb2, redf, redi);
+          kstar = bb2;
+        }
+        __syncthreads();
+        if (warp == 0) {
+          float tk = -INFINITY;
+          int tx = INT_MAX;
+          if (kstar != INT_MAX) {
+            const int64_t xb = static_cast<int64_t>(kstar) * kRaceBlock + lane * 8;
+            const uint4 wa =
+                philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 1u + static_cast<uint32_t>(xb >> 2));
+            const uint4 wb =
+                philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 2u + static_cast<uint32_t>(xb >> 2));
+            const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const int64_t x = xb + e;
+              if (x < V) {
+                const float qe = q_row[x];
+                float v;
+                if (degen) {
+                  v = qe;
+                } else {
+                  const float z = ld1(zp_row, x);
+                  const bool in = !masked || (z - Mp >= logb);
+                  const float pit = in ? ex2(fmaf(fmaf(c1, z, -alpha * ld1(zq_row, x)), k2, -Mk2)) * invS : 0.f;
+                  v = fmaxf(pit - c * qe, 0.f) / D;
+                }
+                if (v > 0.f) {
+                  const float key = race_key(lg2(v), w[e]);
+                  if (key > tk) {
+                    tk = key;
+                    tx = static_cast<int>(x);
+                  }
+                }
+              }
+            }
+          }
+          warp_argmax(tk, tx);
+          if (lane == 0) rs->term = tx;
+        }
+        __syncthreads();
+        term = rs->term;
+      }
+      if (tid == 0) {
+        RowRecord r;
+        r.acc_child = acc;
+        r.term_token = acc < 0 ? term : -1;
+        r.status = rs->status;
+        r.reserved = 0;
+        p.rec[g] = r;
+      }
+      __syncthreads();
+      continue;
+    }
+
+    // ================= a row
+    const int item = rs->item;
     const int b = item % p.B, n = item / p.B;  // node-major order
     const int64_t g = static_cast<int64_t>(b) * N + n;
     const float alpha = p.alpha[b];
@@ -347,82 +520,50 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
     const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
     const float* q_row = sampled ? p.q + g * p.ldq : nullptr;
 
-    // ---- ring items of this row: [max pass if beta > 0] [stats pass] [a residual pass per
-    // rejected child]; thread 0 keeps up to nst items in flight, never past `limit`
+    // ring items of this row: [max pass if beta > 0] [stats pass]; thread 0 keeps up to nst
+    // items in flight
     const int nknown = (masked ? 2 : 1) * nch_a;
     const uint32_t seq0 = seq;
-    auto pass_of = [&](int L) -> int {
-      if (L < nknown) return (masked && L < nch_a) ? kPassMax : kPassStats;
-      return kPassRes;
-    };
-    // token range and stage layout of item L
-    auto chunk_of = [&](int L, int64_t& x0, int& clen, int& tok) {
-      const bool res = L >= nknown;
-      tok = res ? sp.tok_r : sp.tok_a;
-      const int c = res ? (L - nknown) % nch_r : L % nch_a;
-      x0 = static_cast<int64_t>(c) * tok;
-      clen = static_cast<int>((V - x0) < tok ? (V - x0) : tok);
-    };
+    auto pass_of = [&](int L) -> int { return (masked && L < nch_a) ? kPassMax : kPassStats; };
     auto issue = [&](int L, uint64_t pol) {  // thread 0 only
       const uint32_t sq = seq0 + static_cast<uint32_t>(L);
       const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-      int64_t x0;
-      int clen, tok;
-      chunk_of(L, x0, clen, tok);
-      const Stage<TIn> st = stage_at<TIn>(ring, s, tok);
-      const int kind = pass_of(L);
-      uint32_t zb = 0, qb = 0;
-      if (sp.bulk) {
-        zb = static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u;
-        qb = kind == kPassRes ? static_cast<uint32_t>(clen * 4) & ~15u : 0u;
-      }
-      mbar_arrive_expect_tx(&full[s], (kind == kPassMax ? zb : 2u * zb) + qb);
+      const int64_t x0 = static_cast<int64_t>(L % nch_a) * sp.tok_a;
+      const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
+      const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_a);
+      const int kind2 = pass_of(L);
+      const uint32_t zb = sp.bulk ? static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u : 0u;
+      mbar_arrive_expect_tx(&full[s], kind2 == kPassMax ? zb : 2u * zb);
       if (zb) {
         bulk_g2s(st.zp, zp_row + x0, zb, &full[s], pol);
-        if (kind != kPassMax) bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pol);
+        if (kind2 != kPassMax) bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pol);
       }
-      if (qb) bulk_g2s(st.q, q_row + x0, qb, &full[s], pol);
     };
 
-    // thread 0 starts the row's stream at once (rows that may take more than one pass are
-    // kept in L2); warp 1 meanwhile finds the children of node n and checks this row's node
+    // thread 0 starts the row's stream at once (a beta > 0 row keeps its max pass in L2 for the
+    // stats pass; a sampled row with children keeps its logits in L2 for residual pieces); warp
+    // 1 meanwhile lists the children of node n and checks this row
     uint64_t pol = (masked || sampled) ? pol_last : pol_first;
     if (tid == 0) {
       const int first = nknown < sp.nst ? nknown : sp.nst;
       for (int L = 0; L < first; ++L) issue(L, pol);
     }
-    if (warp == 1) {
-      const int32_t* par = p.parents + static_cast<int64_t>(b) * N;
-      const int32_t* tok = p.tokens + static_cast<int64_t>(b) * N;
-      int count = 0;
-      for (int base = n + 1; base < N; base += 32) {
-        const int c = base + lane;
-        const bool is = c < N && par[c] == n;
-        const unsigned msk = __ballot_sync(~0u, is);
-        if (is) {
-          const int pos = count + __popc(msk & ((1u << lane) - 1u));
-          kids[pos] = c;
-          ktok[pos] = tok[c];
-        }
-        count += __popc(msk);
+    scan_children(b, n, 1);
+    if (warp == 1 && lane == 0) {
+      uint32_t st = 0u;
+      const int pp = p.parents[static_cast<int64_t>(b) * N + n];
+      if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
+      if (n > 0) {
+        const int t = p.tokens[static_cast<int64_t>(b) * N + n];
+        if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
       }
-      if (lane == 0) {
-        uint32_t st = 0u;
-        const int pp = par[n];
-        if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
-        if (n > 0) {
-          const int t = tok[n];
-          if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
-        }
-        if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
-          st |= DCD_DEVERR_BAD_PARAM;
-        rs->m = count;
-        rs->status = st;
-      }
+      if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
+        st |= DCD_DEVERR_BAD_PARAM;
+      rs->status = st;
     }
     __syncthreads();
     const int m = rs->m;
-    pol = (masked || (sampled && m > 0)) ? pol_last : pol_first;
+    if (sampled && m == 0 && !masked) pol = pol_first;
     // values at the children's tokens: the loads are issued now and consumed after the stats pass
     float pzp = 0.f, pzq = 0.f, pq = 0.f;
     if (tid < m) {
@@ -434,38 +575,20 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       }
     }
 
-    int limit = nknown;  // items planned so far
-    int L = 0;           // next item to consume
+    int L = 0;  // next item to consume
     bool timed_out = false;
-
-    // Consumes `count` items: waits for each stage, fills a ragged or unaligned remainder with
-    // plain loads, hands the stage to `body`, releases the stage and refills it.
+    // Consumes `count` items: waits for each stage, hands it to `body`, releases and refills it.
     auto run_items = [&](int count, auto&& body) {
       for (int it = 0; it < count; ++it, ++L) {
         const uint32_t sq = seq0 + static_cast<uint32_t>(L);
         const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-        const uint32_t parity = (sq / static_cast<uint32_t>(sp.nst)) & 1u;
-        int64_t x0;
-        int clen, tok;
-        chunk_of(L, x0, clen, tok);
-        const Stage<TIn> st = stage_at<TIn>(ring, s, tok);
-        const int kind = pass_of(L);
-        if (!mbar_wait_bounded(&full[s], parity)) timed_out = true;
-        const int zfirst =
-            sp.bulk ? ((clen * static_cast<int>(sizeof(TIn))) & ~15) / static_cast<int>(sizeof(TIn)) : 0;
-        const int qfirst = sp.bulk ? ((clen * 4) & ~15) / 4 : 0;
-        if (zfirst < clen || (kind == kPassRes && qfirst < clen)) {
-          for (int i = zfirst + tid; i < clen; i += kThreads) {
-            st.zp[i] = zp_row[x0 + i];
-            if (kind != kPassMax) st.zq[i] = zq_row[x0 + i];
-          }
-          if (kind == kPassRes)
-            for (int i = qfirst + tid; i < clen; i += kThreads) st.q[i] = q_row[x0 + i];
-          __syncthreads();
-        }
+        const int64_t x0 = static_cast<int64_t>(L % nch_a) * sp.tok_a;
+        const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
+        const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_a);
+        wait_stage(sq, st, zp_row, zq_row, nullptr, x0, clen, pass_of(L) != kPassMax, false, timed_out);
         body(st, x0, clen);
         __syncthreads();
-        if (tid == 0 && L + sp.nst < limit) issue(L + sp.nst, pol);
+        if (tid == 0 && L + sp.nst < nknown) issue(L + sp.nst, pol);
       }
     };
 
@@ -485,10 +608,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       Mp = block_max(lm, redf);
     }
 
-    // ---- pass B: the CD score s' on P_beta.  Each lane keeps an online max, a sum of
-    // 2^((s' - max) k2) rescaled whenever its max grows, and its argmax.  Rows that end in a
-    // race over pi_CD itself (sampled leaves) also record, per 256-token block (one warp, 8
-    // tokens a lane), the block's max and its sum relative to that max.
+    // ---- pass B: the CD score s' on P_beta; per lane an online max, rescaled sum and argmax;
+    // per 256-token block (one warp, 8 tokens a lane) the max and sum for a leaf's race
     const bool leaf_race = sampled && m == 0;
     float lmax = -INFINITY, lsum = 0.f;
     int larg = INT_MAX;
@@ -540,6 +661,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         }
       }
     });
+    seq = seq0 + static_cast<uint32_t>(L);
     if (tid < m) {
       czp[tid] = pzp;
       czq[tid] = pzq;
@@ -552,14 +674,13 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       czq[k] = ok ? ld1(zq_row, t) : 0.f;
       cq[k] = (ok && sampled) ? q_row[t] : 0.f;
     }
-    // row statistics from the lanes' (max, sum, argmax) (the reductions below also publish
-    // czp/czq/cq)
+    // row statistics from the lanes' (max, sum, argmax) (the reductions also publish czp/czq/cq)
     const float M = block_max(lmax, redf);
     const float S = block_sum(lmax > -INFINITY ? lsum * ex2((lmax - M) * k2) : 0.f, redf);
     float lbest = lmax;
     block_argmax(lbest, larg, redf, redi);
     const int arg = larg;
-    uint32_t status = rs->status;
+    uint32_t status = rs->status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
     if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
     const float logS = logf(S);
     const float invS = 1.f / S;
@@ -580,6 +701,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
     }
 
     int acc = -1, term = -1;
+    bool handed_over = false;
     if (!sampled) {
       // ---- greedy rule: the first child whose token is the argmax
       for (int k = 0; k < m; ++k)
@@ -588,152 +710,99 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
           break;
         }
       if (acc < 0) term = arg;
+    } else if (m > 0) {
+      // ---- sampled rule, first sibling: accept child 0 iff u <= pi_CD,T(t) / q(t); a rejection
+      // queues the first residual pass (the row's record is written when its chain ends)
+      if (tid == 0) {
+        const bool in = !masked || (czp[0] - Mp >= logb);
+        const float rt = in ? ex2(fmaf(fmaf(c1, czp[0], -alpha * czq[0]), k2, -Mk2)) * invS : 0.f;
+        const float qt = cq[0];
+        const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
+        const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[0]);
+        const float u = u01(philox_block(p.seed, p.offset, G, 0u).x);
+        int accept = u <= ratio ? 1 : 0;
+        if (!accept && !(status & (DCD_DEVERR_BAD_PARENT | DCD_DEVERR_BAD_TOKEN | DCD_DEVERR_BAD_PARAM |
+                                   DCD_DEVERR_NONFINITE))) {
+          const int s = static_cast<int>(atomicAdd(&sp.hdr->nslots, 1u));
+          SlotHead* sh = slot_head(sp, s);
+          sh->g = static_cast<int32_t>(g);
+          sh->m = m;
+          sh->M = M;
+          sh->S = S;
+          sh->Mp = Mp;
+          sh->c = 0.f;  // r_0 = pi: c_0 = 0, D_0 = 1
+          sh->D = 1.f;
+          sh->degen = 0;
+          sh->status = status;
+          create_job(sp, s, 1);
+          accept = -1;
+        }
+        rs->accept = accept;
+      }
+      __syncthreads();
+      if (rs->accept == 1) acc = kids[0];
+      if (rs->accept == -1) handed_over = true;
     } else {
-      // ---- sampled rule: test the children in order; each rejection streams one residual pass.
-      // r_j(x) = max(0, r_{j-1}(x) - q(x)) / Z_j with r_0 = pi_CD,T; invZ[j] = 0 marks Z_j = 0,
-      // where r_{j-1} equals q exactly and r_j is taken as q.
-      auto residual_at = [&](float s, bool in, float qv, int levels) -> float {
-        float r = in ? ex2(fmaf(s, k2, -Mk2)) * invS : 0.f;
-        for (int i = 1; i <= levels; ++i) {
-          const float iz = invZ[i];
-          r = iz > 0.f ? fmaxf(r - qv, 0.f) * iz : qv;
-        }
-        return r;
-      };
-      for (int j = 0; j < m; ++j) {
-        if (tid == 0) {
-          const bool in = !masked || (czp[j] - Mp >= logb);
-          const float rt = residual_at(fmaf(c1, czp[j], -alpha * czq[j]), in, cq[j], j);
-          const float qt = cq[j];
-          const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
-          const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[j]);
-          const float u = u01(philox_block(p.seed, p.offset, G, 0u).x);
-          rs->accept = u <= ratio;
-        }
-        __syncthreads();
-        if (rs->accept) {
-          acc = kids[j];
-          break;
-        }
-        // rejected: one more pass gives Z_{j+1}; after the last child it also keeps the block
-        // masses of the final residual and of q for the terminal race
-        const bool last = j + 1 == m;
-        const int first = limit;
-        limit += nch_r;
-        if (tid == 0)
-          for (int Li = first; Li < limit && Li < first + sp.nst; ++Li) issue(Li, pol);
-        float zl = 0.f;
-        run_items(nch_r, [&](const Stage<TIn>& st, int64_t x0, int clen) {
-          for (int kb = warp; kb * kRaceBlock < sp.tok_r; kb += kWarps) {
-            if (kb * kRaceBlock >= clen) break;  // warp-uniform
-            const int i0 = kb * kRaceBlock + lane * 8;
-            float zp[8], zq[8], qv[8];
-            ld8(st.zp + i0, zp);
-            ld8(st.zq + i0, zq);
-            ld8(st.q + i0, qv);
-            float part = 0.f, partq = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const bool valid = i0 + e < clen;
-              const float qe = valid ? qv[e] : 0.f;
-              const bool in = valid && (!masked || (zp[e] - Mp >= logb));
-              const float r = residual_at(fmaf(c1, zp[e], -alpha * zq[e]), in, qe, j);
-              part += valid ? fmaxf(r - qe, 0.f) : 0.f;
-              partq += qe;
-            }
-            zl += part;
-            if (last) {
-              const float br = warp_sum(part);
-              const float bqq = warp_sum(partq);
-              if (lane == 0) {
-                const int kabs = static_cast<int>(x0 / kRaceBlock) + kb;
-                bres[kabs] = br;
-                bq[kabs] = bqq;
-              }
-            }
+      // ---- sampled leaf: the terminal token is drawn from pi_CD,T by the two-level race: a
+      // 256-token block by its mass ...
+      float bk = -INFINITY;
+      int bb = INT_MAX;
+      for (int k = tid; k < sp.nblk; k += kThreads) {
+        if (bmax[k] > -INFINITY && bsum[k] > 0.f) {
+          const float lm = lg2(bsum[k]) + (bmax[k] - M) * k2;
+          const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
+                                       0x80000000u | (static_cast<uint32_t>(k) >> 2));
+          const float key = race_key(lm, word_of(w, k & 3));
+          if (key > bk) {
+            bk = key;
+            bb = k;
           }
-        });
-        const float Z = block_sum(zl, redf);
-        if (tid == 0) invZ[j + 1] = Z > 0.f ? 1.f / Z : 0.f;
-        __syncthreads();
+        }
       }
-      if (acc < 0) {
-        // ---- terminal draw, two-level exponential race: a 256-token block by its mass ...
-        const bool leaf = m == 0;
-        const bool degen = !leaf && !(invZ[m] > 0.f);
-        float bk = -INFINITY;
-        int bb = INT_MAX;
-        for (int k = tid; k < sp.nblk; k += kThreads) {
-          float lm = -INFINITY;
-          if (leaf) {
-            if (bmax[k] > -INFINITY && bsum[k] > 0.f) lm = lg2(bsum[k]) + (bmax[k] - M) * k2;
-          } else {
-            const float Rk = degen ? bq[k] : bres[k];
-            if (Rk > 0.f) lm = lg2(Rk);
-          }
-          if (lm > -INFINITY) {
-            const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
-                                         0x80000000u | (static_cast<uint32_t>(k) >> 2));
-            const float key = race_key(lm, word_of(w, k & 3));
-            if (key > bk) {
-              bk = key;
-              bb = k;
-            }
-          }
-        }
-        block_argmax(bk, bb, redf, redi);
-        // ... then a token of that block (warp 0 re-reads the block's 256 tokens)
-        if (warp == 0) {
-          float tk = -INFINITY;
-          int tx = INT_MAX;
-          if (bb != INT_MAX) {
-            const int64_t xb = static_cast<int64_t>(bb) * kRaceBlock + lane * 8;
-            const uint4 wa = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
-                                          1u + static_cast<uint32_t>(xb >> 2));
-            const uint4 wb = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
-                                          2u + static_cast<uint32_t>(xb >> 2));
-            const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+      block_argmax(bk, bb, redf, redi);
+      // ... then a token of that block (warp 0 re-reads the block's 256 tokens)
+      if (warp == 0) {
+        float tk = -INFINITY;
+        int tx = INT_MAX;
+        if (bb != INT_MAX) {
+          const int64_t xb = static_cast<int64_t>(bb) * kRaceBlock + lane * 8;
+          const uint4 wa =
+              philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 1u + static_cast<uint32_t>(xb >> 2));
+          const uint4 wb =
+              philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 2u + static_cast<uint32_t>(xb >> 2));
+          const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const int64_t x = xb + e;
-              if (x < V) {
-                const float z = ld1(zp_row, x);
-                const bool in = !masked || (z - Mp >= logb);
-                const float s = fmaf(c1, z, -alpha * ld1(zq_row, x));
-                float v;
-                if (leaf) {
-                  v = in ? ex2(fmaf(s, k2, -Mk2)) : 0.f;
-                } else {
-                  const float qe = q_row[x];
-                  v = degen ? qe : fmaxf(residual_at(s, in, qe, m - 1) - qe, 0.f);
-                }
-                if (v > 0.f) {
-                  const float key = race_key(lg2(v), w[e]);
-                  if (key > tk) {
-                    tk = key;
-                    tx = static_cast<int>(x);
-                  }
+          for (int e = 0; e < 8; ++e) {
+            const int64_t x = xb + e;
+            if (x < V) {
+              const float z = ld1(zp_row, x);
+              const bool in = !masked || (z - Mp >= logb);
+              const float v = in ? ex2(fmaf(fmaf(c1, z, -alpha * ld1(zq_row, x)), k2, -Mk2)) : 0.f;
+              if (v > 0.f) {
+                const float key = race_key(lg2(v), w[e]);
+                if (key > tk) {
+                  tk = key;
+                  tx = static_cast<int>(x);
                 }
               }
             }
           }
-          warp_argmax(tk, tx);
-          if (lane == 0) rs->term = tx;
         }
-        __syncthreads();
-        term = rs->term;
+        warp_argmax(tk, tx);
+        if (lane == 0) rs->term = tx;
       }
+      __syncthreads();
+      term = rs->term;
     }
-    if (tid == 0) {
+    if (tid == 0 && !handed_over) {
       RowRecord r;
       r.acc_child = acc;
       r.term_token = acc < 0 ? term : -1;
-      r.status = status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
+      r.status = status;
       r.reserved = 0;
       p.rec[g] = r;
     }
-    seq = seq0 + static_cast<uint32_t>(L);
-    __syncthreads();  // row state in shared memory is rewritten by the next row
+    __syncthreads();  // row state in shared memory is rewritten by the next work
   }
 }
 
@@ -866,39 +935,39 @@ struct Layout {
   size_t total;
 };
 
-Layout layout_for(int N, int nblk, int nst, int stage_bytes) {
+Layout layout_for(int N, int nblk, int nst) {
   Layout l;
   l.meta_offset = 8 * kMaxStages + 64 * 4;
-  const size_t meta_end = static_cast<size_t>(l.meta_offset) + sizeof(RowShared) + static_cast<size_t>(N) * 4 * 6;
+  const size_t meta_end = static_cast<size_t>(l.meta_offset) + sizeof(RowShared) + static_cast<size_t>(N) * 4 * 5;
   l.blk_offset = static_cast<int>((meta_end + 15) & ~static_cast<size_t>(15));
-  const size_t blk_end = static_cast<size_t>(l.blk_offset) + static_cast<size_t>(nblk) * 4 * 4;
+  const size_t blk_end = static_cast<size_t>(l.blk_offset) + static_cast<size_t>(nblk) * 4 * 2;
   l.stage_offset = static_cast<int>((blk_end + 127) & ~static_cast<size_t>(127));
-  l.total = static_cast<size_t>(l.stage_offset) + static_cast<size_t>(nst) * stage_bytes;
+  l.total = static_cast<size_t>(l.stage_offset) + static_cast<size_t>(nst) * kStageBytes;
   return l;
 }
 
-// Tokens per stage: z_p and z_q fill a stage in the max / stats passes; z_p, z_q and q share
-// it in residual passes (whole race blocks of 256 tokens either way).
+// Tokens per stage: z_p and z_q fill a stage in row passes; z_p, z_q and q share it in residual
+// pieces (whole race blocks of 256 tokens either way).
 int tokens_a(int es) { return kStageBytes / (2 * es); }
 int tokens_r(int es) { return kStageBytes / (2 * es + 4) / kRaceBlock * kRaceBlock; }
 
 }  // namespace
 
+int residual_pieces(int64_t V, int dtype) {
+  const int es = dtype == DCD_BF16 ? 2 : 4;
+  return static_cast<int>((V + tokens_r(es) - 1) / tokens_r(es));
+}
+
+size_t slot_bytes(int64_t V, int dtype) {
+  return sizeof(SlotHead) + static_cast<size_t>(residual_pieces(V, dtype)) * sizeof(PiecePart);
+}
+
 RowGeometry row_geometry(const ScoreArgs& a) {
   RowGeometry geo{};
   const int es = a.dtype == DCD_BF16 ? 2 : 4;
   const int nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
-  int nst = a.force_stages;
-  if (nst <= 0) {
-    // the deepest ring (up to 3 stages) that still lets two CTAs share an SM
-    nst = 2;
-    for (int s = 3; s >= 2; --s)
-      if (2 * (layout_for(a.N, nblk, s, kStageBytes).total + 1024) <= kSmemPerSm) {
-        nst = s;
-        break;
-      }
-  }
-  const Layout l = layout_for(a.N, nblk, nst, kStageBytes);
+  const int nst = a.force_stages > 0 ? a.force_stages : 2;
+  const Layout l = layout_for(a.N, nblk, nst);
   const int per_sm = static_cast<int>(kSmemPerSm / (l.total + 1024));
   geo.stages = nst;
   geo.stage_tokens = tokens_a(es);
@@ -925,15 +994,19 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.nst = geo.stages;
   sp.tok_a = tokens_a(es);
   sp.tok_r = tokens_r(es);
+  sp.npieces = residual_pieces(a.V, a.dtype);
   sp.bulk = geo.bulk;
   sp.nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
-  const Layout l = layout_for(a.N, sp.nblk, sp.nst, kStageBytes);
+  const Layout l = layout_for(a.N, sp.nblk, sp.nst);
   sp.meta_offset = l.meta_offset;
   sp.blk_offset = l.blk_offset;
   sp.stage_offset = l.stage_offset;
-  sp.work = a.err + 1;  // header word 1
-  // the device error word and the work counter start every call at zero
-  e = cudaMemsetAsync(a.err, 0, 2 * sizeof(uint32_t), stream);
+  sp.slot_bytes = static_cast<int32_t>(slot_bytes(a.V, a.dtype));
+  sp.hdr = a.hdr;
+  sp.jobs = a.jobs;
+  sp.slots = a.slots;
+  // the header counters and the job list start every call at zero
+  e = cudaMemsetAsync(a.hdr, 0, kWorkspaceHeader + static_cast<size_t>(R) * sizeof(Job), stream);
   if (e != cudaSuccess) return e;
   int64_t grid = static_cast<int64_t>(sms) * geo.ctas_per_sm;
   if (grid > R) grid = R;

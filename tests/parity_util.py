@@ -32,8 +32,9 @@ AMB_MASK = 1e-5
 
 
 def records(ws: torch.Tensor, R: int):
-    """Per-row records the row kernel leaves after the 256-byte workspace header."""
-    raw = ws[256:256 + 16 * R].cpu().numpy().view(np.int32).reshape(R, 4)
+    """Per-row records the kernels leave in the workspace (after the 256-byte header and R jobs)."""
+    off = 256 + 16 * R
+    raw = ws[off:off + 16 * R].cpu().numpy().view(np.int32).reshape(R, 4)
     return dict(acc_child=raw[:, 0].copy(), term_token=raw[:, 1].copy(), status=raw[:, 2].view(np.uint32).copy())
 
 

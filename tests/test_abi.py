@@ -65,7 +65,7 @@ def test_status_strings_and_version(lib):
 
 def test_workspace_bytes(lib):
     n = dcd.workspace_bytes(32, 60, 128256)
-    assert n >= 256 + 32 * 60 * 16 and n % 256 == 0
+    assert n >= 256 + 32 * 60 * 32 and n % 256 == 0
     bad = dcd.make_shape(1, 0, 10, 0)
     assert lib.dcd_workspace_bytes(ctypes.byref(bad)) == 0
     bad = dcd.make_shape(1, 4, 10, 5)

@@ -473,3 +473,29 @@ def test_subset_of_a_batch_draws_the_batch_uniforms():
         assert full["bonus"][b] == sub["bonus"][i]
         assert np.array_equal(full["rows"][b]["acc_child"], sub["rows"][i]["acc_child"])
         assert np.array_equal(full["rows"][b]["term_token"], sub["rows"][i]["term_token"])
+
+
+def test_residual_chain_closed_form():
+    """The iterated residual r_j = normalise(max(0, r_{j-1} - q)) of Algorithm 1 equals
+    max(0, pi - c_j q) / D_j with c_0 = 0, D_0 = 1, c_{j+1} = c_j + D_j, D_j = sum max(0, pi - c_j q)
+    (proof by induction on j); the GPU library evaluates the chain in this form."""
+    rng = np.random.default_rng(0)
+    for trial in range(8):
+        V = 300
+        zp = rng.standard_normal(V) * 2
+        zq = 0.7 * zp + rng.standard_normal(V)
+        q = np.exp(zp + rng.standard_normal(V))
+        q = (q / q.sum()).astype(np.float32)
+        toks = rng.integers(0, V, size=6)
+        alpha, beta = 0.2, (0.0 if trial % 2 else 0.05)
+        ratios, rm = oracle.row_chain(zp, zq, alpha, beta, 1.0, q, toks)
+        pi = np.exp(oracle.row_logpi(zp, zq, alpha, beta, 1.0)["logpi"])
+        qd = q.astype(np.float64)
+        c, D = 0.0, 1.0
+        closed = []
+        for t in toks:
+            closed.append(max(0.0, pi[t] - c * qd[t]) / D / qd[t])
+            c, D = c + D, None
+            D = np.maximum(0.0, pi - c * qd).sum()
+        np.testing.assert_allclose(closed, ratios, rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(np.maximum(0.0, pi - c * qd) / D, rm, rtol=0, atol=1e-14)

@@ -51,7 +51,7 @@ def test_noalloc_rejects_shapes_beyond_its_capacity():
     import ctypes
     lib = dcd.load()
     P = ctypes.c_void_p(0x10000)
-    big = dcd.make_shape(700, 60, 1000, dcd.DCD_BF16)  # 42000 rows > 32752
+    big = dcd.make_shape(2000, 60, 128256, dcd.DCD_BF16)  # 120000 rows need far more than 4 MiB
     rc = lib.dcd_verify_sample_noalloc(ctypes.byref(big), P, P, P, P, P, P, None, P, 0, 0, P, P, P, None, None,
                                        None, None, None)
     assert rc == -3
