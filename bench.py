@@ -197,7 +197,8 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     # weak scaling: every rank verifies its own full batch
-    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch)
+    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch,
+                                    temperatures=(0.0,) if args.greedy else (0.0, 1.0))
     B, N, V = w.B, w.N, w.V
     R = B * N
     out = dcd.alloc_outputs(B, N, dev)
@@ -207,8 +208,12 @@ def run_ours(args):
     def step(i, evs=None):
         if evs is not None:
             evs[0].record(stream)
-        dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q, temperature=w.temperature,
-                           seed=w.seed, offset=i, out=out, workspace=ws, stream=stream)
+        if w.q is None:
+            dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, out=out, workspace=ws,
+                               stream=stream)
+        else:
+            dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q,
+                               temperature=w.temperature, seed=w.seed, offset=i, out=out, workspace=ws, stream=stream)
         if evs is not None:
             evs[1].record(stream)
         dcd.dcd_tree_walk(B, N, V, out, ws, stream=stream)
@@ -337,6 +342,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
     ap.add_argument("--no-soak", action="store_true", help="skip the 1 s clock soak (profiling runs)")
+    ap.add_argument("--greedy", action="store_true", help="every sequence greedy (profiling case)")
     ap.add_argument("--batch", type=int, default=32,
                     help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
     args = ap.parse_args()

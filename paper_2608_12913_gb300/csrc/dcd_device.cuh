@@ -167,6 +167,35 @@ __device__ __forceinline__ void ld8(const __nv_bfloat16* p, float v[8]) {
   v[6] = __uint_as_float(a.w << 16); v[7] = __uint_as_float(a.w & 0xffff0000u);
 }
 
+// The same 8 tokens as four fp32 pairs (operands of the packed fp32x2 instructions).
+__device__ __forceinline__ void ld8x2(const float* p, float2 v[4]) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0];
+  const float4 b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = make_float2(a.x, a.y);
+  v[1] = make_float2(a.z, a.w);
+  v[2] = make_float2(b.x, b.y);
+  v[3] = make_float2(b.z, b.w);
+}
+
+__device__ __forceinline__ void ld8x2(const __nv_bfloat16* p, float2 v[4]) {
+  const uint4 a = *reinterpret_cast<const uint4*>(p);
+  v[0] = make_float2(__uint_as_float(a.x << 16), __uint_as_float(a.x & 0xffff0000u));
+  v[1] = make_float2(__uint_as_float(a.y << 16), __uint_as_float(a.y & 0xffff0000u));
+  v[2] = make_float2(__uint_as_float(a.z << 16), __uint_as_float(a.z & 0xffff0000u));
+  v[3] = make_float2(__uint_as_float(a.w << 16), __uint_as_float(a.w & 0xffff0000u));
+}
+
+// max(a, b, c) in one instruction (NaN operands are ignored, as by fmaxf).
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+__device__ __forceinline__ float max8(const float u[8]) {
+  return fmaxf(max3(max3(u[0], u[1], u[2]), u[3], u[4]), max3(u[5], u[6], u[7]));
+}
+
 __device__ __forceinline__ float ld1(const float* p, int64_t i) { return p[i]; }
 __device__ __forceinline__ float ld1(const __nv_bfloat16* p, int64_t i) { return __bfloat162float(p[i]); }
 

@@ -19,7 +19,8 @@ struct WsHeader {
   uint32_t job_alloc;  // residual passes created
   uint32_t job_head;   // first pass that may still have unclaimed pieces
   uint32_t nslots;     // rows handed to residual passes
-  uint32_t reserved[59];
+  uint32_t rows_done;  // rows whose record is written
+  uint32_t reserved[58];
 };
 static_assert(sizeof(WsHeader) == kWorkspaceHeader, "WsHeader layout");
 

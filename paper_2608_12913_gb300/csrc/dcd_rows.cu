@@ -10,8 +10,9 @@
 //    stage as soon as the block has consumed it.  The "stats" pass computes the CD score
 //    s' = (1 + alpha) z_p - alpha z_q (Eq. 1; the two log-softmax shifts are constant per
 //    row and cancel in the normaliser) on the plausibility set P_beta of Sec. 2.1; every
-//    lane keeps an online max, a sum of 2^((s' - max) k2) (k2 = log2(e) / T) rescaled when
-//    its max grows, and its argmax, reduced over the block at the end of the row.  With
+//    lane keeps an online max of the scaled score u = k2 s' (k2 = log2(e) / T), a sum of
+//    2^(u - max) rescaled when its max grows, and its argmax, reduced over the block at the
+//    end of the row.  With
 //    beta > 0 a "max" pass over z_p comes first.  Rows whose terminal draw races over
 //    pi_CD itself (sampled leaves) also keep per-256-token block maxima and sums, i.e. the
 //    block masses of pi_CD.  The greedy rule, the first sibling test of the sampled rule
@@ -22,13 +23,14 @@
 //    j-th residual is r_j = max(0, pi - c_j q) / D_j, where c_j = c_{j-1} + D_{j-1} and
 //    D_j = sum_x max(0, pi(x) - c_j q(x)) (induction on j from r_j = normalise(max(0,
 //    r_{j-1} - q))), so a pass needs only two scalars from the one before.  A row that
-//    needs a pass is handed to a job list; the pass is split into pieces of 4096 tokens
-//    that any CTA claims before taking a new row.  Each piece writes its partial sum (and,
+//    needs a pass is handed to a job list; the pass is split into pieces of four ring
+//    stages (16384 tokens for bf16 logits) that any CTA claims before taking a new row.  Each piece writes its partial sum (and,
 //    in the pass after the last sibling, its best race key) to its own slot; the CTA that
 //    finishes a pass's last piece (an atomic ticket, no waiting) sums the slots in a fixed
 //    order, tests the next sibling, and either queues the next pass or runs the terminal
-//    race.  Nothing waits on another CTA, so a CTA leaves when no piece is claimable and no
-//    row is left: work queued later belongs to a CTA that is still running.
+//    race.  A CTA with no row left polls for pieces until every row's record is written
+//    (bounded; all CTAs are co-resident under a cooperative launch), so the passes of late
+//    chains still spread over the whole GPU.
 //
 //  A node without an accepted child draws its terminal token by a two-level exponential
 //  race: a 256-token block by its mass, then a token of that block, whose 256 values are
@@ -70,7 +72,8 @@ struct SParams {
   ScoreArgs a;
   int32_t nst;           // ring depth (stages of kStageBytes)
   int32_t tok_a;         // tokens per stage in row passes (z_p, then z_q)
-  int32_t tok_r;         // tokens per residual piece (z_p, z_q, then q)
+  int32_t tok_r;         // tokens per stage in residual pieces (z_p, z_q, then q)
+  int32_t piece_stages;  // stages per residual piece
   int32_t npieces;       // pieces per residual pass
   int32_t bulk;          // 1: bulk asynchronous copies, 0: plain loads
   int32_t nblk;          // race blocks per row, ceil(V / 256)
@@ -146,17 +149,18 @@ __device__ __forceinline__ void create_job(const SParams& sp, int s, int J) {
 }
 
 // The sibling test of child `node` (token t): accept iff u <= r(t) / q(t) with
-// r = max(0, pi - c q) / D, or r = q once a pass found no residual mass (`degen`).  One thread.
+// r = max(0, pi - c q) / D, or r = q once a pass found no residual mass (`degen`); pi(t) =
+// 2^(u(t) - M) / S in the scaled score u = k2 s'.  One thread.
 template <typename TIn>
 __device__ bool sibling_test(const ScoreArgs& p, int b, int node, int t, const TIn* zp_row, const TIn* zq_row,
-                             const float* q_row, float c1, float alpha, bool masked, float Mp, float logb, float k2,
-                             float Mk2, float invS, float c, float D, bool degen) {
+                             const float* q_row, float c1k, float ak, bool masked, float Mp, float logb, float M,
+                             float invS, float c, float D, bool degen) {
   const bool ok = t >= 0 && t < p.V;
   const float z = ok ? ld1(zp_row, t) : 0.f;
   const float zz = ok ? ld1(zq_row, t) : 0.f;
   const float qt = ok ? q_row[t] : 0.f;
   const bool in = ok && (!masked || (z - Mp >= logb));
-  const float pit = in ? ex2(fmaf(fmaf(c1, z, -alpha * zz), k2, -Mk2)) * invS : 0.f;
+  const float pit = in ? ex2(fmaf(c1k, z, -ak * zz) - M) * invS : 0.f;
   const float rt = degen ? qt : fmaxf(pit - c * qt, 0.f) / D;
   const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
   const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * p.N + node);
@@ -240,28 +244,42 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   };
 
   for (;;) {
-    // ---- next work: a residual piece if one can be claimed, else the next row
+    // ---- next work: a residual piece if one can be claimed, else the next row.  With no row
+    // left, a CTA stays (all CTAs are co-resident: cooperative launch) until every row's record
+    // is written, to take pieces of passes other CTAs queue; the wait is bounded.
     if (tid == 0) {
       int kind = kWorkNone, job = -1, piece = 0;
-      const uint32_t alloc = ld_volatile(&sp.hdr->job_alloc);
-      for (uint32_t k = ld_volatile(&sp.hdr->job_head); k < alloc; ++k) {
-        if (ld_volatile(&sp.jobs[k].J) == 0) break;  // not yet published
-        const uint32_t pc = atomicAdd(&sp.jobs[k].next_piece, 1u);
-        if (pc < static_cast<uint32_t>(sp.npieces)) {
-          job = static_cast<int>(k);
-          piece = static_cast<int>(pc);
+      const long long t0 = clock64();
+      for (;;) {
+        const uint32_t alloc = ld_volatile(&sp.hdr->job_alloc);
+        for (uint32_t k = ld_volatile(&sp.hdr->job_head); k < alloc; ++k) {
+          if (ld_volatile(&sp.jobs[k].J) == 0) break;  // not yet published
+          const uint32_t pc = atomicAdd(&sp.jobs[k].next_piece, 1u);
+          if (pc < static_cast<uint32_t>(sp.npieces)) {
+            job = static_cast<int>(k);
+            piece = static_cast<int>(pc);
+            break;
+          }
+          atomicMax(&sp.hdr->job_head, k + 1u);
+        }
+        if (job >= 0) {
+          kind = kWorkPiece;
+          rs->item = job;
+          rs->piece = piece;
           break;
         }
-        atomicMax(&sp.hdr->job_head, k + 1u);
-      }
-      if (job >= 0) {
-        kind = kWorkPiece;
-        rs->item = job;
-        rs->piece = piece;
-      } else if (rs->next < R) {
-        kind = kWorkRow;
-        rs->item = rs->next;
-        rs->next = static_cast<int32_t>(atomicAdd(&sp.hdr->work, 1u));
+        if (rs->next < R) {
+          kind = kWorkRow;
+          rs->item = rs->next;
+          rs->next = static_cast<int32_t>(atomicAdd(&sp.hdr->work, 1u));
+          break;
+        }
+        if (ld_volatile(&sp.hdr->rows_done) >= static_cast<uint32_t>(R)) break;
+        if (clock64() - t0 > kWaitCycles) {
+          atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+          break;
+        }
+        __nanosleep(256);
       }
       rs->kind = kind;
     }
@@ -295,65 +313,78 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       const float T = p.temp[b];
       const bool masked = beta > 0.f;
       const float k2 = kLog2e / T;
-      const float c1 = 1.f + alpha;
+      const float c1k = (1.f + alpha) * k2, ak = alpha * k2;  // u = k2 s' = c1k z_p - ak z_q
       const float logb = masked ? logf(beta) : -INFINITY;
       const float M = rs->M, invS = 1.f / rs->S, Mp = rs->Mp, cJ = rs->c;
-      const float Mk2 = M * k2;
       const bool race = J == m;  // the pass after the last sibling also ranks race blocks
       const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
       const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
       const float* q_row = p.q + g * p.ldq;
-      const int64_t x0 = static_cast<int64_t>(piece) * sp.tok_r;
-      const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
-      const uint32_t sq = seq;
-      const int s_idx = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-      const Stage<TIn> st = stage_at<TIn>(ring, s_idx, sp.tok_r);
-      if (tid == 0) {
-        uint64_t* bar = &full[s_idx];
+      // the piece's stages, streamed through the ring like a row
+      const int64_t piece_lo = static_cast<int64_t>(piece) * sp.piece_stages * sp.tok_r;
+      const int64_t rem = (V - piece_lo + sp.tok_r - 1) / sp.tok_r;
+      const int nst_piece = static_cast<int>(rem < sp.piece_stages ? rem : sp.piece_stages);
+      const uint32_t seq0 = seq;
+      auto issue_piece = [&](int L) {  // thread 0 only
+        const uint32_t sq = seq0 + static_cast<uint32_t>(L);
+        const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
+        const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_r);
+        const int64_t x0 = piece_lo + static_cast<int64_t>(L) * sp.tok_r;
+        const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
         const uint32_t zb = sp.bulk ? static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u : 0u;
         const uint32_t qb = sp.bulk ? static_cast<uint32_t>(clen * 4) & ~15u : 0u;
-        mbar_arrive_expect_tx(bar, 2u * zb + qb);
+        mbar_arrive_expect_tx(&full[s], 2u * zb + qb);
         if (zb) {
-          bulk_g2s(st.zp, zp_row + x0, zb, bar, pol_last);
-          bulk_g2s(st.zq, zq_row + x0, zb, bar, pol_last);
+          bulk_g2s(st.zp, zp_row + x0, zb, &full[s], pol_last);
+          bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pol_last);
         }
-        if (qb) bulk_g2s(st.q, q_row + x0, qb, bar, pol_last);
-      }
+        if (qb) bulk_g2s(st.q, q_row + x0, qb, &full[s], pol_last);
+      };
+      if (tid == 0)
+        for (int L = 0; L < nst_piece && L < sp.nst; ++L) issue_piece(L);
       bool timed_out = false;
-      wait_stage(sq, st, zp_row, zq_row, q_row, x0, clen, true, true, timed_out);
       float zl = 0.f, bk = -INFINITY;
       int bb = INT_MAX;
-      for (int kb = warp; kb * kRaceBlock < sp.tok_r; kb += kWarps) {
-        if (kb * kRaceBlock >= clen) break;  // warp-uniform
-        const int i0 = kb * kRaceBlock + lane * 8;
-        float zp[8], zq[8], qv[8];
-        ld8(st.zp + i0, zp);
-        ld8(st.zq + i0, zq);
-        ld8(st.q + i0, qv);
-        float part = 0.f;
+      for (int L = 0; L < nst_piece; ++L) {
+        const uint32_t sq = seq0 + static_cast<uint32_t>(L);
+        const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(sq % static_cast<uint32_t>(sp.nst)), sp.tok_r);
+        const int64_t x0 = piece_lo + static_cast<int64_t>(L) * sp.tok_r;
+        const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
+        wait_stage(sq, st, zp_row, zq_row, q_row, x0, clen, true, true, timed_out);
+        for (int kb = warp; kb * kRaceBlock < sp.tok_r; kb += kWarps) {
+          if (kb * kRaceBlock >= clen) break;  // warp-uniform
+          const int i0 = kb * kRaceBlock + lane * 8;
+          float zp[8], zq[8], qv[8];
+          ld8(st.zp + i0, zp);
+          ld8(st.zq + i0, zq);
+          ld8(st.q + i0, qv);
+          float part = 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const bool valid = i0 + e < clen;
-          const bool in = valid && (!masked || (zp[e] - Mp >= logb));
-          const float pit = in ? ex2(fmaf(fmaf(c1, zp[e], -alpha * zq[e]), k2, -Mk2)) * invS : 0.f;
-          part += valid ? fmaxf(pit - cJ * qv[e], 0.f) : 0.f;
-        }
-        zl += part;
-        if (race) {
-          const float R_b = warp_sum(part);
-          if (lane == 0 && R_b > 0.f) {
-            const uint32_t kabs = static_cast<uint32_t>(x0 / kRaceBlock) + static_cast<uint32_t>(kb);
-            const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (kabs >> 2));
-            const float key = race_key(lg2(R_b), word_of(w, static_cast<int>(kabs & 3)));
-            if (key > bk) {
-              bk = key;
-              bb = static_cast<int>(kabs);
+          for (int e = 0; e < 8; ++e) {
+            const bool valid = i0 + e < clen;
+            const bool in = valid && (!masked || (zp[e] - Mp >= logb));
+            const float pit = in ? ex2(fmaf(c1k, zp[e], -ak * zq[e]) - M) * invS : 0.f;
+            part += valid ? fmaxf(pit - cJ * qv[e], 0.f) : 0.f;
+          }
+          zl += part;
+          if (race) {
+            const float R_b = warp_sum(part);
+            if (lane == 0 && R_b > 0.f) {
+              const uint32_t kabs = static_cast<uint32_t>(x0 / kRaceBlock) + static_cast<uint32_t>(kb);
+              const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (kabs >> 2));
+              const float key = race_key(lg2(R_b), word_of(w, static_cast<int>(kabs & 3)));
+              if (key > bk) {
+                bk = key;
+                bb = static_cast<int>(kabs);
+              }
             }
           }
         }
+        __syncthreads();
+        if (tid == 0 && L + sp.nst < nst_piece) issue_piece(L + sp.nst);
       }
-      seq = sq + 1;
-      const float zsum = block_sum(zl, redf);  // also frees the stage (all reads are done)
+      seq = seq0 + static_cast<uint32_t>(nst_piece);
+      const float zsum = block_sum(zl, redf);
       block_argmax(bk, bb, redf, redi);
       if (tid == 0) {
         PiecePart pp;
@@ -396,8 +427,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         int acc = -1;
         bool queued = false;
         for (int j = J; j < m; ++j) {
-          if (sibling_test<TIn>(p, b, kids[j], ktok[j], zp_row, zq_row, q_row, c1, alpha, masked, Mp, logb, k2, Mk2,
-                                invS, c, D, degen)) {
+          if (sibling_test<TIn>(p, b, kids[j], ktok[j], zp_row, zq_row, q_row, c1k, ak, masked, Mp, logb, M, invS, c,
+                                D, degen)) {
             acc = kids[j];
             break;
           }
@@ -472,7 +503,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
                 } else {
                   const float z = ld1(zp_row, x);
                   const bool in = !masked || (z - Mp >= logb);
-                  const float pit = in ? ex2(fmaf(fmaf(c1, z, -alpha * ld1(zq_row, x)), k2, -Mk2)) * invS : 0.f;
+                  const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
                   v = fmaxf(pit - c * qe, 0.f) / D;
                 }
                 if (v > 0.f) {
@@ -498,6 +529,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         r.status = rs->status;
         r.reserved = 0;
         p.rec[g] = r;
+        __threadfence();
+        atomicAdd(&sp.hdr->rows_done, 1u);
       }
       __syncthreads();
       continue;
@@ -514,7 +547,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
     const bool masked = beta > 0.f;
     const float invT = T > 0.f ? 1.f / T : 1.f;
     const float k2 = kLog2e * invT;  // exp(x / T) = 2^(x * k2)
-    const float c1 = 1.f + alpha;
+    // scores are kept in the scaled unit u = k2 s' = c1k z_p - ak z_q, so pi_CD,T ~ 2^u
+    const float c1k = (1.f + alpha) * k2, ak = alpha * k2;
     const float logb = masked ? logf(beta) : -INFINITY;
     const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
     const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
@@ -608,49 +642,63 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       Mp = block_max(lm, redf);
     }
 
-    // ---- pass B: the CD score s' on P_beta; per lane an online max, rescaled sum and argmax;
-    // per 256-token block (one warp, 8 tokens a lane) the max and sum for a leaf's race
+    // ---- pass B: the scaled CD score u on P_beta; per lane an online max, rescaled sum of 2^(u -
+    // max) and argmax; per 256-token block (one warp, 8 tokens a lane) the max and sum for a
+    // leaf's race.  Full blocks of unmasked rows take a path without per-token predicates,
+    // on packed fp32x2 arithmetic.
     const bool leaf_race = sampled && m == 0;
+    const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
     float lmax = -INFINITY, lsum = 0.f;
     int larg = INT_MAX;
     run_items(nch_a, [&](const Stage<TIn>& st, int64_t x0, int clen) {
       for (int kb = warp; kb * kRaceBlock < sp.tok_a; kb += kWarps) {
         if (kb * kRaceBlock >= clen) break;  // warp-uniform
         const int i0 = kb * kRaceBlock + lane * 8;
-        float zp[8], zq[8], sv[8];
-        ld8(st.zp + i0, zp);
-        ld8(st.zq + i0, zq);
-        float gm = -INFINITY;
+        float u[8];
+        if (!masked && (kb + 1) * kRaceBlock <= clen) {  // warp-uniform
+          float2 zp2[4], zq2[4];
+          ld8x2(st.zp + i0, zp2);
+          ld8x2(st.zq + i0, zq2);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const bool in = (i0 + e < clen) && (!masked || (zp[e] - Mp >= logb));
-          sv[e] = in ? fmaf(c1, zp[e], -alpha * zq[e]) : -INFINITY;
-          gm = fmaxf(gm, sv[e]);
+          for (int k = 0; k < 4; ++k) {
+            const float2 s2 = __ffma2_rn(zp2[k], c1k2, __fmul2_rn(zq2[k], nak2));
+            u[2 * k] = s2.x;
+            u[2 * k + 1] = s2.y;
+          }
+        } else {
+          float zp[8], zq[8];
+          ld8(st.zp + i0, zp);
+          ld8(st.zq + i0, zq);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const bool in = (i0 + e < clen) && (!masked || (zp[e] - Mp >= logb));
+            u[e] = in ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
+          }
         }
+        const float gm = max8(u);
         if (gm > lmax) {
-          lsum *= ex2((lmax - gm) * k2);  // 0 while lmax is -inf
+          lsum *= ex2(lmax - gm);  // 0 while lmax is -inf
           lmax = gm;
 #pragma unroll
           for (int e = 7; e >= 0; --e)
-            if (sv[e] == gm) larg = static_cast<int>(x0) + i0 + e;
+            if (u[e] == gm) larg = static_cast<int>(x0) + i0 + e;
         }
         if (lmax > -INFINITY) {
-          const float mk = lmax * k2;
-          float s0 = 0.f, s1 = 0.f;
+          const float2 nm2 = make_float2(-lmax, -lmax);
+          float2 acc2 = make_float2(0.f, 0.f);
 #pragma unroll
-          for (int e = 0; e < 8; e += 2) {
-            s0 += ex2(fmaf(sv[e], k2, -mk));
-            s1 += ex2(fmaf(sv[e + 1], k2, -mk));
+          for (int k = 0; k < 4; ++k) {
+            const float2 d = __fadd2_rn(make_float2(u[2 * k], u[2 * k + 1]), nm2);
+            acc2 = __fadd2_rn(acc2, make_float2(ex2(d.x), ex2(d.y)));
           }
-          lsum += s0 + s1;
+          lsum += acc2.x + acc2.y;
         }
         if (leaf_race) {
           const float bm = warp_max(gm);
           float part = 0.f;
           if (bm > -INFINITY) {
-            const float mk = bm * k2;
 #pragma unroll
-            for (int e = 0; e < 8; ++e) part += ex2(fmaf(sv[e], k2, -mk));
+            for (int e = 0; e < 8; ++e) part += ex2(u[e] - bm);
           }
           const float bs = warp_sum(part);
           if (lane == 0) {
@@ -674,9 +722,10 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       czq[k] = ok ? ld1(zq_row, t) : 0.f;
       cq[k] = (ok && sampled) ? q_row[t] : 0.f;
     }
-    // row statistics from the lanes' (max, sum, argmax) (the reductions also publish czp/czq/cq)
+    // row statistics from the lanes' (max, sum, argmax) (the reductions also publish czp/czq/cq):
+    // M = max u, S = sum 2^(u - M), so log sum exp(s' / T) = M ln 2 + ln S
     const float M = block_max(lmax, redf);
-    const float S = block_sum(lmax > -INFINITY ? lsum * ex2((lmax - M) * k2) : 0.f, redf);
+    const float S = block_sum(lmax > -INFINITY ? lsum * ex2(lmax - M) : 0.f, redf);
     float lbest = lmax;
     block_argmax(lbest, larg, redf, redi);
     const int arg = larg;
@@ -684,19 +733,19 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
     if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
     const float logS = logf(S);
     const float invS = 1.f / S;
-    const float Mk2 = M * k2;
+    constexpr float kLn2 = 0.69314718055994531f;
 
     // ---- outputs of the Eq. 1 target
     if (tid == 0) {
       if (p.cd_argmax) p.cd_argmax[g] = arg;
-      if (p.cd_lse) p.cd_lse[g] = M * invT + logS;
+      if (p.cd_lse) p.cd_lse[g] = M * kLn2 + logS;
       if (n == 0 && p.cd_logprob) p.cd_logprob[g] = 0.f;
     }
     if (p.cd_logprob) {
       for (int k = tid; k < m; k += kThreads) {
         const bool in = !masked || (czp[k] - Mp >= logb);
         p.cd_logprob[static_cast<int64_t>(b) * N + kids[k]] =
-            in ? (fmaf(c1, czp[k], -alpha * czq[k]) - M) * invT - logS : -INFINITY;
+            in ? (fmaf(c1k, czp[k], -ak * czq[k]) - M) * kLn2 - logS : -INFINITY;
       }
     }
 
@@ -715,7 +764,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       // queues the first residual pass (the row's record is written when its chain ends)
       if (tid == 0) {
         const bool in = !masked || (czp[0] - Mp >= logb);
-        const float rt = in ? ex2(fmaf(fmaf(c1, czp[0], -alpha * czq[0]), k2, -Mk2)) * invS : 0.f;
+        const float rt = in ? ex2(fmaf(c1k, czp[0], -ak * czq[0]) - M) * invS : 0.f;
         const float qt = cq[0];
         const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
         const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[0]);
@@ -749,7 +798,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       int bb = INT_MAX;
       for (int k = tid; k < sp.nblk; k += kThreads) {
         if (bmax[k] > -INFINITY && bsum[k] > 0.f) {
-          const float lm = lg2(bsum[k]) + (bmax[k] - M) * k2;
+          const float lm = lg2(bsum[k]) + (bmax[k] - M);
           const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
                                        0x80000000u | (static_cast<uint32_t>(k) >> 2));
           const float key = race_key(lm, word_of(w, k & 3));
@@ -777,7 +826,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
             if (x < V) {
               const float z = ld1(zp_row, x);
               const bool in = !masked || (z - Mp >= logb);
-              const float v = in ? ex2(fmaf(fmaf(c1, z, -alpha * ld1(zq_row, x)), k2, -Mk2)) : 0.f;
+              const float v = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) : 0.f;
               if (v > 0.f) {
                 const float key = race_key(lg2(v), w[e]);
                 if (key > tk) {
@@ -801,6 +850,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       r.status = status;
       r.reserved = 0;
       p.rec[g] = r;
+      __threadfence();
+      atomicAdd(&sp.hdr->rows_done, 1u);
     }
     __syncthreads();  // row state in shared memory is rewritten by the next work
   }
@@ -953,9 +1004,13 @@ int tokens_r(int es) { return kStageBytes / (2 * es + 4) / kRaceBlock * kRaceBlo
 
 }  // namespace
 
+// A residual piece covers up to kPieceStages ring stages (16384 tokens for bf16 logits).
+constexpr int kPieceStages = 4;
+
 int residual_pieces(int64_t V, int dtype) {
   const int es = dtype == DCD_BF16 ? 2 : 4;
-  return static_cast<int>((V + tokens_r(es) - 1) / tokens_r(es));
+  const int64_t tok = static_cast<int64_t>(tokens_r(es)) * kPieceStages;
+  return static_cast<int>((V + tok - 1) / tok);
 }
 
 size_t slot_bytes(int64_t V, int dtype) {
@@ -994,6 +1049,7 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.nst = geo.stages;
   sp.tok_a = tokens_a(es);
   sp.tok_r = tokens_r(es);
+  sp.piece_stages = kPieceStages;
   sp.npieces = residual_pieces(a.V, a.dtype);
   sp.bulk = geo.bulk;
   sp.nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
@@ -1008,14 +1064,29 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   // the header counters and the job list start every call at zero
   e = cudaMemsetAsync(a.hdr, 0, kWorkspaceHeader + static_cast<size_t>(R) * sizeof(Job), stream);
   if (e != cudaSuccess) return e;
-  int64_t grid = static_cast<int64_t>(sms) * geo.ctas_per_sm;
+  // a CTA may wait for work queued by another, so all CTAs must be resident at once: the grid is
+  // the resident capacity (capped at the row count) and the launch is cooperative
+  int per_sm = 0;
+  e = a.dtype == DCD_BF16
+          ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<__nv_bfloat16>, kThreads, geo.smem)
+          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<float>, kThreads, geo.smem);
+  if (e != cudaSuccess) return e;
+  if (per_sm > geo.ctas_per_sm) per_sm = geo.ctas_per_sm;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  int64_t grid = static_cast<int64_t>(sms) * per_sm;
   if (grid > R) grid = R;
-  if (grid < 1) grid = 1;
-  if (a.dtype == DCD_BF16)
-    score_rows_kernel<__nv_bfloat16><<<static_cast<unsigned>(grid), kThreads, geo.smem, stream>>>(sp);
-  else
-    score_rows_kernel<float><<<static_cast<unsigned>(grid), kThreads, geo.smem, stream>>>(sp);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = geo.smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (a.dtype == DCD_BF16) return cudaLaunchKernelEx(&cfg, score_rows_kernel<__nv_bfloat16>, sp);
+  return cudaLaunchKernelEx(&cfg, score_rows_kernel<float>, sp);
 }
 
 cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_t* err, int32_t* accept_len,
