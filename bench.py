@@ -47,7 +47,7 @@ def _peaks():
 
 def _kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for name in ("dcd_rows.cu", "dcd_internal.h"):
+    for name in ("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h"):
         with open(os.path.join(ROOT, "paper_2608_12913_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -119,14 +119,31 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(win), "window": "from 1 s before the timed region to its end"}
 
 
-def algorithmic_bytes(w) -> int:
-    """Bytes the path must move per step: both logit rows of every node (bf16), q for the
-    non-leaf rows of sampled sequences (fp32), the tree, parameters and outputs."""
+def algorithmic_bytes(w, residual_rows: float) -> float:
+    """Bytes the step must move: both logit rows of every node (bf16), the draft distribution q
+    of every row whose sampled rule needs a residual (a rejected sibling; the other rows need q
+    only at their children's tokens), the tree, parameters and outputs."""
     es = 2 if w.dtype == "bf16" else 4
     logits = 2 * w.R * w.V * es
-    qb = w.sampled_rows_with_children() * w.V * 4
+    qb = residual_rows * w.V * 4
     small = w.R * (4 + 4) + w.B * 12 + w.R * 12 + w.B * (8 + w.N * 4)
     return logits + qb + small
+
+
+def residual_rows_per_step(w, out, ws, stream, offsets) -> float:
+    """Mean number of rows handed to residual passes over the given Philox offsets (the
+    workspace header's word 4 counts them; the outcome depends only on inputs and offset)."""
+    import torch
+    from paper_2608_12913_gb300 import dcd
+    if w.q is None:
+        return 0.0
+    counts = []
+    for off in offsets:
+        dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q,
+                           temperature=w.temperature, seed=w.seed, offset=off, out=out, workspace=ws, stream=stream)
+        counts.append(ws[16:20].view(torch.int32).clone())
+    torch.cuda.synchronize()
+    return float(torch.stack(counts).double().mean().item())
 
 
 def _dist_env():
@@ -260,8 +277,11 @@ def run_ours(args):
     ms_per_step = elapsed_ms / args.steps
     value = world * R / (ms_per_step / 1e3)
 
-    # roofline of the dominant kernel (the row kernel) from its own events
-    alg = algorithmic_bytes(w)
+    # roofline of the dominant kernel (the row kernel) from its own events; the rows that took
+    # residual passes are counted on a replay of every 32nd timed offset
+    replay = [1_000_000 + k for k in range(0, args.steps, 32)]
+    res_rows = residual_rows_per_step(w, out, ws, stream, replay)
+    alg = algorithmic_bytes(w, res_rows)
     row_avg_s = statistics.mean(row_ms) / 1e3
     achieved = alg / row_avg_s / 1e9
     peak, peak_kind = _peaks()
@@ -269,7 +289,8 @@ def run_ours(args):
     traffic = _profiled_traffic(khash)
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": traffic, "kernel": "score_rows_kernel", "peak_source": f"{peak_kind} hbm_gbs",
-                "algorithmic_bytes_per_launch": alg, "row_kernel_ms": row_avg_s * 1e3,
+                "algorithmic_bytes_per_launch": alg, "residual_rows_per_step": res_rows,
+                "row_kernel_ms": row_avg_s * 1e3,
                 "kernel_source_sha256_16": khash}
 
     # end to end through the public API: pinned host inputs -> device, verify, results -> host
@@ -317,7 +338,7 @@ def run_ours(args):
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": WORKLOAD if B == 32 else f"{WORKLOAD} (profiling case, B={B})", "B": B, "N": N, "V": V, "rows": R, "logits": "bf16",
                        "sampled_sequences": int((w.temperature > 0).sum().item()),
-                       "bytes_per_step": alg, "l2": "inputs (1.48 GB per step) larger than L2; no flush",
+                       "bytes_per_step": alg, "l2": "inputs (1.97 GB resident) larger than L2; no flush",
                        "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
             "roofline": roofline,
             "clocks": sampler.summary(t_wall0, t_wall1),

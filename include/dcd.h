@@ -29,11 +29,16 @@
  *   duplicate sibling tokens -> lowest node id).  Sampled (T > 0): with r_0 = pi_CD,T
  *   child j is accepted iff u_j <= r_{j-1}(t_j) / q(t_j); after a rejection
  *   r_j = normalise(max(0, r_{j-1} - q)) (Algorithm 1, generalised to sibling lists);
- *   a node with no accepted child draws its terminal token from its last residual
- *   (pi_CD,T at a leaf) by an exponential race argmax_x log r(x) - log(-log u_x).
+ *   a node with no accepted child draws its terminal token from its last residual r
+ *   (pi_CD,T at a leaf) by a two-level exponential race: the block k of 1024
+ *   consecutive tokens maximising log R_k - log(-log v_k), R_k = sum of r over the
+ *   block, then the token x of that block maximising log r(x) - log(-log u_x).  The
+ *   two levels together draw x with probability r(x) (Algorithm 1 leaves the sampling
+ *   method open).
  * - Randomness: Philox4x32-10 (Salmon et al., SC'11), key = (seed_lo, seed_hi).
  *   The acceptance uniform of node c uses counter (b*N + c, 0, offset_lo, offset_hi)
- *   word 0; the race uniform of token x in row g uses counter (g, 1 + x/4, offset_lo,
+ *   word 0; in row g the block uniform v_k uses counter (g, 2^31 + k/4, offset_lo,
+ *   offset_hi) word k%4 and the token uniform u_x counter (g, 1 + x/4, offset_lo,
  *   offset_hi) word x%4; a word w maps to u = ((w >> 9) + 0.5) * 2^-23 in (0, 1).
  *   One call consumes one offset value: advance `offset` by one per call.
  * - accept_len[b] counts accepted drafted tokens (the bonus token is excluded, as in
@@ -46,9 +51,11 @@
  *   s'(x) / T_eff - cd_lse[g]); T_eff = T, or 1 for greedy sequences.
  * - Memory: every array pointer is a DEVICE pointer owned by the caller.  The
  *   library allocates nothing per call; scratch lives in the caller's workspace
- *   (dcd_workspace_bytes: 256 bytes plus, per row, 96 bytes and 16 bytes per 4096
- *   vocabulary tokens (bf16 logits); its contents need no initialisation).  Calls are asynchronous and ordered on `stream`; host-side
- *   argument checks return a negative status before anything is launched.  Two
+ *   (dcd_workspace_bytes: 256 bytes plus, per row, 96 bytes and 16 bytes per
+ *   16384 vocabulary tokens (bf16 logits; 8192 for fp32), rounded up to 256; its
+ *   contents need no initialisation).  Calls are asynchronous and ordered on
+ *   `stream`; host-side argument checks return a negative status before anything is
+ *   launched.  Two
  *   calls that share a workspace must not overlap on the device.
  * - Thread safety: entry points may be called from several host threads, each with
  *   its own workspace.

@@ -33,7 +33,7 @@
  * as 1, 2, 3", SC'11), key = (seed_lo, seed_hi).  The acceptance uniform of
  * node c (global id G = b*N + c) uses counter (G, 0, off_lo, off_hi), word 0;
  * the race uniform of token x in row G uses counter (G, 1 + x/4, off_lo,
- * off_hi), word x%4; the race uniform of token block k (ids 256k .. 256k+255)
+ * off_hi), word x%4; the race uniform of token block k (ids 1024k .. 1024k+1023)
  * uses counter (G, 2^31 + k/4, off_lo, off_hi), word k%4.  A 32-bit word w
  * becomes u = ((w >> 9) + 0.5) * 2^-23, a value in (0, 1) that fp32 also holds
  * exactly.  Terminal tokens are drawn by a two-level exponential race: a block
@@ -109,7 +109,7 @@ double dcd_oracle_race_uniform(uint64_t seed, uint64_t offset, uint32_t G, int64
   return dcd_oracle_u01(philox_word(seed, offset, G, (uint32_t)(1 + (x >> 2)), (int)(x & 3)));
 }
 
-/* Exponential-race uniform of token block k (tokens 256k .. 256k+255) in global row G. */
+/* Exponential-race uniform of token block k (tokens 1024k .. 1024k+1023) in global row G. */
 double dcd_oracle_block_uniform(uint64_t seed, uint64_t offset, uint32_t G, int64_t k) {
   return dcd_oracle_u01(philox_word(seed, offset, G, 0x80000000u | (uint32_t)(k >> 2), (int)(k & 3)));
 }
@@ -245,7 +245,7 @@ static double accept_ratio(double rt, double qt) {
   return rt > 0.0 ? INFINITY : 0.0;
 }
 
-#define RACE_BLOCK 256
+#define RACE_BLOCK 1024
 
 /*
  * Draw from r (unnormalised, r >= 0) by a two-level exponential race: first a block of

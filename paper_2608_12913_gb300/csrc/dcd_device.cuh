@@ -15,7 +15,8 @@ namespace dev {
 
 constexpr int kThreads = 256;  // threads per CTA of every row kernel
 constexpr int kWarps = kThreads / 32;
-constexpr int kRaceBlock = 256;                   // tokens per block of the two-level terminal race
+constexpr int kRaceBlock = 1024;                  // tokens per block of the two-level terminal race
+constexpr int kSub = 256;                         // tokens a warp handles at once (8 a lane)
 constexpr long long kWaitCycles = 4000000000ll;  // bounded waits: about two seconds at the boost clock
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -249,6 +250,34 @@ __device__ __forceinline__ float block_sum(float v, float* redf) {
   for (int w = 0; w < kWarps; ++w) s += redf[w];
   __syncthreads();
   return s;
+}
+
+// Combines per-thread (max m, sum s of 2^(x - m), argmax) over the block in log2 units: every
+// thread gets the block max, the sum rescaled to it, and the argmax (ties to the lowest index).
+__device__ __forceinline__ void block_stats(float& m, float& s, int& arg, float* redf, int* redi) {
+  auto merge = [](float& m1, float& s1, int& a1, float m2, float s2, int a2) {
+    const float M = fmaxf(m1, m2);
+    const float t1 = m1 > -INFINITY ? s1 * ex2(m1 - M) : 0.f;
+    const float t2 = m2 > -INFINITY ? s2 * ex2(m2 - M) : 0.f;
+    if (m2 > m1 || (m2 == m1 && a2 < a1)) a1 = a2;
+    m1 = M;
+    s1 = t1 + t2;
+  };
+#pragma unroll
+  for (int o = 16; o; o >>= 1)
+    merge(m, s, arg, __shfl_xor_sync(~0u, m, o), __shfl_xor_sync(~0u, s, o), __shfl_xor_sync(~0u, arg, o));
+  if ((threadIdx.x & 31) == 0) {
+    redf[threadIdx.x >> 5] = m;
+    redf[kWarps + (threadIdx.x >> 5)] = s;
+    redi[threadIdx.x >> 5] = arg;
+  }
+  __syncthreads();
+  m = redf[0];
+  s = redf[kWarps];
+  arg = redi[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) merge(m, s, arg, redf[w], redf[kWarps + w], redi[w]);
+  __syncthreads();
 }
 
 __device__ __forceinline__ float block_max(float v, float* redf) {

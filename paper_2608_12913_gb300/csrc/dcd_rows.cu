@@ -1,6 +1,7 @@
 // dcd_rows.cu -- the streaming kernels of the CD verification step on sm_103a.
 //
-// score_rows_kernel: a persistent grid (a few CTAs per SM) with two kinds of work.
+// score_rows_kernel: a persistent, cooperatively launched grid (a few CTAs per SM) with two
+// kinds of work.
 //
 //  * Rows.  A CTA claims whole tree-node rows g = b * N + n from a work counter, in
 //    node-major order (every sequence's node 0, then every node 1, ...), so internal
@@ -9,14 +10,14 @@
 //    asynchronous copies that complete on one mbarrier per stage; thread 0 refills a
 //    stage as soon as the block has consumed it.  The "stats" pass computes the CD score
 //    s' = (1 + alpha) z_p - alpha z_q (Eq. 1; the two log-softmax shifts are constant per
-//    row and cancel in the normaliser) on the plausibility set P_beta of Sec. 2.1; every
-//    lane keeps an online max of the scaled score u = k2 s' (k2 = log2(e) / T), a sum of
-//    2^(u - max) rescaled when its max grows, and its argmax, reduced over the block at the
-//    end of the row.  With
-//    beta > 0 a "max" pass over z_p comes first.  Rows whose terminal draw races over
-//    pi_CD itself (sampled leaves) also keep per-256-token block maxima and sums, i.e. the
-//    block masses of pi_CD.  The greedy rule, the first sibling test of the sampled rule
-//    and the leaf race then finish the row.
+//    row and cancel in the normaliser) on the plausibility set P_beta of Sec. 2.1, in the
+//    scaled unit u = k2 s' (k2 = log2(e) / T, so pi_CD,T ~ 2^u).  A warp takes a
+//    contiguous eighth of each stage; every lane keeps an online max of u, a sum of
+//    2^(u - max) rescaled when its max grows, and its argmax, combined over the block at the
+//    end of the row.  With beta > 0 a "max" pass over z_p comes first.  Sampled rows also
+//    get, from the same exponentials, each 1024-token block's mass of pi_CD for a terminal
+//    race.  The greedy rule, the first sibling test of the sampled rule and the leaf race
+//    then finish the row.
 //
 //  * Residual pieces.  After a rejected sibling, Algorithm 1 (generalised to sibling
 //    lists) needs the next residual over the whole vocabulary.  With c_0 = 0, D_0 = 1 the
@@ -24,17 +25,17 @@
 //    D_j = sum_x max(0, pi(x) - c_j q(x)) (induction on j from r_j = normalise(max(0,
 //    r_{j-1} - q))), so a pass needs only two scalars from the one before.  A row that
 //    needs a pass is handed to a job list; the pass is split into pieces of four ring
-//    stages (16384 tokens for bf16 logits) that any CTA claims before taking a new row.  Each piece writes its partial sum (and,
-//    in the pass after the last sibling, its best race key) to its own slot; the CTA that
-//    finishes a pass's last piece (an atomic ticket, no waiting) sums the slots in a fixed
-//    order, tests the next sibling, and either queues the next pass or runs the terminal
-//    race.  A CTA with no row left polls for pieces until every row's record is written
-//    (bounded; all CTAs are co-resident under a cooperative launch), so the passes of late
-//    chains still spread over the whole GPU.
+//    stages (16384 tokens for bf16 logits) that any CTA claims before taking a new row.
+//    Each piece writes its partial sum (and, in the pass after the last sibling, its best
+//    race key) to its own slot; the CTA that finishes a pass's last piece (an atomic
+//    ticket, no waiting) sums the slots in a fixed order, tests the next sibling, and
+//    either queues the next pass or runs the terminal race.  A CTA with no row left polls
+//    for pieces until every row's record is written (bounded; all CTAs are co-resident
+//    under a cooperative launch), so the passes of late chains still spread over the GPU.
 //
 //  A node without an accepted child draws its terminal token by a two-level exponential
-//  race: a 256-token block by its mass, then a token of that block, whose 256 values are
-//  re-read directly.
+//  race: a 1024-token block by its mass, then a token of that block (four tokens a thread,
+//  re-read directly).
 // tree_walk_kernel: one thread per sequence follows the accepted children.
 // terminal_residual_kernel: one block per sequence rebuilds the distribution its bonus
 //   token was drawn from (test output only).
@@ -61,8 +62,10 @@ using namespace dev;
 #endif
 constexpr int kStageBytes = DCD_STAGE_KIB * 1024;  // bytes per ring stage
 constexpr int kMaxStages = 8;
+constexpr int kPieceStages = 4;                    // ring stages per residual piece
 constexpr size_t kSmemMax = 227 * 1024;
 constexpr size_t kSmemPerSm = 228 * 1024;
+constexpr float kLn2 = 0.69314718055994531f;
 
 enum PassKind { kPassMax = 0, kPassStats = 1 };
 enum WorkKind { kWorkNone = 0, kWorkRow = 1, kWorkPiece = 2 };
@@ -73,10 +76,9 @@ struct SParams {
   int32_t nst;           // ring depth (stages of kStageBytes)
   int32_t tok_a;         // tokens per stage in row passes (z_p, then z_q)
   int32_t tok_r;         // tokens per stage in residual pieces (z_p, z_q, then q)
-  int32_t piece_stages;  // stages per residual piece
   int32_t npieces;       // pieces per residual pass
   int32_t bulk;          // 1: bulk asynchronous copies, 0: plain loads
-  int32_t nblk;          // race blocks per row, ceil(V / 256)
+  int32_t nblk;          // race blocks per row, ceil(V / 1024)
   int32_t meta_offset;   // byte offsets into dynamic shared memory
   int32_t blk_offset;
   int32_t stage_offset;
@@ -95,7 +97,7 @@ struct RowShared {
   int32_t m;         // children of the row's node
   uint32_t status;   // DCD_DEVERR_* bits
   int32_t accept;    // outcome of a sibling test
-  int32_t term;      // terminal token, or winning race block
+  int32_t term;      // winning race block of a completed pass
   int32_t last;      // this CTA finished a pass's last piece
   int32_t degen;     // a pass found no residual mass left
   int32_t slot;      // slot of the handed-over row
@@ -103,6 +105,8 @@ struct RowShared {
   int32_t g;         // row of the piece
   float M, S, Mp, c, D;
   int32_t pad[2];
+  float wref[2][kWarps];  // per-warp shares of race-block masses, double-buffered by stage
+  float wsum[2][kWarps];
 };
 
 template <typename TIn>
@@ -148,9 +152,60 @@ __device__ __forceinline__ void create_job(const SParams& sp, int s, int J) {
   *reinterpret_cast<volatile int32_t*>(&job->J) = J;
 }
 
+// Lists the children of node n (ascending id) into kids / ktok with the calling warp; returns
+// their count in every lane.
+__device__ __forceinline__ int list_children(const ScoreArgs& p, int b, int n, int* kids, int* ktok) {
+  const int lane = threadIdx.x & 31;
+  const int32_t* parr = p.parents + static_cast<int64_t>(b) * p.N;
+  const int32_t* tokr = p.tokens + static_cast<int64_t>(b) * p.N;
+  int count = 0;
+  for (int base = n + 1; base < p.N; base += 32) {
+    const int c = base + lane;
+    const bool is = c < p.N && parr[c] == n;
+    const unsigned msk = __ballot_sync(~0u, is);
+    if (is) {
+      const int pos = count + __popc(msk & ((1u << lane) - 1u));
+      kids[pos] = c;
+      ktok[pos] = tokr[c];
+    }
+    count += __popc(msk);
+  }
+  __syncwarp();
+  return count;
+}
+
+// The scaled CD score u = c1k z_p - ak z_q of 8 tokens of a stage; tokens past `clen` or
+// outside P_beta get -inf.  A whole 256-token group of an unmasked row skips the per-token
+// predicates and uses packed fp32x2 arithmetic (the same roundings as the scalar path).
+template <typename TIn>
+__device__ __forceinline__ void scores8(const TIn* zp_s, const TIn* zq_s, int i0, int sb, int clen, bool masked,
+                                        float c1k, float ak, float Mp, float logb, float u[8]) {
+  if (!masked && sb + kSub <= clen) {
+    const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
+    float2 zp2[4], zq2[4];
+    ld8x2(zp_s + i0, zp2);
+    ld8x2(zq_s + i0, zq2);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 s2 = __ffma2_rn(zp2[k], c1k2, __fmul2_rn(zq2[k], nak2));
+      u[2 * k] = s2.x;
+      u[2 * k + 1] = s2.y;
+    }
+  } else {
+    float zp[8], zq[8];
+    ld8(zp_s + i0, zp);
+    ld8(zq_s + i0, zq);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const bool in = (i0 + e < clen) && (!masked || (zp[e] - Mp >= logb));
+      u[e] = in ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
+    }
+  }
+}
+
 // The sibling test of child `node` (token t): accept iff u <= r(t) / q(t) with
 // r = max(0, pi - c q) / D, or r = q once a pass found no residual mass (`degen`); pi(t) =
-// 2^(u(t) - M) / S in the scaled score u = k2 s'.  One thread.
+// 2^(u(t) - M) / S.  One thread.
 template <typename TIn>
 __device__ bool sibling_test(const ScoreArgs& p, int b, int node, int t, const TIn* zp_row, const TIn* zq_row,
                              const float* q_row, float c1k, float ak, bool masked, float Mp, float logb, float M,
@@ -168,9 +223,48 @@ __device__ bool sibling_test(const ScoreArgs& p, int b, int node, int t, const T
   return u <= ratio;
 }
 
+// Second level of the terminal race: the token x of race block `kstar` with the largest
+// log2 r(x) - log2(-log2 u_x), four tokens a thread (one Philox call, counter 1 + x / 4).
+// `mass(x)` returns r(x) up to a common factor.  Every thread of the block calls it and gets
+// the token (INT_MAX when no block had mass).
+template <typename MassFn>
+__device__ int token_race(const ScoreArgs& p, int64_t g, int kstar, MassFn mass, float* redf, int* redi) {
+  float tk = -INFINITY;
+  int tx = INT_MAX;
+  if (kstar != INT_MAX) {
+    const int64_t x = static_cast<int64_t>(kstar) * kRaceBlock + threadIdx.x * 4;
+    if (x < p.V) {
+      const uint4 w =
+          philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 1u + static_cast<uint32_t>(x >> 2));
+      const uint32_t words[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (x + e < p.V) {
+          const float v = mass(x + e);
+          if (v > 0.f) {
+            const float key = race_key(lg2(v), words[e]);
+            if (key > tk) {
+              tk = key;
+              tx = static_cast<int>(x + e);
+            }
+          }
+        }
+      }
+    }
+  }
+  block_argmax(tk, tx, redf, redi);
+  return tx;
+}
+
+// First level of the race for one block: its key from log2 of its mass.
+__device__ __forceinline__ float block_key(const ScoreArgs& p, int64_t g, int k, float log2_mass) {
+  const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (static_cast<uint32_t>(k) >> 2));
+  return race_key(log2_mass, word_of(w, k & 3));
+}
+
 // ------------------------------------------------------------------------------------------
 template <typename TIn>
-__global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_constant__ SParams sp) {
+__global__ void __launch_bounds__(kThreads, 3) score_rows_kernel(const __grid_constant__ SParams sp) {
   const ScoreArgs& p = sp.a;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int N = p.N;
@@ -188,8 +282,8 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   float* czp = reinterpret_cast<float*>(ktok + N);                // [N] z_p at those tokens
   float* czq = czp + N;                                           // [N] z_q at those tokens
   float* cq = czq + N;                                            // [N] q at those tokens
-  float* bmax = reinterpret_cast<float*>(smem + sp.blk_offset);   // [nblk] block max of s'
-  float* bsum = bmax + sp.nblk;                                   // [nblk] block sums
+  float* bmax = reinterpret_cast<float*>(smem + sp.blk_offset);   // [nblk] block reference of u
+  float* bsum = bmax + sp.nblk;                                   // [nblk] block sum of 2^(u - ref)
   unsigned char* ring = smem + sp.stage_offset;
 
   if (tid == 0) {
@@ -201,27 +295,6 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
   const uint64_t pol_last = l2_policy_evict_last();
   const uint64_t pol_first = l2_policy_evict_first();
   uint32_t seq = 0;  // ring items consumed by this CTA so far (identical in every thread)
-
-  // Lists the children of node n of sequence b (warp `w`), ascending id, and their count.
-  auto scan_children = [&](int b, int n, int w) {
-    if (warp == w) {
-      const int32_t* par = p.parents + static_cast<int64_t>(b) * N;
-      const int32_t* tok = p.tokens + static_cast<int64_t>(b) * N;
-      int count = 0;
-      for (int base = n + 1; base < N; base += 32) {
-        const int c = base + lane;
-        const bool is = c < N && par[c] == n;
-        const unsigned msk = __ballot_sync(~0u, is);
-        if (is) {
-          const int pos = count + __popc(msk & ((1u << lane) - 1u));
-          kids[pos] = c;
-          ktok[pos] = tok[c];
-        }
-        count += __popc(msk);
-      }
-      if (lane == 0) rs->m = count;
-    }
-  };
 
   // Waits for ring item `sq`, then fills a ragged or unaligned remainder with plain loads.
   auto wait_stage = [&](uint32_t sq, const Stage<TIn>& st, const TIn* zp_row, const TIn* zq_row,
@@ -320,10 +393,12 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
       const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
       const float* q_row = p.q + g * p.ldq;
-      // the piece's stages, streamed through the ring like a row
-      const int64_t piece_lo = static_cast<int64_t>(piece) * sp.piece_stages * sp.tok_r;
+      // the piece's stages, streamed through the ring like a row; a warp takes tok_r / 8
+      // consecutive tokens of each stage, so `wpb` warps cover one race block
+      const int tpw = sp.tok_r / kWarps, wpb = kRaceBlock / tpw;
+      const int64_t piece_lo = static_cast<int64_t>(piece) * kPieceStages * sp.tok_r;
       const int64_t rem = (V - piece_lo + sp.tok_r - 1) / sp.tok_r;
-      const int nst_piece = static_cast<int>(rem < sp.piece_stages ? rem : sp.piece_stages);
+      const int nst_piece = static_cast<int>(rem < kPieceStages ? rem : kPieceStages);
       const uint32_t seq0 = seq;
       auto issue_piece = [&](int L) {  // thread 0 only
         const uint32_t sq = seq0 + static_cast<uint32_t>(L);
@@ -350,38 +425,39 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(sq % static_cast<uint32_t>(sp.nst)), sp.tok_r);
         const int64_t x0 = piece_lo + static_cast<int64_t>(L) * sp.tok_r;
         const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
+        const int par = L & 1;
         wait_stage(sq, st, zp_row, zq_row, q_row, x0, clen, true, true, timed_out);
-        for (int kb = warp; kb * kRaceBlock < sp.tok_r; kb += kWarps) {
-          if (kb * kRaceBlock >= clen) break;  // warp-uniform
-          const int i0 = kb * kRaceBlock + lane * 8;
-          float zp[8], zq[8], qv[8];
-          ld8(st.zp + i0, zp);
-          ld8(st.zq + i0, zq);
+        float part = 0.f;
+        for (int sb = warp * tpw; sb < (warp + 1) * tpw && sb < clen; sb += kSub) {  // warp-uniform
+          const int i0 = sb + lane * 8;
+          float u[8], qv[8];
+          scores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
           ld8(st.q + i0, qv);
-          float part = 0.f;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const bool valid = i0 + e < clen;
-            const bool in = valid && (!masked || (zp[e] - Mp >= logb));
-            const float pit = in ? ex2(fmaf(c1k, zp[e], -ak * zq[e]) - M) * invS : 0.f;
-            part += valid ? fmaxf(pit - cJ * qv[e], 0.f) : 0.f;
-          }
-          zl += part;
-          if (race) {
-            const float R_b = warp_sum(part);
-            if (lane == 0 && R_b > 0.f) {
-              const uint32_t kabs = static_cast<uint32_t>(x0 / kRaceBlock) + static_cast<uint32_t>(kb);
-              const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (kabs >> 2));
-              const float key = race_key(lg2(R_b), word_of(w, static_cast<int>(kabs & 3)));
-              if (key > bk) {
-                bk = key;
-                bb = static_cast<int>(kabs);
-              }
-            }
-          }
+          for (int e = 0; e < 8; ++e)
+            part += (i0 + e < clen) ? fmaxf(ex2(u[e] - M) * invS - cJ * qv[e], 0.f) : 0.f;
+        }
+        zl += part;
+        if (race) {
+          const float ws = warp_sum(part);
+          if (lane == 0) rs->wsum[par][warp] = ws;
         }
         __syncthreads();
         if (tid == 0 && L + sp.nst < nst_piece) issue_piece(L + sp.nst);
+        // block masses of the last pass's residual (read while the next stage streams in; the
+        // shares are double-buffered, so the next stage's writes go to the other half)
+        if (race && tid < sp.tok_r / kRaceBlock && x0 + static_cast<int64_t>(tid) * kRaceBlock < V) {
+          float mass = 0.f;
+          for (int w = 0; w < wpb; ++w) mass += rs->wsum[par][tid * wpb + w];
+          if (mass > 0.f) {
+            const int kabs = static_cast<int>(x0 / kRaceBlock) + tid;
+            const float key = block_key(p, g, kabs, lg2(mass));
+            if (key > bk) {
+              bk = key;
+              bb = kabs;
+            }
+          }
+        }
       }
       seq = seq0 + static_cast<uint32_t>(nst_piece);
       const float zsum = block_sum(zl, redf);
@@ -402,7 +478,7 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
 
       // ================= the pass is complete: next sibling test, next pass or terminal race
       const int n = static_cast<int>(g % N);
-      scan_children(b, n, 0);
+      if (warp == 0) list_children(p, b, n, kids, ktok);
       if (tid == 0) {
         __threadfence();  // every piece's part was written before its ticket
         SlotHead* sh = slot_head(sp, rs->slot);
@@ -459,19 +535,17 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         const float c = rs->c, D = rs->D;
         int kstar = rs->term;
         if (degen) {
-          // block masses of q, streamed by this CTA alone (rare: a residual without mass)
+          // block masses of q, computed by this CTA alone (rare: a residual without mass)
           float bk2 = -INFINITY;
           int bb2 = INT_MAX;
           for (int kb = warp; kb < sp.nblk; kb += kWarps) {
-            const int64_t xb = static_cast<int64_t>(kb) * kRaceBlock + lane * 8;
             float part = 0.f;
-            for (int e = 0; e < 8; ++e)
-              if (xb + e < V) part += q_row[xb + e];
-            const float R_b = warp_sum(part);
-            if (lane == 0 && R_b > 0.f) {
-              const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
-                                           0x80000000u | (static_cast<uint32_t>(kb) >> 2));
-              const float key = race_key(lg2(R_b), word_of(w, kb & 3));
+            for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < V && x < (kb + 1) * kRaceBlock;
+                 x += 32)
+              part += q_row[x];
+            const float mass = warp_sum(part);
+            if (lane == 0 && mass > 0.f) {
+              const float key = block_key(p, g, kb, lg2(mass));
               if (key > bk2) {
                 bk2 = key;
                 bb2 = kb;
@@ -481,46 +555,17 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
           block_argmax(bk2, bb2, redf, redi);
           kstar = bb2;
         }
-        __syncthreads();
-        if (warp == 0) {
-          float tk = -INFINITY;
-          int tx = INT_MAX;
-          if (kstar != INT_MAX) {
-            const int64_t xb = static_cast<int64_t>(kstar) * kRaceBlock + lane * 8;
-            const uint4 wa =
-                philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 1u + static_cast<uint32_t>(xb >> 2));
-            const uint4 wb =
-                philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 2u + static_cast<uint32_t>(xb >> 2));
-            const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const int64_t x = xb + e;
-              if (x < V) {
-                const float qe = q_row[x];
-                float v;
-                if (degen) {
-                  v = qe;
-                } else {
-                  const float z = ld1(zp_row, x);
-                  const bool in = !masked || (z - Mp >= logb);
-                  const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
-                  v = fmaxf(pit - c * qe, 0.f) / D;
-                }
-                if (v > 0.f) {
-                  const float key = race_key(lg2(v), w[e]);
-                  if (key > tk) {
-                    tk = key;
-                    tx = static_cast<int>(x);
-                  }
-                }
-              }
-            }
-          }
-          warp_argmax(tk, tx);
-          if (lane == 0) rs->term = tx;
-        }
-        __syncthreads();
-        term = rs->term;
+        term = token_race(
+            p, g, kstar,
+            [&](int64_t x) -> float {
+              const float qe = q_row[x];
+              if (degen) return qe;
+              const float z = ld1(zp_row, x);
+              const bool in = !masked || (z - Mp >= logb);
+              const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
+              return fmaxf(pit - c * qe, 0.f) / D;
+            },
+            redf, redi);
       }
       if (tid == 0) {
         RowRecord r;
@@ -574,45 +619,48 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       }
     };
 
-    // thread 0 starts the row's stream at once (a beta > 0 row keeps its max pass in L2 for the
-    // stats pass; a sampled row with children keeps its logits in L2 for residual pieces); warp
-    // 1 meanwhile lists the children of node n and checks this row
-    uint64_t pol = (masked || sampled) ? pol_last : pol_first;
+    // Thread 0 starts the row's stream at once.  A beta > 0 row keeps its max pass in L2 for
+    // the stats pass, and a sampled row its logits for residual pieces until it is known to be
+    // a leaf.  Warp 1 meanwhile lists the children of node n, checks the row and loads the
+    // values at the children's tokens, which are consumed after the stats pass; the first
+    // stage barrier publishes the child count.
     if (tid == 0) {
+      const uint64_t pol0 = (masked || sampled) ? pol_last : pol_first;
       const int first = nknown < sp.nst ? nknown : sp.nst;
-      for (int L = 0; L < first; ++L) issue(L, pol);
+      for (int L = 0; L < first; ++L) issue(L, pol0);
     }
-    scan_children(b, n, 1);
-    if (warp == 1 && lane == 0) {
-      uint32_t st = 0u;
-      const int pp = p.parents[static_cast<int64_t>(b) * N + n];
-      if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
-      if (n > 0) {
-        const int t = p.tokens[static_cast<int64_t>(b) * N + n];
-        if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
-      }
-      if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
-        st |= DCD_DEVERR_BAD_PARAM;
-      rs->status = st;
-    }
-    __syncthreads();
-    const int m = rs->m;
-    if (sampled && m == 0 && !masked) pol = pol_first;
-    // values at the children's tokens: the loads are issued now and consumed after the stats pass
     float pzp = 0.f, pzq = 0.f, pq = 0.f;
-    if (tid < m) {
-      const int t = ktok[tid];
-      if (t >= 0 && t < V) {
-        pzp = ld1(zp_row, t);
-        pzq = ld1(zq_row, t);
-        if (sampled) pq = q_row[t];
+    if (warp == 1) {
+      const int count = list_children(p, b, n, kids, ktok);
+      if (lane < count) {
+        const int t = ktok[lane];
+        if (t >= 0 && t < V) {
+          pzp = ld1(zp_row, t);
+          pzq = ld1(zq_row, t);
+          if (sampled) pq = q_row[t];
+        }
+      }
+      if (lane == 0) {
+        uint32_t st = 0u;
+        const int pp = p.parents[static_cast<int64_t>(b) * N + n];
+        if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
+        if (n > 0) {
+          const int t = p.tokens[static_cast<int64_t>(b) * N + n];
+          if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
+        }
+        if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
+          st |= DCD_DEVERR_BAD_PARAM;
+        rs->m = count;
+        rs->status = st;
       }
     }
 
     int L = 0;  // next item to consume
     bool timed_out = false;
-    // Consumes `count` items: waits for each stage, hands it to `body`, releases and refills it.
-    auto run_items = [&](int count, auto&& body) {
+    // Consumes `count` items: waits for each stage, hands it to `body`, refills the stage once
+    // the block has finished it, then runs `after` (which may read what `body` left in shared
+    // memory, double-buffered by item parity).
+    auto run_items = [&](int count, auto&& body, auto&& after) {
       for (int it = 0; it < count; ++it, ++L) {
         const uint32_t sq = seq0 + static_cast<uint32_t>(L);
         const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
@@ -620,120 +668,120 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
         const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_a);
         wait_stage(sq, st, zp_row, zq_row, nullptr, x0, clen, pass_of(L) != kPassMax, false, timed_out);
-        body(st, x0, clen);
+        body(st, x0, clen, L & 1);
         __syncthreads();
-        if (tid == 0 && L + sp.nst < nknown) issue(L + sp.nst, pol);
+        if (tid == 0 && L + sp.nst < nknown) {
+          const bool keep = (masked && L + sp.nst < nch_a) || (sampled && rs->m > 0);
+          issue(L + sp.nst, keep ? pol_last : pol_first);
+        }
+        after(x0, clen, L & 1);
       }
     };
+    auto no_after = [](int64_t, int, int) {};
 
     // ---- pass A (beta > 0): the expert max, for P_beta = {x : z_p(x) - max z_p >= log beta}
     float Mp = 0.f;
     if (masked) {
       float lm = -INFINITY;
-      run_items(nch_a, [&](const Stage<TIn>& st, int64_t, int clen) {
-        for (int i0 = tid * 8; i0 < clen; i0 += kThreads * 8) {
-          float zp[8];
-          ld8(st.zp + i0, zp);
+      run_items(
+          nch_a,
+          [&](const Stage<TIn>& st, int64_t, int clen, int) {
+            for (int i0 = tid * 8; i0 < clen; i0 += kThreads * 8) {
+              float zp[8];
+              ld8(st.zp + i0, zp);
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (i0 + e < clen) lm = fmaxf(lm, zp[e]);
-        }
-      });
+              for (int e = 0; e < 8; ++e)
+                if (i0 + e < clen) lm = fmaxf(lm, zp[e]);
+            }
+          },
+          no_after);
       Mp = block_max(lm, redf);
     }
 
-    // ---- pass B: the scaled CD score u on P_beta; per lane an online max, rescaled sum of 2^(u -
-    // max) and argmax; per 256-token block (one warp, 8 tokens a lane) the max and sum for a
-    // leaf's race.  Full blocks of unmasked rows take a path without per-token predicates,
-    // on packed fp32x2 arithmetic.
-    const bool leaf_race = sampled && m == 0;
-    const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
+    // ---- pass B: per lane an online max of u on P_beta, the sum of 2^(u - max) rescaled when
+    // the max grows, and the argmax.  A warp takes tok_a / 8 consecutive tokens of each stage, so
+    // `wpb` warps cover one race block; for sampled rows each warp also reports its share of the
+    // stage's mass, which threads 0.. combine into the block masses after the stage barrier.
+    const int tpw = sp.tok_a / kWarps, wpb = kRaceBlock / tpw;
     float lmax = -INFINITY, lsum = 0.f;
     int larg = INT_MAX;
-    run_items(nch_a, [&](const Stage<TIn>& st, int64_t x0, int clen) {
-      for (int kb = warp; kb * kRaceBlock < sp.tok_a; kb += kWarps) {
-        if (kb * kRaceBlock >= clen) break;  // warp-uniform
-        const int i0 = kb * kRaceBlock + lane * 8;
-        float u[8];
-        if (!masked && (kb + 1) * kRaceBlock <= clen) {  // warp-uniform
-          float2 zp2[4], zq2[4];
-          ld8x2(st.zp + i0, zp2);
-          ld8x2(st.zq + i0, zq2);
+    run_items(
+        nch_a,
+        [&](const Stage<TIn>& st, int64_t x0, int clen, int par) {
+          float bpart = 0.f;  // this lane's share of the warp's mass in this stage, relative to lmax
+          for (int sb = warp * tpw; sb < (warp + 1) * tpw && sb < clen; sb += kSub) {  // warp-uniform
+            const int i0 = sb + lane * 8;
+            float u[8];
+            scores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
+            const float gm = max8(u);
+            if (gm > lmax) {
+              const float f = ex2(lmax - gm);  // 0 while lmax is -inf
+              lsum *= f;
+              bpart *= f;
+              lmax = gm;
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const float2 s2 = __ffma2_rn(zp2[k], c1k2, __fmul2_rn(zq2[k], nak2));
-            u[2 * k] = s2.x;
-            u[2 * k + 1] = s2.y;
-          }
-        } else {
-          float zp[8], zq[8];
-          ld8(st.zp + i0, zp);
-          ld8(st.zq + i0, zq);
+              for (int e = 7; e >= 0; --e)
+                if (u[e] == gm) larg = static_cast<int>(x0) + i0 + e;
+            }
+            if (lmax > -INFINITY) {
+              const float2 nm2 = make_float2(-lmax, -lmax);
+              float2 acc2 = make_float2(0.f, 0.f);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const bool in = (i0 + e < clen) && (!masked || (zp[e] - Mp >= logb));
-            u[e] = in ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
+              for (int k = 0; k < 4; ++k) {
+                const float2 d = __fadd2_rn(make_float2(u[2 * k], u[2 * k + 1]), nm2);
+                acc2 = __fadd2_rn(acc2, make_float2(ex2(d.x), ex2(d.y)));
+              }
+              const float a = acc2.x + acc2.y;
+              lsum += a;
+              bpart += a;
+            }
           }
-        }
-        const float gm = max8(u);
-        if (gm > lmax) {
-          lsum *= ex2(lmax - gm);  // 0 while lmax is -inf
-          lmax = gm;
-#pragma unroll
-          for (int e = 7; e >= 0; --e)
-            if (u[e] == gm) larg = static_cast<int>(x0) + i0 + e;
-        }
-        if (lmax > -INFINITY) {
-          const float2 nm2 = make_float2(-lmax, -lmax);
-          float2 acc2 = make_float2(0.f, 0.f);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const float2 d = __fadd2_rn(make_float2(u[2 * k], u[2 * k + 1]), nm2);
-            acc2 = __fadd2_rn(acc2, make_float2(ex2(d.x), ex2(d.y)));
+          if (sampled) {
+            const float ref = warp_max(lmax);
+            const float ws = warp_sum(lmax > -INFINITY ? bpart * ex2(lmax - ref) : 0.f);
+            if (lane == 0) {
+              rs->wref[par][warp] = ref;
+              rs->wsum[par][warp] = ws;
+            }
           }
-          lsum += acc2.x + acc2.y;
-        }
-        if (leaf_race) {
-          const float bm = warp_max(gm);
-          float part = 0.f;
-          if (bm > -INFINITY) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) part += ex2(u[e] - bm);
+        },
+        [&](int64_t x0, int clen, int par) {
+          if (sampled && tid < sp.tok_a / kRaceBlock && tid * kRaceBlock < clen) {
+            float ref = -INFINITY, sum = 0.f;
+            for (int w = 0; w < wpb; ++w) ref = fmaxf(ref, rs->wref[par][tid * wpb + w]);
+            if (ref > -INFINITY)
+              for (int w = 0; w < wpb; ++w) {
+                const float r = rs->wref[par][tid * wpb + w];
+                if (r > -INFINITY) sum += rs->wsum[par][tid * wpb + w] * ex2(r - ref);
+              }
+            const int kabs = static_cast<int>(x0 / kRaceBlock) + tid;
+            bmax[kabs] = ref;
+            bsum[kabs] = sum;
           }
-          const float bs = warp_sum(part);
-          if (lane == 0) {
-            const int kabs = static_cast<int>(x0 / kRaceBlock) + kb;
-            bmax[kabs] = bm;
-            bsum[kabs] = bs;
-          }
-        }
-      }
-    });
+        });
     seq = seq0 + static_cast<uint32_t>(L);
-    if (tid < m) {
-      czp[tid] = pzp;
-      czq[tid] = pzq;
-      cq[tid] = pq;
+    const int m = rs->m;
+    if (warp == 1 && lane < m) {
+      czp[lane] = pzp;
+      czq[lane] = pzq;
+      cq[lane] = pq;
     }
-    for (int k = kThreads + tid; k < m; k += kThreads) {  // rows with more children than threads
+    for (int k = 32 + tid; k < m; k += kThreads) {  // nodes with more children than a warp has lanes
       const int t = ktok[k];
       const bool ok = t >= 0 && t < V;
       czp[k] = ok ? ld1(zp_row, t) : 0.f;
       czq[k] = ok ? ld1(zq_row, t) : 0.f;
       cq[k] = (ok && sampled) ? q_row[t] : 0.f;
     }
-    // row statistics from the lanes' (max, sum, argmax) (the reductions also publish czp/czq/cq):
+    // row statistics (the reduction's barriers also publish czp / czq / cq and the block masses):
     // M = max u, S = sum 2^(u - M), so log sum exp(s' / T) = M ln 2 + ln S
-    const float M = block_max(lmax, redf);
-    const float S = block_sum(lmax > -INFINITY ? lsum * ex2(lmax - M) : 0.f, redf);
-    float lbest = lmax;
-    block_argmax(lbest, larg, redf, redi);
-    const int arg = larg;
+    float M = lmax, S = lsum;
+    int arg = larg;
+    block_stats(M, S, arg, redf, redi);
     uint32_t status = rs->status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
     if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
     const float logS = logf(S);
     const float invS = 1.f / S;
-    constexpr float kLn2 = 0.69314718055994531f;
 
     // ---- outputs of the Eq. 1 target
     if (tid == 0) {
@@ -793,15 +841,12 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
       if (rs->accept == -1) handed_over = true;
     } else {
       // ---- sampled leaf: the terminal token is drawn from pi_CD,T by the two-level race: a
-      // 256-token block by its mass ...
+      // 1024-token block by its mass 2^(bmax - M) bsum ...
       float bk = -INFINITY;
       int bb = INT_MAX;
       for (int k = tid; k < sp.nblk; k += kThreads) {
         if (bmax[k] > -INFINITY && bsum[k] > 0.f) {
-          const float lm = lg2(bsum[k]) + (bmax[k] - M);
-          const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g),
-                                       0x80000000u | (static_cast<uint32_t>(k) >> 2));
-          const float key = race_key(lm, word_of(w, k & 3));
+          const float key = block_key(p, g, k, lg2(bsum[k]) + (bmax[k] - M));
           if (key > bk) {
             bk = key;
             bb = k;
@@ -809,39 +854,15 @@ __global__ void __launch_bounds__(kThreads) score_rows_kernel(const __grid_const
         }
       }
       block_argmax(bk, bb, redf, redi);
-      // ... then a token of that block (warp 0 re-reads the block's 256 tokens)
-      if (warp == 0) {
-        float tk = -INFINITY;
-        int tx = INT_MAX;
-        if (bb != INT_MAX) {
-          const int64_t xb = static_cast<int64_t>(bb) * kRaceBlock + lane * 8;
-          const uint4 wa =
-              philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 1u + static_cast<uint32_t>(xb >> 2));
-          const uint4 wb =
-              philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 2u + static_cast<uint32_t>(xb >> 2));
-          const uint32_t w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int64_t x = xb + e;
-            if (x < V) {
-              const float z = ld1(zp_row, x);
-              const bool in = !masked || (z - Mp >= logb);
-              const float v = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) : 0.f;
-              if (v > 0.f) {
-                const float key = race_key(lg2(v), w[e]);
-                if (key > tk) {
-                  tk = key;
-                  tx = static_cast<int>(x);
-                }
-              }
-            }
-          }
-        }
-        warp_argmax(tk, tx);
-        if (lane == 0) rs->term = tx;
-      }
-      __syncthreads();
-      term = rs->term;
+      // ... then a token of that block
+      term = token_race(
+          p, g, bb,
+          [&](int64_t x) -> float {
+            const float z = ld1(zp_row, x);
+            const bool in = !masked || (z - Mp >= logb);
+            return in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) : 0.f;
+          },
+          redf, redi);
     }
     if (tid == 0 && !handed_over) {
       RowRecord r;
@@ -997,15 +1018,19 @@ Layout layout_for(int N, int nblk, int nst) {
   return l;
 }
 
-// Tokens per stage: z_p and z_q fill a stage in row passes; z_p, z_q and q share it in residual
-// pieces (whole race blocks of 256 tokens either way).
-int tokens_a(int es) { return kStageBytes / (2 * es); }
+// Tokens per stage, in whole race blocks: z_p and z_q fill a stage in row passes; z_p, z_q and
+// q share it in residual pieces.
+int tokens_a(int es) { return kStageBytes / (2 * es) / kRaceBlock * kRaceBlock; }
 int tokens_r(int es) { return kStageBytes / (2 * es + 4) / kRaceBlock * kRaceBlock; }
 
-}  // namespace
+// A warp takes tok / 8 tokens of a stage in groups of 256, and whole warps cover a race block.
+bool stage_split_ok(int tok) {
+  const int tpw = tok / kWarps;
+  return tok > 0 && tok % (kWarps * kSub) == 0 && tpw <= kRaceBlock && kRaceBlock % tpw == 0 &&
+         tok / kRaceBlock <= kThreads;
+}
 
-// A residual piece covers up to kPieceStages ring stages (16384 tokens for bf16 logits).
-constexpr int kPieceStages = 4;
+}  // namespace
 
 int residual_pieces(int64_t V, int dtype) {
   const int es = dtype == DCD_BF16 ? 2 : 4;
@@ -1038,18 +1063,18 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   const int64_t R = static_cast<int64_t>(a.B) * a.N;
   if (R == 0) return cudaSuccess;
   const RowGeometry geo = row_geometry(a);
-  if (geo.smem > kSmemMax || geo.stages < 1 || geo.stages > kMaxStages || geo.ctas_per_sm < 1)
+  const int es = a.dtype == DCD_BF16 ? 2 : 4;
+  if (geo.smem > kSmemMax || geo.stages < 1 || geo.stages > kMaxStages || geo.ctas_per_sm < 1 ||
+      !stage_split_ok(tokens_a(es)) || !stage_split_ok(tokens_r(es)))
     return cudaErrorInvalidConfiguration;
   int sms = 0;
   cudaError_t e = a.dtype == DCD_BF16 ? prepare_kernel<__nv_bfloat16>(&sms) : prepare_kernel<float>(&sms);
   if (e != cudaSuccess) return e;
-  const int es = a.dtype == DCD_BF16 ? 2 : 4;
   SParams sp;
   sp.a = a;
   sp.nst = geo.stages;
   sp.tok_a = tokens_a(es);
   sp.tok_r = tokens_r(es);
-  sp.piece_stages = kPieceStages;
   sp.npieces = residual_pieces(a.V, a.dtype);
   sp.bulk = geo.bulk;
   sp.nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);

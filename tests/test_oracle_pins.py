@@ -229,11 +229,11 @@ def test_exponential_race_samples_target():
 
 @pytest.mark.parametrize("T", [1.0, 0.7])
 def test_two_level_race_samples_target_across_blocks(T):
-    """V spans several 256-token blocks (the last one ragged): the bonus is still drawn from pi_CD."""
+    """V spans several 1024-token blocks (the last one ragged): the bonus is still drawn from pi_CD."""
     rng = np.random.default_rng(78)
-    V, B = 600, 120000
+    V, B = 2500, 200000
     zp = 0.6 * rng.standard_normal(V)
-    zp[[5, 300, 599]] += 2.5  # mass in every block
+    zp[[5, 1100, 2499]] += 2.5  # mass in every block
     zq = 0.7 * zp + 0.5 * rng.standard_normal(V)
     res = oracle.verify(B=B, N=1, V=V, dtype="f64", z_exp=zp, z_ama=zq, ld=0,
                         tokens=np.zeros((B, 1), np.int32), parents=np.full((B, 1), -1, np.int32),
@@ -242,7 +242,7 @@ def test_two_level_race_samples_target_across_blocks(T):
     pi = np.exp(oracle.row_logpi(zp, zq, 0.3, 0.0, T)["logpi"])
     counts = np.bincount(res["bonus"], minlength=V)
     # block marginals and the token-level fit
-    for lo, hi in ((0, 256), (256, 512), (512, 600)):
+    for lo, hi in ((0, 1024), (1024, 2048), (2048, 2500)):
         p = pi[lo:hi].sum()
         assert abs(counts[lo:hi].sum() / B - p) < 4 * np.sqrt(p * (1 - p) / B)
     assert stats.chisquare(counts, B * pi).pvalue > 1e-4
@@ -251,8 +251,8 @@ def test_two_level_race_samples_target_across_blocks(T):
 def test_race_returns_a_point_mass_wherever_it_sits():
     """A row whose whole mass is on one token (first, last or interior of a block, or in the ragged
     last block) always yields that token, whatever the uniforms."""
-    V, B = 700, 400
-    for hot in (0, 255, 256, 511, 512, 640, 699):
+    V, B = 2100, 300
+    for hot in (0, 1023, 1024, 2047, 2048, 2070, 2099):
         zp = np.zeros(V)
         zp[hot] = 200.0  # exp(-200) leaves every other token without representable mass
         res = oracle.verify(B=B, N=1, V=V, dtype="f64", z_exp=zp, z_ama=zp, ld=0,
@@ -288,7 +288,7 @@ def _algorithm1_chain(zp_rows, zq_rows, q_rows, drafts, alpha, T, seed, offset, 
     return k - 1, _two_level_race(P, seed, offset, b * N + row)
 
 
-def _two_level_race(P, seed, offset, G, block=256):
+def _two_level_race(P, seed, offset, G, block=1024):
     """Sample from P with the library's two-level exponential race (block, then token)."""
     V = len(P)
     nb = (V + block - 1) // block
