@@ -25,8 +25,9 @@ bool shape_ok(const dcd_shape* s, bool need_q) {
 
 size_t workspace_bytes_for(const dcd_shape* s) {
   const size_t rows = static_cast<size_t>(s->B) * static_cast<size_t>(s->N);
-  const size_t raw = dcd::kWorkspaceHeader +
-                     rows * (sizeof(dcd::Job) + sizeof(dcd::RowRecord) + dcd::slot_bytes(s->V, s->logits_dtype));
+  const size_t raw = dcd::kWorkspaceHeader + dcd::part_counter_bytes(rows) +
+                     rows * (sizeof(dcd::Job) + sizeof(dcd::RowRecord) + dcd::kMaxParts * sizeof(dcd::RowPart) +
+                             dcd::slot_bytes(s->V, s->logits_dtype));
   return (raw + 255) & ~static_cast<size_t>(255);
 }
 
@@ -39,19 +40,27 @@ int check_workspace(const dcd_shape* s, const void* ws, size_t bytes) {
 struct WsView {
   dcd::WsHeader* hdr;
   dcd::Job* jobs;
+  uint32_t* pdone;
   dcd::RowRecord* rec;
+  dcd::RowPart* parts;
   unsigned char* slots;
 };
 
 WsView view(void* ws, const dcd_shape* s) {
   const size_t rows = static_cast<size_t>(s->B) * static_cast<size_t>(s->N);
-  char* base = static_cast<char*>(ws);
+  char* p = static_cast<char*>(ws);
   WsView v;
-  v.hdr = reinterpret_cast<dcd::WsHeader*>(base);
-  v.jobs = reinterpret_cast<dcd::Job*>(base + dcd::kWorkspaceHeader);
-  v.rec = reinterpret_cast<dcd::RowRecord*>(base + dcd::kWorkspaceHeader + rows * sizeof(dcd::Job));
-  v.slots = reinterpret_cast<unsigned char*>(base + dcd::kWorkspaceHeader +
-                                             rows * (sizeof(dcd::Job) + sizeof(dcd::RowRecord)));
+  v.hdr = reinterpret_cast<dcd::WsHeader*>(p);
+  p += dcd::kWorkspaceHeader;
+  v.pdone = reinterpret_cast<uint32_t*>(p);
+  p += dcd::part_counter_bytes(rows);
+  v.jobs = reinterpret_cast<dcd::Job*>(p);
+  p += rows * sizeof(dcd::Job);
+  v.rec = reinterpret_cast<dcd::RowRecord*>(p);
+  p += rows * sizeof(dcd::RowRecord);
+  v.parts = reinterpret_cast<dcd::RowPart*>(p);
+  p += rows * dcd::kMaxParts * sizeof(dcd::RowPart);
+  v.slots = reinterpret_cast<unsigned char*>(p);
   return v;
 }
 
@@ -84,7 +93,9 @@ dcd::ScoreArgs make_args(const dcd_shape* s, const void* z_exp, const void* z_am
   const WsView v = view(ws, s);
   a.hdr = v.hdr;
   a.jobs = v.jobs;
+  a.pdone = v.pdone;
   a.rec = v.rec;
+  a.parts = v.parts;
   a.slots = v.slots;
   a.force_stages = 0;
   a.force_plain = 0;

@@ -13,7 +13,8 @@
 namespace dcd {
 namespace dev {
 
-constexpr int kThreads = 256;  // threads per CTA of every row kernel
+constexpr int kThreads = 256;  // compute threads per CTA of every row kernel (the consumers of a
+                               // warp-specialised CTA)
 constexpr int kWarps = kThreads / 32;
 constexpr int kRaceBlock = 1024;                  // tokens per block of the two-level terminal race
 constexpr int kSub = 256;                         // tokens a warp handles at once (8 a lane)
@@ -102,6 +103,14 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       "%4;" ::"r"(smem_addr(dst)),
       "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
       : "memory");
+}
+
+// Ticket counter: an atomic add with acquire-release semantics at GPU scope, so that writes made
+// before it are visible to whoever draws a later ticket, and that one sees them after its own.
+__device__ __forceinline__ uint32_t atomic_add_acq_rel(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
 }
 
 __device__ __forceinline__ float ex2(float x) {
@@ -201,7 +210,18 @@ __device__ __forceinline__ float ld1(const float* p, int64_t i) { return p[i]; }
 __device__ __forceinline__ float ld1(const __nv_bfloat16* p, int64_t i) { return __bfloat162float(p[i]); }
 
 // ------------------------------------------------------------------------------------------
-// Reductions.
+// Reductions.  A block reduction synchronises the threads that take part in it: the whole CTA
+// (SyncCta), or the kThreads consumer threads of a warp-specialised CTA, whose producer warp
+// does not take part (SyncConsumers, named barrier 1).
+struct SyncCta {
+  __device__ __forceinline__ void operator()() const { __syncthreads(); }
+};
+struct SyncConsumers {
+  __device__ __forceinline__ void operator()() const {
+    asm volatile("bar.sync 1, %0;" ::"n"(kThreads) : "memory");
+  }
+};
+
 __device__ __forceinline__ void argmax_merge(float& v, int& i, float v2, int i2) {
   if (v2 > v || (v2 == v && i2 < i)) {
     v = v2;
@@ -227,34 +247,37 @@ __device__ __forceinline__ void warp_argmax(float& v, int& i) {
 }
 
 // Block reductions: every thread gets the result; the scratch is free again on return.
-__device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int* redi) {
+template <typename Sync = SyncCta>
+__device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int* redi, Sync sync = Sync()) {
   warp_argmax(v, i);
   if ((threadIdx.x & 31) == 0) {
     redf[threadIdx.x >> 5] = v;
     redi[threadIdx.x >> 5] = i;
   }
-  __syncthreads();
+  sync();
   v = redf[0];
   i = redi[0];
 #pragma unroll
   for (int w = 1; w < kWarps; ++w) argmax_merge(v, i, redf[w], redi[w]);
-  __syncthreads();
+  sync();
 }
 
-__device__ __forceinline__ float block_sum(float v, float* redf) {
+template <typename Sync = SyncCta>
+__device__ __forceinline__ float block_sum(float v, float* redf, Sync sync = Sync()) {
   v = warp_sum(v);
   if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
-  __syncthreads();
+  sync();
   float s = 0.f;
 #pragma unroll
   for (int w = 0; w < kWarps; ++w) s += redf[w];
-  __syncthreads();
+  sync();
   return s;
 }
 
 // Combines per-thread (max m, sum s of 2^(x - m), argmax) over the block in log2 units: every
 // thread gets the block max, the sum rescaled to it, and the argmax (ties to the lowest index).
-__device__ __forceinline__ void block_stats(float& m, float& s, int& arg, float* redf, int* redi) {
+template <typename Sync = SyncCta>
+__device__ __forceinline__ void block_stats(float& m, float& s, int& arg, float* redf, int* redi, Sync sync = Sync()) {
   auto merge = [](float& m1, float& s1, int& a1, float m2, float s2, int a2) {
     const float M = fmaxf(m1, m2);
     const float t1 = m1 > -INFINITY ? s1 * ex2(m1 - M) : 0.f;
@@ -271,23 +294,24 @@ __device__ __forceinline__ void block_stats(float& m, float& s, int& arg, float*
     redf[kWarps + (threadIdx.x >> 5)] = s;
     redi[threadIdx.x >> 5] = arg;
   }
-  __syncthreads();
+  sync();
   m = redf[0];
   s = redf[kWarps];
   arg = redi[0];
 #pragma unroll
   for (int w = 1; w < kWarps; ++w) merge(m, s, arg, redf[w], redf[kWarps + w], redi[w]);
-  __syncthreads();
+  sync();
 }
 
-__device__ __forceinline__ float block_max(float v, float* redf) {
+template <typename Sync = SyncCta>
+__device__ __forceinline__ float block_max(float v, float* redf, Sync sync = Sync()) {
   v = warp_max(v);
   if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = v;
-  __syncthreads();
+  sync();
   float s = -INFINITY;
 #pragma unroll
   for (int w = 0; w < kWarps; ++w) s = fmaxf(s, redf[w]);
-  __syncthreads();
+  sync();
   return s;
 }
 

@@ -7,30 +7,43 @@
 namespace dcd {
 
 // Workspace layout, all in the caller's buffer:
-//   [WsHeader, 256 B][Job x R][RowRecord x R][slot x R]
-// The header and the job list are zeroed at the start of every call; records and slots are
-// written before they are read.  R = B * N rows; a slot (SlotHead + one PiecePart per residual
-// piece) holds the chain state of a row whose first sibling was rejected.
+//   [WsHeader, 256 B][part counter x R, padded to 16 B][Job x R][RowRecord x R]
+//   [RowPart x kMaxParts x R][slot x R]
+// The header and the part counters are zeroed at the start of every call; the rest is written
+// before it is read.  R = B * N rows; a row streamed in parts leaves one RowPart
+// per part; a slot (SlotHead + one PiecePart per residual piece) holds the chain state of a row
+// whose first sibling was rejected.
 constexpr size_t kWorkspaceHeader = 256;
+constexpr int kMaxParts = 4;  // parts a row may be split into
+
+inline size_t part_counter_bytes(size_t rows) { return (rows * 4 + 15) & ~static_cast<size_t>(15); }
 
 struct WsHeader {
   uint32_t err;        // DCD_DEVERR_* bits of the call (read by dcd_get_device_error)
   uint32_t work;       // rows claimed by the streaming kernel
-  uint32_t job_alloc;  // residual passes created
-  uint32_t job_head;   // first pass that may still have unclaimed pieces
-  uint32_t nslots;     // rows handed to residual passes
-  uint32_t rows_done;  // rows whose record is written
-  uint32_t reserved[58];
+  uint32_t job_alloc;       // residual passes created
+  uint32_t jobs_published;  // passes published, in creation order
+  uint32_t nslots;          // rows handed to residual passes
+  uint32_t rows_done;       // rows whose record is written
+  uint32_t job_head;        // passes before it have every piece claimed
+  uint32_t reserved[57];
 };
 static_assert(sizeof(WsHeader) == kWorkspaceHeader, "WsHeader layout");
 
-struct Job {            // one residual pass of one row
-  int32_t slot;         // the row's slot
-  int32_t J;            // the pass (rejections so far, >= 1); 0 until published
-  uint32_t next_piece;  // pieces claimed
-  uint32_t done;        // pieces finished
+struct Job {             // one residual pass of one row, with what streaming it needs
+  int32_t slot;          // the row's slot
+  int32_t J;             // the pass (rejections so far, >= 1)
+  uint32_t next_piece;   // pieces claimed
+  uint32_t done;         // pieces finished
+  int32_t g, m;          // row, children of its node
+  uint32_t status;       // DCD_DEVERR_* bits of the row so far
+  int32_t pad0;
+  float M, S, Mp;        // the row's max, normaliser and expert max
+  float c;               // c_J of the residual this pass sums
+  float alpha, beta, T;  // the sequence's parameters
+  int32_t pad1;
 };
-static_assert(sizeof(Job) == 16, "Job layout");
+static_assert(sizeof(Job) == 64, "Job layout");
 
 struct RowRecord {
   int32_t acc_child;   // accepted child node id, -1 if none
@@ -39,6 +52,16 @@ struct RowRecord {
   int32_t reserved;
 };
 static_assert(sizeof(RowRecord) == 16, "RowRecord layout");
+
+struct RowPart {    // one part's statistics of a row streamed in parts
+  float M, S;        // max of u over the part and sum of 2^(u - M)
+  int32_t arg;       // argmax (lowest token on ties)
+  float key;         // best terminal-race block key of the part (log2 mass without the row max)
+  int32_t blk;       // its block, INT_MAX if none
+  int32_t timed_out;
+  int32_t pad[2];
+};
+static_assert(sizeof(RowPart) == 32, "RowPart layout");
 
 struct SlotHead {  // chain state of a handed-over row
   int32_t g, m;    // row, children of its node
@@ -76,7 +99,9 @@ struct ScoreArgs {
   float* cd_lse;      // may be null
   WsHeader* hdr;
   Job* jobs;
+  uint32_t* pdone;  // per row: parts finished
   RowRecord* rec;
+  RowPart* parts;   // per row: kMaxParts part statistics
   unsigned char* slots;
   int32_t force_stages;   // 0 = automatic, else the ring depth to use (tests / tuning)
   int32_t force_plain;    // 1 = plain loads instead of bulk async copies

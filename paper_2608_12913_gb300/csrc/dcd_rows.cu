@@ -1,37 +1,40 @@
 // dcd_rows.cu -- the streaming kernels of the CD verification step on sm_103a.
 //
-// score_rows_kernel: a persistent, cooperatively launched grid (a few CTAs per SM) with two
-// kinds of work.
+// score_rows_kernel: a persistent, cooperatively launched grid (a few CTAs per SM).  Each CTA
+// is warp-specialised: one producer warp claims work and streams it into a ring of 32 KB
+// shared-memory stages with bulk asynchronous copies (one "full" mbarrier per stage, completed
+// by the copies' byte count; one "empty" mbarrier per stage, on which the eight consumer warps
+// release it); the eight consumer warps compute.  The producer runs ahead across work items:
+// while the consumers finish one item (its last stages and its epilogue), the next item is
+// already claimed, described to them through a small descriptor queue, and streaming in.
+// Work comes in two kinds.
 //
-//  * Rows.  A CTA claims whole tree-node rows g = b * N + n from a work counter, in
-//    node-major order (every sequence's node 0, then every node 1, ...), so internal
-//    nodes -- the rows that may start residual work -- come first and leaves last.  A
-//    row is streamed through a ring of 32 KB shared-memory stages filled by bulk
-//    asynchronous copies that complete on one mbarrier per stage; thread 0 refills a
-//    stage as soon as the block has consumed it.  The "stats" pass computes the CD score
-//    s' = (1 + alpha) z_p - alpha z_q (Eq. 1; the two log-softmax shifts are constant per
-//    row and cancel in the normaliser) on the plausibility set P_beta of Sec. 2.1, in the
-//    scaled unit u = k2 s' (k2 = log2(e) / T, so pi_CD,T ~ 2^u).  A warp takes a
-//    contiguous eighth of each stage; every lane keeps an online max of u, a sum of
-//    2^(u - max) rescaled when its max grows, and its argmax, combined over the block at the
-//    end of the row.  With beta > 0 a "max" pass over z_p comes first.  Sampled rows also
-//    get, from the same exponentials, each 1024-token block's mass of pi_CD for a terminal
-//    race.  The greedy rule, the first sibling test of the sampled rule and the leaf race
-//    then finish the row.
+//  * Rows.  Whole tree-node rows g = b * N + n, claimed from a counter in node-major order
+//    (every sequence's node 0, then every node 1, ...), so internal nodes -- the rows that may
+//    start residual work -- come first and leaves last.  The "stats" pass computes the CD
+//    score s' = (1 + alpha) z_p - alpha z_q (Eq. 1; the two log-softmax shifts are constant
+//    per row and cancel in the normaliser) on the plausibility set P_beta of Sec. 2.1, in the
+//    scaled unit u = k2 s' (k2 = log2(e) / T, so pi_CD,T ~ 2^u).  A warp takes a contiguous
+//    eighth of each stage; every lane keeps an online max of u, a sum of 2^(u - max) rescaled
+//    when its max grows, and its argmax, combined over the consumers at the end of the row.
+//    With beta > 0 a "max" pass over z_p comes first.  Sampled rows also keep each warp's
+//    share of the row's mass, from which a leaf gets the mass of every 1024-token block for
+//    its terminal race.  The greedy rule, the first sibling test of the sampled rule and the
+//    leaf race then finish the row.
 //
-//  * Residual pieces.  After a rejected sibling, Algorithm 1 (generalised to sibling
-//    lists) needs the next residual over the whole vocabulary.  With c_0 = 0, D_0 = 1 the
-//    j-th residual is r_j = max(0, pi - c_j q) / D_j, where c_j = c_{j-1} + D_{j-1} and
-//    D_j = sum_x max(0, pi(x) - c_j q(x)) (induction on j from r_j = normalise(max(0,
-//    r_{j-1} - q))), so a pass needs only two scalars from the one before.  A row that
-//    needs a pass is handed to a job list; the pass is split into pieces of four ring
-//    stages (16384 tokens for bf16 logits) that any CTA claims before taking a new row.
-//    Each piece writes its partial sum (and, in the pass after the last sibling, its best
-//    race key) to its own slot; the CTA that finishes a pass's last piece (an atomic
-//    ticket, no waiting) sums the slots in a fixed order, tests the next sibling, and
-//    either queues the next pass or runs the terminal race.  A CTA with no row left polls
-//    for pieces until every row's record is written (bounded; all CTAs are co-resident
-//    under a cooperative launch), so the passes of late chains still spread over the GPU.
+//  * Residual pieces.  After a rejected sibling, Algorithm 1 (generalised to sibling lists)
+//    needs the next residual over the whole vocabulary.  With c_0 = 0, D_0 = 1 the j-th
+//    residual is r_j = max(0, pi - c_j q) / D_j, where c_j = c_{j-1} + D_{j-1} and D_j =
+//    sum_x max(0, pi(x) - c_j q(x)) (induction on j from r_j = normalise(max(0, r_{j-1} -
+//    q))), so a pass needs only two scalars from the one before.  A row that needs a pass is
+//    handed to a job list; the pass is split into pieces of four ring stages (16384 tokens for
+//    bf16 logits) that any CTA's producer claims before taking a new row.  Each piece writes
+//    its partial sum (and, in the pass after the last sibling, its best race key) to its own
+//    slot; the CTA that finishes a pass's last piece (an atomic ticket, no waiting) sums the
+//    slots in a fixed order, tests the next sibling, and either queues the next pass or runs
+//    the terminal race.  A producer with no row left polls for pieces until every row's record
+//    is written (bounded; all CTAs are co-resident under a cooperative launch), so the passes
+//    of late chains still spread over the GPU.
 //
 //  A node without an accepted child draws its terminal token by a two-level exponential
 //  race: a 1024-token block by its mass, then a token of that block (four tokens a thread,
@@ -63,12 +66,14 @@ using namespace dev;
 constexpr int kStageBytes = DCD_STAGE_KIB * 1024;  // bytes per ring stage
 constexpr int kMaxStages = 8;
 constexpr int kPieceStages = 4;                    // ring stages per residual piece
+constexpr int kDesc = 4;                           // work descriptors in flight per CTA
+constexpr int kCtaThreads = kThreads + 32;         // eight consumer warps and one producer warp
+constexpr int kMinCtasPerSm = 3;
 constexpr size_t kSmemMax = 227 * 1024;
 constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr float kLn2 = 0.69314718055994531f;
 
-enum PassKind { kPassMax = 0, kPassStats = 1 };
-enum WorkKind { kWorkNone = 0, kWorkRow = 1, kWorkPiece = 2 };
+enum WorkKind { kWorkNone = 0, kWorkRow = 1, kWorkPiece = 2, kWorkPart = 3 };
 
 // ------------------------------------------------------------------------------------------
 struct SParams {
@@ -79,34 +84,45 @@ struct SParams {
   int32_t npieces;       // pieces per residual pass
   int32_t bulk;          // 1: bulk asynchronous copies, 0: plain loads
   int32_t nblk;          // race blocks per row, ceil(V / 1024)
+  int32_t nchunk;        // warp chunks per row in the stats pass, ceil(V / (tok_a / 8))
   int32_t meta_offset;   // byte offsets into dynamic shared memory
-  int32_t blk_offset;
+  int32_t chunk_offset;
   int32_t stage_offset;
   int32_t slot_bytes;
+  int32_t r_whole;       // row items streamed whole; the rows after them are streamed in parts
+  int32_t parts;         // parts of such a row (stages of the stats pass split in runs of spp)
+  int32_t spp;           // stats-pass stages per part
+  int32_t items;         // row items: r_whole + (R - r_whole) * parts
   WsHeader* hdr;         // counters, zeroed before the launch
   Job* jobs;             // residual passes (zeroed before the launch)
   unsigned char* slots;  // per handed-over row: SlotHead + npieces PieceParts
 };
 
-// Row / piece state shared by the block (written by one thread, read after a barrier).
+// A work item as the producer hands it to the consumers.
+struct WorkDesc {
+  int32_t kind;        // WorkKind
+  int32_t g;           // row
+  int32_t job, piece;  // residual piece: job index and piece index; row part: part index
+  int32_t J;           // residual pass (rejections so far)
+  int32_t slot;        // slot of the handed-over row
+  int32_t m;           // children of the row's node
+  uint32_t status;     // DCD_DEVERR_* bits carried by the slot
+  float alpha, beta, T;
+  float M, S, Mp, c;   // pieces: the row's max, normaliser, expert max and c_J
+  int32_t pad;
+};
+static_assert(sizeof(WorkDesc) == 64, "WorkDesc layout");
+
+// Consumer state shared by the eight consumer warps (written by one thread, read after a
+// consumer barrier).
 struct RowShared {
-  int32_t next;      // the next claimed row item
-  int32_t kind;      // WorkKind of the current work
-  int32_t item;      // row item or job index
-  int32_t piece;     // piece index
-  int32_t m;         // children of the row's node
-  uint32_t status;   // DCD_DEVERR_* bits
-  int32_t accept;    // outcome of a sibling test
-  int32_t term;      // winning race block of a completed pass
-  int32_t last;      // this CTA finished a pass's last piece
-  int32_t degen;     // a pass found no residual mass left
-  int32_t slot;      // slot of the handed-over row
-  int32_t J;         // residual pass index (rejections so far)
-  int32_t g;         // row of the piece
-  float M, S, Mp, c, D;
-  int32_t pad[2];
-  float wref[2][kWarps];  // per-warp shares of race-block masses, double-buffered by stage
-  float wsum[2][kWarps];
+  int32_t m;        // children of the row's node
+  uint32_t status;  // DCD_DEVERR_* bits
+  int32_t accept;   // outcome of a sibling test
+  int32_t term;     // winning race block of a completed pass
+  int32_t last;     // this CTA finished a pass's last piece
+  int32_t degen;    // a pass found no residual mass left
+  float c, D;
 };
 
 template <typename TIn>
@@ -129,9 +145,6 @@ __device__ __forceinline__ Stage<TIn> stage_at(unsigned char* base, int s, int t
 __device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
   return *reinterpret_cast<const volatile uint32_t*>(p);
 }
-__device__ __forceinline__ int32_t ld_volatile(const int32_t* p) {
-  return *reinterpret_cast<const volatile int32_t*>(p);
-}
 
 __device__ __forceinline__ SlotHead* slot_head(const SParams& sp, int s) {
   return reinterpret_cast<SlotHead*>(sp.slots + static_cast<size_t>(s) * sp.slot_bytes);
@@ -141,15 +154,34 @@ __device__ __forceinline__ PiecePart* slot_parts(const SParams& sp, int s) {
   return reinterpret_cast<PiecePart*>(sp.slots + static_cast<size_t>(s) * sp.slot_bytes + sizeof(SlotHead));
 }
 
-// Publishes residual pass J of slot s (thread 0 of the creating CTA).
-__device__ __forceinline__ void create_job(const SParams& sp, int s, int J) {
+// Publishes residual pass `job` (its counters are reset here; one consumer thread).  Passes are
+// published in creation order, so the passes with unclaimed pieces are the window [job_head,
+// jobs_published); the wait for the previous creator spans a few stores and is bounded.
+__device__ __forceinline__ void create_job(const SParams& sp, Job job) {
   const uint32_t k = atomicAdd(&sp.hdr->job_alloc, 1u);
-  Job* job = &sp.jobs[k];
-  job->slot = s;
-  job->next_piece = 0u;
-  job->done = 0u;
+  job.next_piece = 0u;
+  job.done = 0u;
+  job.pad0 = job.pad1 = 0;
+  sp.jobs[k] = job;
   __threadfence();
-  *reinterpret_cast<volatile int32_t*>(&job->J) = J;
+  const long long t0 = clock64();
+  while (ld_volatile(&sp.hdr->jobs_published) != k) {
+    if (clock64() - t0 > kWaitCycles) {
+      atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+      break;
+    }
+  }
+  *reinterpret_cast<volatile uint32_t*>(&sp.hdr->jobs_published) = k + 1u;
+}
+
+// A published pass record, read past the non-coherent L1.
+__device__ __forceinline__ Job load_job(const Job* j) {
+  Job r;
+  const int4* src = reinterpret_cast<const int4*>(j);
+  int4* dst = reinterpret_cast<int4*>(&r);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) dst[i] = __ldcg(src + i);
+  return r;
 }
 
 // Lists the children of node n (ascending id) into kids / ktok with the calling warp; returns
@@ -224,9 +256,9 @@ __device__ bool sibling_test(const ScoreArgs& p, int b, int node, int t, const T
 }
 
 // Second level of the terminal race: the token x of race block `kstar` with the largest
-// log2 r(x) - log2(-log2 u_x), four tokens a thread (one Philox call, counter 1 + x / 4).
-// `mass(x)` returns r(x) up to a common factor.  Every thread of the block calls it and gets
-// the token (INT_MAX when no block had mass).
+// log2 r(x) - log2(-log2 u_x), four tokens a consumer thread (one Philox call, counter
+// 1 + x / 4).  `mass(x)` returns r(x) up to a common factor.  Every consumer thread calls it
+// and gets the token (INT_MAX when no block had mass).
 template <typename MassFn>
 __device__ int token_race(const ScoreArgs& p, int64_t g, int kstar, MassFn mass, float* redf, int* redi) {
   float tk = -INFINITY;
@@ -252,181 +284,342 @@ __device__ int token_race(const ScoreArgs& p, int64_t g, int kstar, MassFn mass,
       }
     }
   }
-  block_argmax(tk, tx, redf, redi);
+  block_argmax(tk, tx, redf, redi, SyncConsumers());
   return tx;
 }
 
 // First level of the race for one block: its key from log2 of its mass.
 __device__ __forceinline__ float block_key(const ScoreArgs& p, int64_t g, int k, float log2_mass) {
-  const uint4 w = philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (static_cast<uint32_t>(k) >> 2));
+  const uint4 w =
+      philox_block(p.seed, p.offset, static_cast<uint32_t>(g), 0x80000000u | (static_cast<uint32_t>(k) >> 2));
   return race_key(log2_mass, word_of(w, k & 3));
+}
+
+__device__ __forceinline__ void warp_release(uint64_t* bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
 }
 
 // ------------------------------------------------------------------------------------------
 template <typename TIn>
-__global__ void __launch_bounds__(kThreads, 3) score_rows_kernel(const __grid_constant__ SParams sp) {
+__global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(const __grid_constant__ SParams sp) {
   const ScoreArgs& p = sp.a;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int N = p.N;
   const int64_t V = p.V;
   const int R = p.B * N;
-  const int nch_a = static_cast<int>((V + sp.tok_a - 1) / sp.tok_a);  // chunks of a max / stats pass
+  const int nch_a = static_cast<int>((V + sp.tok_a - 1) / sp.tok_a);  // stages of a max / stats pass
+  const SyncConsumers csync;
 
   extern __shared__ __align__(128) unsigned char smem[];
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem);             // [kMaxStages]
-  float* redf = reinterpret_cast<float*>(smem + 8 * kMaxStages);  // [32]
-  int* redi = reinterpret_cast<int*>(redf + 32);                  // [32]
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem);  // [kMaxStages] stage filled
+  uint64_t* empty = full + kMaxStages;                 // [kMaxStages] stage released by the consumers
+  uint64_t* dfull = empty + kMaxStages;                // [kDesc] descriptor written
+  uint64_t* dempty = dfull + kDesc;                    // [kDesc] descriptor released
+  float* redf = reinterpret_cast<float*>(dempty + kDesc);  // [32]
+  int* redi = reinterpret_cast<int*>(redf + 32);           // [32]
+  WorkDesc* desc = reinterpret_cast<WorkDesc*>(redi + 32); // [kDesc]
   RowShared* rs = reinterpret_cast<RowShared*>(smem + sp.meta_offset);
-  int* kids = reinterpret_cast<int*>(rs + 1);                     // [N] children, ascending id
-  int* ktok = kids + N;                                           // [N] their tokens
-  float* czp = reinterpret_cast<float*>(ktok + N);                // [N] z_p at those tokens
-  float* czq = czp + N;                                           // [N] z_q at those tokens
-  float* cq = czq + N;                                            // [N] q at those tokens
-  float* bmax = reinterpret_cast<float*>(smem + sp.blk_offset);   // [nblk] block reference of u
-  float* bsum = bmax + sp.nblk;                                   // [nblk] block sum of 2^(u - ref)
+  int* kids = reinterpret_cast<int*>(rs + 1);                    // [N] children, ascending id
+  int* ktok = kids + N;                                          // [N] their tokens
+  float* czp = reinterpret_cast<float*>(ktok + N);               // [N] z_p at those tokens
+  float* czq = czp + N;                                          // [N] z_q at those tokens
+  float* cq = czq + N;                                           // [N] q at those tokens
+  float* cref = reinterpret_cast<float*>(smem + sp.chunk_offset);  // [nchunk] warp chunk reference
+  float* csum = cref + sp.nchunk;                                // [nchunk] chunk sum of 2^(u - ref)
   unsigned char* ring = smem + sp.stage_offset;
 
   if (tid == 0) {
-    for (int s = 0; s < sp.nst; ++s) mbar_init(&full[s], 1);
+    for (int s = 0; s < sp.nst; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kWarps);
+    }
+    for (int d = 0; d < kDesc; ++d) {
+      mbar_init(&dfull[d], 1);
+      mbar_init(&dempty[d], 1);
+    }
     fence_mbar_init();
-    rs->next = static_cast<int32_t>(atomicAdd(&sp.hdr->work, 1u));
   }
-  __syncthreads();
-  const uint64_t pol_last = l2_policy_evict_last();
-  const uint64_t pol_first = l2_policy_evict_first();
-  uint32_t seq = 0;  // ring items consumed by this CTA so far (identical in every thread)
+  __syncthreads();  // the last CTA-wide barrier: from here on the two roles synchronise by mbarriers
 
-  // Waits for ring item `sq`, then fills a ragged or unaligned remainder with plain loads.
-  auto wait_stage = [&](uint32_t sq, const Stage<TIn>& st, const TIn* zp_row, const TIn* zq_row,
-                        const float* q_row, int64_t x0, int clen, bool with_zq, bool with_q, bool& timed_out) {
-    const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-    const uint32_t parity = (sq / static_cast<uint32_t>(sp.nst)) & 1u;
-    if (!mbar_wait_bounded(&full[s], parity)) timed_out = true;
-    const int zfirst =
-        sp.bulk ? ((clen * static_cast<int>(sizeof(TIn))) & ~15) / static_cast<int>(sizeof(TIn)) : 0;
-    const int qfirst = sp.bulk ? ((clen * 4) & ~15) / 4 : 0;
-    if (zfirst < clen || (with_q && qfirst < clen)) {
-      for (int i = zfirst + tid; i < clen; i += kThreads) {
-        st.zp[i] = zp_row[x0 + i];
-        if (with_zq) st.zq[i] = zq_row[x0 + i];
+  if (warp == kWarps) {
+    // ===================================== producer warp
+    const uint64_t pol_last = l2_policy_evict_last();
+    const uint64_t pol_first = l2_policy_evict_first();
+    uint32_t issued = 0;  // ring items issued
+
+    // The next row item and what streaming it needs are fetched while the current item streams,
+    // so switching items costs no dependent round trip; `nr` is claimed one ahead.
+    struct RowMeta {
+      int item, g, part, m;
+      float alpha, beta, T;
+    };
+    auto load_meta = [&](int item) -> RowMeta {  // the whole warp, `item` uniform
+      RowMeta mt;
+      mt.item = item;
+      mt.g = -1;
+      mt.part = -1;
+      mt.m = 0;
+      mt.alpha = mt.beta = mt.T = 0.f;
+      if (item >= sp.items) return mt;
+      int r = item;  // row items: whole rows in node-major order, then parts of the last rows
+      if (item >= sp.r_whole) {
+        r = sp.r_whole + (item - sp.r_whole) / sp.parts;
+        mt.part = (item - sp.r_whole) % sp.parts;
       }
-      if (with_q)
-        for (int i = qfirst + tid; i < clen; i += kThreads) st.q[i] = q_row[x0 + i];
-      __syncthreads();
-    }
-  };
+      const int b = r % p.B, n = r / p.B;
+      mt.g = b * N + n;
+      mt.alpha = p.alpha[b];
+      mt.beta = p.beta ? p.beta[b] : 0.f;
+      mt.T = p.temp ? p.temp[b] : 0.f;
+      const int32_t* parr = p.parents + static_cast<int64_t>(b) * N;  // children of node n
+      for (int base = n + 1; base < N; base += 32) {
+        const int c = base + lane;
+        mt.m += __popc(__ballot_sync(~0u, c < N && parr[c] == n));
+      }
+      return mt;
+    };
+    int nr = 0;  // lane 0: the next row item (its claim returns while the current item streams)
+    if (lane == 0) nr = static_cast<int>(atomicAdd(&sp.hdr->work, 1u));
+    RowMeta meta;
+    bool meta_stale = true;  // `meta` was used; the next one is fetched after the next issue
+    auto refresh_meta = [&]() {  // the whole warp
+      nr = __shfl_sync(~0u, nr, 0);
+      meta = load_meta(nr);
+      meta_stale = false;
+    };
+    refresh_meta();
+    uint32_t pub_seen = 0u, head_seen = 0u;  // job-list state read before the last issue (lane 0)
 
-  for (;;) {
-    // ---- next work: a residual piece if one can be claimed, else the next row.  With no row
-    // left, a CTA stays (all CTAs are co-resident: cooperative launch) until every row's record
-    // is written, to take pieces of passes other CTAs queue; the wait is bounded.
-    if (tid == 0) {
-      int kind = kWorkNone, job = -1, piece = 0;
-      const long long t0 = clock64();
-      for (;;) {
-        const uint32_t alloc = ld_volatile(&sp.hdr->job_alloc);
-        for (uint32_t k = ld_volatile(&sp.hdr->job_head); k < alloc; ++k) {
-          if (ld_volatile(&sp.jobs[k].J) == 0) break;  // not yet published
-          const uint32_t pc = atomicAdd(&sp.jobs[k].next_piece, 1u);
-          if (pc < static_cast<uint32_t>(sp.npieces)) {
-            job = static_cast<int>(k);
-            piece = static_cast<int>(pc);
-            break;
+    for (uint32_t w = 0;; ++w) {
+      // ---- claim: a residual piece if one is available, else the next row item; with no row
+      // item left, poll (bounded) for pieces until every row's record is written.  The last row
+      // items are parts of rows, so the rows still streaming at the end are spread over more CTAs.
+      int kind = kWorkNone;
+      WorkDesc D;
+      int nitems = 0, tok = sp.tok_a, nmax = 0;  // items; tokens per item; leading max-pass items
+      bool with_q = false;
+      uint64_t pol = pol_first;
+      int64_t x_lo = 0;
+      for (bool skip = true; skip;) {
+        skip = false;
+        if (meta_stale) refresh_meta();  // after a skipped part
+        int item = 0, piece = 0;
+        kind = kWorkNone;
+        Job job_rec;  // lane 0: the claimed pass
+        if (lane == 0) {
+          const long long t0 = clock64();
+          for (int poll = 0;; ++poll) {
+            // a piece of the oldest published pass that still has one (the first look uses the
+            // state read during the last issue).  The scan reaches pass k only after finding every
+            // pass between the head and k without pieces, so whoever claims the last piece of k
+            // may move the head past it.
+            const uint32_t pub = poll ? ld_volatile(&sp.hdr->jobs_published) : pub_seen;
+            for (uint32_t k = poll ? ld_volatile(&sp.hdr->job_head) : head_seen; k < pub; ++k) {
+              const uint32_t pc = atomicAdd(&sp.jobs[k].next_piece, 1u);
+              if (pc < static_cast<uint32_t>(sp.npieces)) {
+                if (pc + 1u == static_cast<uint32_t>(sp.npieces)) atomicMax(&sp.hdr->job_head, k + 1u);
+                kind = kWorkPiece;
+                item = static_cast<int>(k);
+                piece = static_cast<int>(pc);
+                __threadfence();  // the record was written before the pass was published
+                job_rec = load_job(&sp.jobs[k]);
+                break;
+              }
+            }
+            if (kind != kWorkNone) break;
+            if (meta.g >= 0) {
+              kind = kWorkRow;
+              nr = static_cast<int>(atomicAdd(&sp.hdr->work, 1u));  // its result is read after the next issue
+              break;
+            }
+            if (poll && ld_volatile(&sp.hdr->rows_done) >= static_cast<uint32_t>(R)) break;
+            if (clock64() - t0 > kWaitCycles) {
+              atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+              break;
+            }
+            if (poll) __nanosleep(256);
           }
-          atomicMax(&sp.hdr->job_head, k + 1u);
         }
-        if (job >= 0) {
-          kind = kWorkPiece;
-          rs->item = job;
-          rs->piece = piece;
-          break;
-        }
-        if (rs->next < R) {
-          kind = kWorkRow;
-          rs->item = rs->next;
-          rs->next = static_cast<int32_t>(atomicAdd(&sp.hdr->work, 1u));
-          break;
-        }
-        if (ld_volatile(&sp.hdr->rows_done) >= static_cast<uint32_t>(R)) break;
-        if (clock64() - t0 > kWaitCycles) {
-          atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
-          break;
-        }
-        __nanosleep(256);
-      }
-      rs->kind = kind;
-    }
-    __syncthreads();
-    const int kind = rs->kind;
-    if (kind == kWorkNone) break;
+        kind = __shfl_sync(~0u, kind, 0);
+        item = __shfl_sync(~0u, item, 0);
+        piece = __shfl_sync(~0u, piece, 0);
 
-    if (kind == kWorkPiece) {
-      // ================= one piece of residual pass J of a handed-over row
-      if (tid == 0) {
-        __threadfence();  // the job and its slot were written before J was published
-        const Job* job = &sp.jobs[rs->item];
-        const int s = ld_volatile(&job->slot);
-        const SlotHead* sh = slot_head(sp, s);
-        rs->slot = s;
-        rs->J = ld_volatile(&job->J);
-        rs->g = sh->g;
-        rs->m = sh->m;
-        rs->M = sh->M;
-        rs->S = sh->S;
-        rs->Mp = sh->Mp;
-        rs->c = sh->c + sh->D;  // c_J = c_{J-1} + D_{J-1}
-        rs->status = sh->status;
+        D.kind = kind;
+        D.g = 0;
+        D.job = item;
+        D.piece = piece;
+        D.J = 0;
+        D.slot = 0;
+        D.m = 0;
+        D.status = 0u;
+        D.alpha = D.beta = D.T = 0.f;
+        D.M = D.S = D.Mp = D.c = 0.f;
+        D.pad = 0;
+        nitems = 0;
+        tok = sp.tok_a;
+        nmax = 0;
+        with_q = false;
+        pol = pol_first;
+        x_lo = 0;
+        if (kind == kWorkRow) {
+          meta_stale = true;
+          D.g = meta.g;
+          D.m = meta.m;
+          D.alpha = meta.alpha;
+          D.beta = meta.beta;
+          D.T = meta.T;
+          const bool masked = D.beta > 0.f;
+          const bool sampled = D.T > 0.f && p.q != nullptr;
+          // a sampled internal row keeps its logits in L2 for residual passes
+          pol = (sampled && meta.m > 0) ? pol_last : pol_first;
+          if (meta.part >= 0 && !masked) {
+            D.kind = kWorkPart;
+            D.piece = meta.part;
+            x_lo = static_cast<int64_t>(meta.part) * sp.spp * sp.tok_a;
+            nitems = nch_a - meta.part * sp.spp < sp.spp ? nch_a - meta.part * sp.spp : sp.spp;
+          } else if (meta.part > 0) {
+            skip = true;  // a beta > 0 row needs its expert max first: its part 0 streams it whole
+          } else {
+            nmax = masked ? nch_a : 0;
+            nitems = nmax + nch_a;
+          }
+        } else if (kind == kWorkPiece) {
+          if (lane == 0) {
+            D.slot = job_rec.slot;
+            D.J = job_rec.J;
+            D.g = job_rec.g;
+            D.m = job_rec.m;
+            D.M = job_rec.M;
+            D.S = job_rec.S;
+            D.Mp = job_rec.Mp;
+            D.c = job_rec.c;
+            D.status = job_rec.status;
+            D.alpha = job_rec.alpha;
+            D.beta = job_rec.beta;
+            D.T = job_rec.T;
+          }
+          D.g = __shfl_sync(~0u, D.g, 0);
+          D.J = __shfl_sync(~0u, D.J, 0);
+          D.m = __shfl_sync(~0u, D.m, 0);
+          tok = sp.tok_r;
+          x_lo = static_cast<int64_t>(piece) * kPieceStages * sp.tok_r;
+          const int64_t rem = (V - x_lo + sp.tok_r - 1) / sp.tok_r;
+          nitems = static_cast<int>(rem < kPieceStages ? rem : kPieceStages);
+          with_q = true;
+          pol = D.J < D.m ? pol_last : pol_first;  // the pass after the last sibling is the last read
+        }
       }
-      __syncthreads();
-      const int64_t g = rs->g;
-      const int J = rs->J, m = rs->m, piece = rs->piece;
-      const int b = static_cast<int>(g / N);
-      const float alpha = p.alpha[b];
-      const float beta = p.beta ? p.beta[b] : 0.f;
-      const float T = p.temp[b];
-      const bool masked = beta > 0.f;
-      const float k2 = kLog2e / T;
-      const float c1k = (1.f + alpha) * k2, ak = alpha * k2;  // u = k2 s' = c1k z_p - ak z_q
-      const float logb = masked ? logf(beta) : -INFINITY;
-      const float M = rs->M, invS = 1.f / rs->S, Mp = rs->Mp, cJ = rs->c;
-      const bool race = J == m;  // the pass after the last sibling also ranks race blocks
+      // ---- publish the descriptor
+      if (lane == 0) {
+        const int d = static_cast<int>(w % kDesc);
+        if (!mbar_wait_bounded(&dempty[d], ((w / kDesc) & 1u) ^ 1u)) atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+        desc[d] = D;
+        mbar_arrive(&dfull[d]);
+      }
+      if (kind == kWorkNone) break;
+
+      // ---- stream the item's stages
+      const int64_t g = D.g;
       const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
       const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
+      const float* q_row = with_q ? p.q + g * p.ldq : nullptr;
+      for (int L = 0; L < nitems; ++L, ++issued) {
+        const int s = static_cast<int>(issued % static_cast<uint32_t>(sp.nst));
+        const uint32_t phase = ((issued / static_cast<uint32_t>(sp.nst)) & 1u) ^ 1u;
+        const bool maxpass = L < nmax;
+        const int64_t x0 = x_lo + static_cast<int64_t>(maxpass ? L : L - nmax) * tok;
+        const int clen = static_cast<int>((V - x0) < tok ? (V - x0) : tok);
+        const Stage<TIn> st = stage_at<TIn>(ring, s, tok);
+        if (lane == 0 && L == nitems - 1) {  // read for the next claim while the stage drains
+          pub_seen = ld_volatile(&sp.hdr->jobs_published);
+          head_seen = ld_volatile(&sp.hdr->job_head);
+        }
+        if (lane == 0 && !mbar_wait_bounded(&empty[s], phase)) atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+        __syncwarp();
+        if (!sp.bulk) {
+          // plain loads (rows whose start or stride is not 16-byte aligned)
+          for (int i = lane; i < clen; i += 32) {
+            st.zp[i] = zp_row[x0 + i];
+            if (!maxpass) st.zq[i] = zq_row[x0 + i];
+            if (with_q) st.q[i] = q_row[x0 + i];
+          }
+          __threadfence_block();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&full[s]);
+        } else if (lane == 0) {
+          // bulk copies of the 16-byte multiple; the ragged remainder is stored first
+          const int zfirst = ((clen * static_cast<int>(sizeof(TIn))) & ~15) / static_cast<int>(sizeof(TIn));
+          const int qfirst = ((clen * 4) & ~15) / 4;
+          for (int i = zfirst; i < clen; ++i) {
+            st.zp[i] = zp_row[x0 + i];
+            if (!maxpass) st.zq[i] = zq_row[x0 + i];
+          }
+          if (with_q)
+            for (int i = qfirst; i < clen; ++i) st.q[i] = q_row[x0 + i];
+          const uint32_t zb = static_cast<uint32_t>(zfirst) * static_cast<uint32_t>(sizeof(TIn));
+          const uint32_t qb = with_q ? static_cast<uint32_t>(qfirst) * 4u : 0u;
+          const uint64_t pl = maxpass ? pol_last : pol;  // the stats pass re-reads the max pass
+          mbar_arrive_expect_tx(&full[s], (maxpass ? zb : 2u * zb) + qb);
+          if (zb) {
+            bulk_g2s(st.zp, zp_row + x0, zb, &full[s], pl);
+            if (!maxpass) bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pl);
+          }
+          if (qb) bulk_g2s(st.q, q_row + x0, qb, &full[s], pl);
+        }
+        if (L == 0 && meta_stale) refresh_meta();  // the next row item's metadata, while this item streams
+      }
+    }
+    return;
+  }
+
+  // ===================================== consumer warps
+  uint32_t seq = 0;  // ring items consumed (identical in every consumer thread)
+  bool timed_out = false;
+  auto wait_full = [&](uint32_t sq) {
+    if (!mbar_wait_bounded(&full[sq % static_cast<uint32_t>(sp.nst)], (sq / static_cast<uint32_t>(sp.nst)) & 1u))
+      timed_out = true;
+  };
+
+  for (uint32_t w = 0;; ++w) {
+    const int d = static_cast<int>(w % kDesc);
+    if (!mbar_wait_bounded(&dfull[d], (w / kDesc) & 1u)) {
+      if (tid == 0) atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+      break;
+    }
+    const WorkDesc D = desc[d];
+    if (D.kind == kWorkNone) break;
+    timed_out = false;
+
+    const int64_t g = D.g;
+    const int b = static_cast<int>(g / N), n = static_cast<int>(g % N);
+    const float alpha = D.alpha, beta = D.beta, T = D.T;
+    const bool masked = beta > 0.f;
+    const float k2 = kLog2e * (T > 0.f ? 1.f / T : 1.f);  // exp(x / T) = 2^(x * k2)
+    // scores are kept in the scaled unit u = k2 s' = c1k z_p - ak z_q, so pi_CD,T ~ 2^u
+    const float c1k = (1.f + alpha) * k2, ak = alpha * k2;
+    const float logb = masked ? logf(beta) : -INFINITY;
+    const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
+    const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
+
+    if (D.kind == kWorkPiece) {
+      // ================= one piece of residual pass J of a handed-over row
+      const int J = D.J, m = D.m, piece = D.piece;
+      const float M = D.M, invS = 1.f / D.S, Mp = D.Mp, cJ = D.c;
+      const bool race = J == m;  // the pass after the last sibling also ranks race blocks
       const float* q_row = p.q + g * p.ldq;
-      // the piece's stages, streamed through the ring like a row; a warp takes tok_r / 8
-      // consecutive tokens of each stage, so `wpb` warps cover one race block
+      // a warp takes tok_r / 8 consecutive tokens of each stage (a chunk); `wpb` chunks make a
+      // race block
       const int tpw = sp.tok_r / kWarps, wpb = kRaceBlock / tpw;
       const int64_t piece_lo = static_cast<int64_t>(piece) * kPieceStages * sp.tok_r;
       const int64_t rem = (V - piece_lo + sp.tok_r - 1) / sp.tok_r;
       const int nst_piece = static_cast<int>(rem < kPieceStages ? rem : kPieceStages);
-      const uint32_t seq0 = seq;
-      auto issue_piece = [&](int L) {  // thread 0 only
-        const uint32_t sq = seq0 + static_cast<uint32_t>(L);
-        const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-        const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_r);
+      float zl = 0.f;
+      for (int L = 0; L < nst_piece; ++L, ++seq) {
+        const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(sp.nst)), sp.tok_r);
         const int64_t x0 = piece_lo + static_cast<int64_t>(L) * sp.tok_r;
         const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
-        const uint32_t zb = sp.bulk ? static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u : 0u;
-        const uint32_t qb = sp.bulk ? static_cast<uint32_t>(clen * 4) & ~15u : 0u;
-        mbar_arrive_expect_tx(&full[s], 2u * zb + qb);
-        if (zb) {
-          bulk_g2s(st.zp, zp_row + x0, zb, &full[s], pol_last);
-          bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pol_last);
-        }
-        if (qb) bulk_g2s(st.q, q_row + x0, qb, &full[s], pol_last);
-      };
-      if (tid == 0)
-        for (int L = 0; L < nst_piece && L < sp.nst; ++L) issue_piece(L);
-      bool timed_out = false;
-      float zl = 0.f, bk = -INFINITY;
-      int bb = INT_MAX;
-      for (int L = 0; L < nst_piece; ++L) {
-        const uint32_t sq = seq0 + static_cast<uint32_t>(L);
-        const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(sq % static_cast<uint32_t>(sp.nst)), sp.tok_r);
-        const int64_t x0 = piece_lo + static_cast<int64_t>(L) * sp.tok_r;
-        const int clen = static_cast<int>((V - x0) < sp.tok_r ? (V - x0) : sp.tok_r);
-        const int par = L & 1;
-        wait_stage(sq, st, zp_row, zq_row, q_row, x0, clen, true, true, timed_out);
+        wait_full(seq);
         float part = 0.f;
         for (int sb = warp * tpw; sb < (warp + 1) * tpw && sb < clen; sb += kSub) {  // warp-uniform
           const int i0 = sb + lane * 8;
@@ -440,197 +633,180 @@ __global__ void __launch_bounds__(kThreads, 3) score_rows_kernel(const __grid_co
         zl += part;
         if (race) {
           const float ws = warp_sum(part);
-          if (lane == 0) rs->wsum[par][warp] = ws;
+          if (lane == 0) csum[L * kWarps + warp] = ws;
         }
-        __syncthreads();
-        if (tid == 0 && L + sp.nst < nst_piece) issue_piece(L + sp.nst);
-        // block masses of the last pass's residual (read while the next stage streams in; the
-        // shares are double-buffered, so the next stage's writes go to the other half)
-        if (race && tid < sp.tok_r / kRaceBlock && x0 + static_cast<int64_t>(tid) * kRaceBlock < V) {
-          float mass = 0.f;
-          for (int w = 0; w < wpb; ++w) mass += rs->wsum[par][tid * wpb + w];
-          if (mass > 0.f) {
-            const int kabs = static_cast<int>(x0 / kRaceBlock) + tid;
-            const float key = block_key(p, g, kabs, lg2(mass));
-            if (key > bk) {
-              bk = key;
-              bb = kabs;
-            }
-          }
+        warp_release(&empty[seq % static_cast<uint32_t>(sp.nst)]);
+      }
+      const float zsum = block_sum(zl, redf, csync);  // its barriers also publish csum
+      // race keys of the piece's blocks (the pass after the last sibling)
+      float bk = -INFINITY;
+      int bb = INT_MAX;
+      if (race && tid < nst_piece * (sp.tok_r / kRaceBlock) &&
+          piece_lo + static_cast<int64_t>(tid) * kRaceBlock < V) {
+        float mass = 0.f;
+        for (int i = 0; i < wpb; ++i) mass += csum[tid * wpb + i];
+        if (mass > 0.f) {
+          const int kabs = static_cast<int>(piece_lo / kRaceBlock) + tid;
+          bk = block_key(p, g, kabs, lg2(mass));
+          bb = kabs;
         }
       }
-      seq = seq0 + static_cast<uint32_t>(nst_piece);
-      const float zsum = block_sum(zl, redf);
-      block_argmax(bk, bb, redf, redi);
+      block_argmax(bk, bb, redf, redi, csync);
       if (tid == 0) {
         PiecePart pp;
         pp.z = zsum;
         pp.key = bk;
         pp.blk = bb;
         pp.timed_out = timed_out ? 1 : 0;
-        slot_parts(sp, rs->slot)[piece] = pp;
-        __threadfence();
-        const uint32_t t = atomicAdd(&sp.jobs[rs->item].done, 1u);
+        slot_parts(sp, D.slot)[piece] = pp;
+        const uint32_t t = atomic_add_acq_rel(&sp.jobs[D.job].done, 1u);
         rs->last = t + 1u == static_cast<uint32_t>(sp.npieces) ? 1 : 0;
       }
-      __syncthreads();
-      if (!rs->last) continue;
-
-      // ================= the pass is complete: next sibling test, next pass or terminal race
-      const int n = static_cast<int>(g % N);
-      if (warp == 0) list_children(p, b, n, kids, ktok);
-      if (tid == 0) {
-        __threadfence();  // every piece's part was written before its ticket
-        SlotHead* sh = slot_head(sp, rs->slot);
-        const PiecePart* parts = slot_parts(sp, rs->slot);
-        float DJ = 0.f, K = -INFINITY;
-        int kstar = INT_MAX;
-        uint32_t st2 = sh->status;
-        for (int k = 0; k < sp.npieces; ++k) {
-          DJ += parts[k].z;
-          argmax_merge(K, kstar, parts[k].key, parts[k].blk);
-          if (parts[k].timed_out) st2 |= DCD_DEVERR_TIMEOUT;
-        }
-        bool degen = sh->degen != 0;
-        float c = sh->c, D = sh->D;
-        if (DJ > 0.f) {
-          c = cJ;
-          D = DJ;
-        } else {
-          degen = true;  // r_{J-1} == q in exact arithmetic: r_J is taken as q from here on
-        }
-        // test the remaining siblings; after a pass without residual mass no pass is needed
-        int acc = -1;
-        bool queued = false;
-        for (int j = J; j < m; ++j) {
-          if (sibling_test<TIn>(p, b, kids[j], ktok[j], zp_row, zq_row, q_row, c1k, ak, masked, Mp, logb, M, invS, c,
-                                D, degen)) {
-            acc = kids[j];
-            break;
+      csync();
+      if (rs->last) {
+        // ================= the pass is complete: next sibling test, next pass or terminal race
+        if (warp == 0) list_children(p, b, n, kids, ktok);
+        if (tid == 0) {
+          SlotHead* sh = slot_head(sp, D.slot);
+          const PiecePart* parts = slot_parts(sp, D.slot);
+          float DJ = 0.f, K = -INFINITY;
+          int kstar = INT_MAX;
+          uint32_t st2 = D.status;
+          for (int k = 0; k < sp.npieces; ++k) {
+            DJ += parts[k].z;
+            argmax_merge(K, kstar, parts[k].key, parts[k].blk);
+            if (parts[k].timed_out) st2 |= DCD_DEVERR_TIMEOUT;
           }
-          if (!degen) {
-            sh->c = c;
-            sh->D = D;
-            sh->degen = 0;
-            sh->status = st2;
-            create_job(sp, rs->slot, j + 1);
-            queued = true;
-            break;
+          bool degen = sh->degen != 0;
+          float c = sh->c, Dn = sh->D;
+          if (DJ > 0.f) {
+            c = cJ;
+            Dn = DJ;
+          } else {
+            degen = true;  // r_{J-1} == q in exact arithmetic: r_J is taken as q from here on
           }
-        }
-        rs->accept = queued ? -2 : acc;
-        rs->term = kstar;  // the winning race block when this pass ranked them
-        rs->status = st2;
-        rs->c = c;
-        rs->D = D;
-        rs->degen = degen ? 1 : 0;
-      }
-      __syncthreads();
-      if (rs->accept == -2) continue;  // the next pass is queued
-      const int acc = rs->accept;
-      int term = -1;
-      if (acc < 0) {
-        // every sibling rejected: terminal draw from r_m, or from q after a pass without mass
-        const bool degen = rs->degen != 0;
-        const float c = rs->c, D = rs->D;
-        int kstar = rs->term;
-        if (degen) {
-          // block masses of q, computed by this CTA alone (rare: a residual without mass)
-          float bk2 = -INFINITY;
-          int bb2 = INT_MAX;
-          for (int kb = warp; kb < sp.nblk; kb += kWarps) {
-            float part = 0.f;
-            for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < V && x < (kb + 1) * kRaceBlock;
-                 x += 32)
-              part += q_row[x];
-            const float mass = warp_sum(part);
-            if (lane == 0 && mass > 0.f) {
-              const float key = block_key(p, g, kb, lg2(mass));
-              if (key > bk2) {
-                bk2 = key;
-                bb2 = kb;
-              }
+          // test the remaining siblings; after a pass without residual mass no pass is needed
+          int acc = -1;
+          bool queued = false;
+          for (int j = J; j < m; ++j) {
+            if (sibling_test<TIn>(p, b, kids[j], ktok[j], zp_row, zq_row, q_row, c1k, ak, masked, Mp, logb, M, invS,
+                                  c, Dn, degen)) {
+              acc = kids[j];
+              break;
+            }
+            if (!degen) {
+              sh->c = c;
+              sh->D = Dn;
+              sh->degen = 0;
+              sh->status = st2;
+              Job nj;
+              nj.slot = D.slot;
+              nj.J = j + 1;
+              nj.g = static_cast<int32_t>(g);
+              nj.m = m;
+              nj.status = st2;
+              nj.M = M;
+              nj.S = D.S;
+              nj.Mp = Mp;
+              nj.c = c + Dn;  // c_{J+1} = c_J + D_J
+              nj.alpha = alpha;
+              nj.beta = beta;
+              nj.T = T;
+              create_job(sp, nj);
+              queued = true;
+              break;
             }
           }
-          block_argmax(bk2, bb2, redf, redi);
-          kstar = bb2;
+          rs->accept = queued ? -2 : acc;
+          rs->term = kstar;  // the winning race block when this pass ranked them
+          rs->status = st2;
+          rs->c = c;
+          rs->D = Dn;
+          rs->degen = degen ? 1 : 0;
         }
-        term = token_race(
-            p, g, kstar,
-            [&](int64_t x) -> float {
-              const float qe = q_row[x];
-              if (degen) return qe;
-              const float z = ld1(zp_row, x);
-              const bool in = !masked || (z - Mp >= logb);
-              const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
-              return fmaxf(pit - c * qe, 0.f) / D;
-            },
-            redf, redi);
+        csync();
+        const int acc = rs->accept;
+        if (acc != -2) {
+          int term = -1;
+          if (acc < 0) {
+            // every sibling rejected: terminal draw from r_m, or from q after a pass without mass
+            const bool degen = rs->degen != 0;
+            const float c = rs->c, Dn = rs->D;
+            int kstar = rs->term;
+            if (degen) {
+              // block masses of q, computed by this CTA alone (rare: a residual without mass)
+              float bk2 = -INFINITY;
+              int bb2 = INT_MAX;
+              for (int kb = warp; kb < sp.nblk; kb += kWarps) {
+                float part = 0.f;
+                for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < V && x < (kb + 1) * kRaceBlock;
+                     x += 32)
+                  part += q_row[x];
+                const float mass = warp_sum(part);
+                if (lane == 0 && mass > 0.f) {
+                  const float key = block_key(p, g, kb, lg2(mass));
+                  if (key > bk2) {
+                    bk2 = key;
+                    bb2 = kb;
+                  }
+                }
+              }
+              block_argmax(bk2, bb2, redf, redi, csync);
+              kstar = bb2;
+            }
+            term = token_race(
+                p, g, kstar,
+                [&](int64_t x) -> float {
+                  const float qe = q_row[x];
+                  if (degen) return qe;
+                  const float z = ld1(zp_row, x);
+                  const bool in = !masked || (z - Mp >= logb);
+                  const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
+                  return fmaxf(pit - c * qe, 0.f) / Dn;
+                },
+                redf, redi);
+          }
+          if (tid == 0) {
+            RowRecord r;
+            r.acc_child = acc;
+            r.term_token = acc < 0 ? term : -1;
+            r.status = rs->status;
+            r.reserved = 0;
+            p.rec[g] = r;
+            atomicAdd(&sp.hdr->rows_done, 1u);  // only counts: records are read after the kernel
+          }
+        }
       }
-      if (tid == 0) {
-        RowRecord r;
-        r.acc_child = acc;
-        r.term_token = acc < 0 ? term : -1;
-        r.status = rs->status;
-        r.reserved = 0;
-        p.rec[g] = r;
-        __threadfence();
-        atomicAdd(&sp.hdr->rows_done, 1u);
-      }
-      __syncthreads();
+      csync();  // consumer state in shared memory is rewritten by the next work
+      if (tid == 0) mbar_arrive(&dempty[d]);
       continue;
     }
 
-    // ================= a row
-    const int item = rs->item;
-    const int b = item % p.B, n = item / p.B;  // node-major order
-    const int64_t g = static_cast<int64_t>(b) * N + n;
-    const float alpha = p.alpha[b];
-    const float beta = p.beta ? p.beta[b] : 0.f;
-    const float T = p.temp ? p.temp[b] : 0.f;
+    // ================= a row, or a part of one
+    const bool is_part = D.kind == kWorkPart;
     const bool sampled = T > 0.f && p.q != nullptr;
-    const bool masked = beta > 0.f;
-    const float invT = T > 0.f ? 1.f / T : 1.f;
-    const float k2 = kLog2e * invT;  // exp(x / T) = 2^(x * k2)
-    // scores are kept in the scaled unit u = k2 s' = c1k z_p - ak z_q, so pi_CD,T ~ 2^u
-    const float c1k = (1.f + alpha) * k2, ak = alpha * k2;
-    const float logb = masked ? logf(beta) : -INFINITY;
-    const TIn* zp_row = static_cast<const TIn*>(p.zp) + g * p.ld;
-    const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
+    const bool leaf_race = sampled && D.m == 0;  // a sampled leaf draws its terminal token here
     const float* q_row = sampled ? p.q + g * p.ldq : nullptr;
+    const int L0 = is_part ? D.piece * sp.spp : 0;  // the stats pass's stages [L0, L0 + nL)
+    const int nL = is_part ? (nch_a - L0 < sp.spp ? nch_a - L0 : sp.spp) : nch_a;
 
-    // ring items of this row: [max pass if beta > 0] [stats pass]; thread 0 keeps up to nst
-    // items in flight
-    const int nknown = (masked ? 2 : 1) * nch_a;
-    const uint32_t seq0 = seq;
-    auto pass_of = [&](int L) -> int { return (masked && L < nch_a) ? kPassMax : kPassStats; };
-    auto issue = [&](int L, uint64_t pol) {  // thread 0 only
-      const uint32_t sq = seq0 + static_cast<uint32_t>(L);
-      const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-      const int64_t x0 = static_cast<int64_t>(L % nch_a) * sp.tok_a;
-      const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
-      const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_a);
-      const int kind2 = pass_of(L);
-      const uint32_t zb = sp.bulk ? static_cast<uint32_t>(clen * static_cast<int>(sizeof(TIn))) & ~15u : 0u;
-      mbar_arrive_expect_tx(&full[s], kind2 == kPassMax ? zb : 2u * zb);
-      if (zb) {
-        bulk_g2s(st.zp, zp_row + x0, zb, &full[s], pol);
-        if (kind2 != kPassMax) bulk_g2s(st.zq, zq_row + x0, zb, &full[s], pol);
-      }
-    };
-
-    // Thread 0 starts the row's stream at once.  A beta > 0 row keeps its max pass in L2 for
-    // the stats pass, and a sampled row its logits for residual pieces until it is known to be
-    // a leaf.  Warp 1 meanwhile lists the children of node n, checks the row and loads the
-    // values at the children's tokens, which are consumed after the stats pass; the first
-    // stage barrier publishes the child count.
-    if (tid == 0) {
-      const uint64_t pol0 = (masked || sampled) ? pol_last : pol_first;
-      const int first = nknown < sp.nst ? nknown : sp.nst;
-      for (int L = 0; L < first; ++L) issue(L, pol0);
-    }
+    // a whole row: warp 1 lists the children of node n, checks the row and loads the values at
+    // the children's tokens while the stats pass streams; they are consumed after it
     float pzp = 0.f, pzq = 0.f, pq = 0.f;
-    if (warp == 1) {
+    auto check_row = [&](int count) {  // lane 0 of the listing warp
+      uint32_t st = 0u;
+      const int pp = p.parents[static_cast<int64_t>(b) * N + n];
+      if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
+      if (n > 0) {
+        const int t = p.tokens[static_cast<int64_t>(b) * N + n];
+        if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
+      }
+      if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
+        st |= DCD_DEVERR_BAD_PARAM;
+      rs->m = count;
+      rs->status = st;
+    };
+    if (!is_part && warp == 1) {
       const int count = list_children(p, b, n, kids, ktok);
       if (lane < count) {
         const int t = ktok[lane];
@@ -640,146 +816,200 @@ __global__ void __launch_bounds__(kThreads, 3) score_rows_kernel(const __grid_co
           if (sampled) pq = q_row[t];
         }
       }
-      if (lane == 0) {
-        uint32_t st = 0u;
-        const int pp = p.parents[static_cast<int64_t>(b) * N + n];
-        if (n == 0 ? pp != -1 : (pp < 0 || pp >= n)) st |= DCD_DEVERR_BAD_PARENT;
-        if (n > 0) {
-          const int t = p.tokens[static_cast<int64_t>(b) * N + n];
-          if (t < 0 || t >= V) st |= DCD_DEVERR_BAD_TOKEN;
-        }
-        if (!(alpha >= 0.f && alpha <= 3.0e38f) || !(beta >= 0.f && beta <= 1.f) || !(T >= 0.f && T <= 3.0e38f))
-          st |= DCD_DEVERR_BAD_PARAM;
-        rs->m = count;
-        rs->status = st;
-      }
+      if (lane == 0) check_row(count);
     }
 
-    int L = 0;  // next item to consume
-    bool timed_out = false;
-    // Consumes `count` items: waits for each stage, hands it to `body`, refills the stage once
-    // the block has finished it, then runs `after` (which may read what `body` left in shared
-    // memory, double-buffered by item parity).
-    auto run_items = [&](int count, auto&& body, auto&& after) {
-      for (int it = 0; it < count; ++it, ++L) {
-        const uint32_t sq = seq0 + static_cast<uint32_t>(L);
-        const int s = static_cast<int>(sq % static_cast<uint32_t>(sp.nst));
-        const int64_t x0 = static_cast<int64_t>(L % nch_a) * sp.tok_a;
-        const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
-        const Stage<TIn> st = stage_at<TIn>(ring, s, sp.tok_a);
-        wait_stage(sq, st, zp_row, zq_row, nullptr, x0, clen, pass_of(L) != kPassMax, false, timed_out);
-        body(st, x0, clen, L & 1);
-        __syncthreads();
-        if (tid == 0 && L + sp.nst < nknown) {
-          const bool keep = (masked && L + sp.nst < nch_a) || (sampled && rs->m > 0);
-          issue(L + sp.nst, keep ? pol_last : pol_first);
-        }
-        after(x0, clen, L & 1);
-      }
-    };
-    auto no_after = [](int64_t, int, int) {};
-
-    // ---- pass A (beta > 0): the expert max, for P_beta = {x : z_p(x) - max z_p >= log beta}
+    // ---- pass A (beta > 0, whole rows): the expert max, for P_beta = {x : z_p(x) - max z_p >=
+    // log beta}
     float Mp = 0.f;
     if (masked) {
       float lm = -INFINITY;
-      run_items(
-          nch_a,
-          [&](const Stage<TIn>& st, int64_t, int clen, int) {
-            for (int i0 = tid * 8; i0 < clen; i0 += kThreads * 8) {
-              float zp[8];
-              ld8(st.zp + i0, zp);
+      for (int L = 0; L < nch_a; ++L, ++seq) {
+        const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(sp.nst)), sp.tok_a);
+        const int64_t x0 = static_cast<int64_t>(L) * sp.tok_a;
+        const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
+        wait_full(seq);
+        for (int i0 = tid * 8; i0 < clen; i0 += kThreads * 8) {
+          float zp[8];
+          ld8(st.zp + i0, zp);
 #pragma unroll
-              for (int e = 0; e < 8; ++e)
-                if (i0 + e < clen) lm = fmaxf(lm, zp[e]);
-            }
-          },
-          no_after);
-      Mp = block_max(lm, redf);
+          for (int e = 0; e < 8; ++e)
+            if (i0 + e < clen) lm = fmaxf(lm, zp[e]);
+        }
+        warp_release(&empty[seq % static_cast<uint32_t>(sp.nst)]);
+      }
+      Mp = block_max(lm, redf, csync);
     }
 
     // ---- pass B: per lane an online max of u on P_beta, the sum of 2^(u - max) rescaled when
-    // the max grows, and the argmax.  A warp takes tok_a / 8 consecutive tokens of each stage, so
-    // `wpb` warps cover one race block; for sampled rows each warp also reports its share of the
-    // stage's mass, which threads 0.. combine into the block masses after the stage barrier.
+    // the max grows, and the argmax.  A warp takes tok_a / 8 consecutive tokens (a chunk) of each
+    // stage; for a sampled leaf it also records the chunk's mass relative to a chunk reference.
     const int tpw = sp.tok_a / kWarps, wpb = kRaceBlock / tpw;
     float lmax = -INFINITY, lsum = 0.f;
     int larg = INT_MAX;
-    run_items(
-        nch_a,
-        [&](const Stage<TIn>& st, int64_t x0, int clen, int par) {
-          float bpart = 0.f;  // this lane's share of the warp's mass in this stage, relative to lmax
-          for (int sb = warp * tpw; sb < (warp + 1) * tpw && sb < clen; sb += kSub) {  // warp-uniform
-            const int i0 = sb + lane * 8;
-            float u[8];
-            scores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
-            const float gm = max8(u);
-            if (gm > lmax) {
-              const float f = ex2(lmax - gm);  // 0 while lmax is -inf
-              lsum *= f;
-              bpart *= f;
-              lmax = gm;
+    for (int L = L0; L < L0 + nL; ++L, ++seq) {
+      const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(sp.nst)), sp.tok_a);
+      const int64_t x0 = static_cast<int64_t>(L) * sp.tok_a;
+      const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
+      wait_full(seq);
+      float bpart = 0.f;  // this lane's share of the chunk's mass, relative to lmax
+      for (int sb = warp * tpw; sb < (warp + 1) * tpw && sb < clen; sb += kSub) {  // warp-uniform
+        const int i0 = sb + lane * 8;
+        float u[8];
+        scores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
+        const float gm = max8(u);
+        if (gm > lmax) {
+          const float f = ex2(lmax - gm);  // 0 while lmax is -inf
+          lsum *= f;
+          bpart *= f;
+          lmax = gm;
 #pragma unroll
-              for (int e = 7; e >= 0; --e)
-                if (u[e] == gm) larg = static_cast<int>(x0) + i0 + e;
-            }
-            if (lmax > -INFINITY) {
-              const float2 nm2 = make_float2(-lmax, -lmax);
-              float2 acc2 = make_float2(0.f, 0.f);
+          for (int e = 7; e >= 0; --e)
+            if (u[e] == gm) larg = static_cast<int>(x0) + i0 + e;
+        }
+        if (lmax > -INFINITY) {
+          const float2 nm2 = make_float2(-lmax, -lmax);
+          float2 acc2 = make_float2(0.f, 0.f);
 #pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                const float2 d = __fadd2_rn(make_float2(u[2 * k], u[2 * k + 1]), nm2);
-                acc2 = __fadd2_rn(acc2, make_float2(ex2(d.x), ex2(d.y)));
-              }
-              const float a = acc2.x + acc2.y;
-              lsum += a;
-              bpart += a;
-            }
+          for (int k = 0; k < 4; ++k) {
+            const float2 dd = __fadd2_rn(make_float2(u[2 * k], u[2 * k + 1]), nm2);
+            acc2 = __fadd2_rn(acc2, make_float2(ex2(dd.x), ex2(dd.y)));
           }
-          if (sampled) {
-            const float ref = warp_max(lmax);
-            const float ws = warp_sum(lmax > -INFINITY ? bpart * ex2(lmax - ref) : 0.f);
-            if (lane == 0) {
-              rs->wref[par][warp] = ref;
-              rs->wsum[par][warp] = ws;
-            }
-          }
-        },
-        [&](int64_t x0, int clen, int par) {
-          if (sampled && tid < sp.tok_a / kRaceBlock && tid * kRaceBlock < clen) {
-            float ref = -INFINITY, sum = 0.f;
-            for (int w = 0; w < wpb; ++w) ref = fmaxf(ref, rs->wref[par][tid * wpb + w]);
-            if (ref > -INFINITY)
-              for (int w = 0; w < wpb; ++w) {
-                const float r = rs->wref[par][tid * wpb + w];
-                if (r > -INFINITY) sum += rs->wsum[par][tid * wpb + w] * ex2(r - ref);
-              }
-            const int kabs = static_cast<int>(x0 / kRaceBlock) + tid;
-            bmax[kabs] = ref;
-            bsum[kabs] = sum;
-          }
-        });
-    seq = seq0 + static_cast<uint32_t>(L);
-    const int m = rs->m;
-    if (warp == 1 && lane < m) {
-      czp[lane] = pzp;
-      czq[lane] = pzq;
-      cq[lane] = pq;
+          const float a = acc2.x + acc2.y;
+          lsum += a;
+          bpart += a;
+        }
+      }
+      if (leaf_race) {
+        const float ref = warp_max(lmax);
+        const float ws = warp_sum(lmax > -INFINITY ? bpart * ex2(lmax - ref) : 0.f);
+        if (lane == 0 && x0 + static_cast<int64_t>(warp) * tpw < V) {
+          const int ch = static_cast<int>(x0 / tpw) + warp;
+          cref[ch] = ref;
+          csum[ch] = ws;
+        }
+      }
+      warp_release(&empty[seq % static_cast<uint32_t>(sp.nst)]);
     }
-    for (int k = 32 + tid; k < m; k += kThreads) {  // nodes with more children than a warp has lanes
-      const int t = ktok[k];
-      const bool ok = t >= 0 && t < V;
-      czp[k] = ok ? ld1(zp_row, t) : 0.f;
-      czq[k] = ok ? ld1(zq_row, t) : 0.f;
-      cq[k] = (ok && sampled) ? q_row[t] : 0.f;
-    }
-    // row statistics (the reduction's barriers also publish czp / czq / cq and the block masses):
-    // M = max u, S = sum 2^(u - M), so log sum exp(s' / T) = M ln 2 + ln S
+    // statistics of the streamed range (the reduction's barriers also publish the chunk masses
+    // and warp 1's child list): M = max u, S = sum 2^(u - M), argmax
     float M = lmax, S = lsum;
     int arg = larg;
-    block_stats(M, S, arg, redf, redi);
-    uint32_t status = rs->status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
+    block_stats(M, S, arg, redf, redi, csync);
+
+    // First level of a leaf's terminal race over the blocks of the streamed range: the key of a
+    // block is log2 of its mass 2^ref * (rescaled chunk sum) against its uniform; the row max is
+    // left out (a common shift), so parts of a row rank their blocks on one scale.
+    auto best_block = [&](float& bk, int& bb) {
+      const int nch_row = static_cast<int>((V + tpw - 1) / tpw);  // chunks a row has
+      const int k_lo = static_cast<int>(static_cast<int64_t>(L0) * sp.tok_a / kRaceBlock);
+      int k_hi = static_cast<int>(static_cast<int64_t>(L0 + nL) * sp.tok_a / kRaceBlock);
+      if (k_hi > sp.nblk) k_hi = sp.nblk;
+      bk = -INFINITY;
+      bb = INT_MAX;
+      for (int k = k_lo + tid; k < k_hi; k += kThreads) {
+        float ref = -INFINITY, sum = 0.f;
+        for (int i = 0; i < wpb && k * wpb + i < nch_row; ++i) ref = fmaxf(ref, cref[k * wpb + i]);
+        if (ref > -INFINITY)
+          for (int i = 0; i < wpb && k * wpb + i < nch_row; ++i) {
+            const float r = cref[k * wpb + i];
+            if (r > -INFINITY) sum += csum[k * wpb + i] * ex2(r - ref);
+          }
+        if (ref > -INFINITY && sum > 0.f) {
+          const float key = block_key(p, g, k, lg2(sum) + ref);
+          if (key > bk) {
+            bk = key;
+            bb = k;
+          }
+        }
+      }
+      block_argmax(bk, bb, redf, redi, csync);
+    };
+
+    uint32_t status;
+    int m, kstar = INT_MAX;
+    if (is_part) {
+      // ---- a part: publish its statistics; the CTA that finishes a row's last part combines
+      // them and finishes the row
+      float bk = -INFINITY;
+      int bb = INT_MAX;
+      if (leaf_race) best_block(bk, bb);
+      if (tid == 0) {
+        RowPart rp;
+        rp.M = M;
+        rp.S = S;
+        rp.arg = arg;
+        rp.key = bk;
+        rp.blk = bb;
+        rp.timed_out = timed_out ? 1 : 0;
+        rp.pad[0] = rp.pad[1] = 0;
+        p.parts[g * kMaxParts + D.piece] = rp;
+        const uint32_t t = atomic_add_acq_rel(&p.pdone[g], 1u);
+        rs->last = t + 1u == static_cast<uint32_t>(sp.parts) ? 1 : 0;
+      }
+      csync();
+      if (!rs->last) {
+        if (tid == 0) mbar_arrive(&dempty[d]);
+        continue;  // no consumer state of this part is read again
+      }
+      if (tid == 0) {
+        float cM = -INFINITY, cS = 0.f, K = -INFINITY;
+        int carg = INT_MAX, kb = INT_MAX, tmo = 0;
+        for (int k = 0; k < sp.parts; ++k) {  // a fixed order: the result does not depend on timing
+          const RowPart rp = p.parts[g * kMaxParts + k];
+          const float nM = fmaxf(cM, rp.M);
+          cS = (cM > -INFINITY ? cS * ex2(cM - nM) : 0.f) + (rp.M > -INFINITY ? rp.S * ex2(rp.M - nM) : 0.f);
+          if (rp.M > cM || (rp.M == cM && rp.arg < carg)) carg = rp.arg;
+          cM = nM;
+          argmax_merge(K, kb, rp.key, rp.blk);
+          tmo |= rp.timed_out;
+        }
+        rs->c = cM;  // (consumer scratch: the combined statistics)
+        rs->D = cS;
+        rs->accept = carg;
+        rs->term = kb;
+        rs->degen = tmo;
+      }
+      if (warp == 1) {
+        const int count = list_children(p, b, n, kids, ktok);
+        if (lane == 0) check_row(count);
+      }
+      csync();
+      M = rs->c;
+      S = rs->D;
+      arg = rs->accept;
+      kstar = rs->term;
+      m = rs->m;
+      status = rs->status | (rs->degen ? DCD_DEVERR_TIMEOUT : 0u);
+      for (int k = tid; k < m; k += kThreads) {
+        const int t = ktok[k];
+        const bool ok = t >= 0 && t < V;
+        czp[k] = ok ? ld1(zp_row, t) : 0.f;
+        czq[k] = ok ? ld1(zq_row, t) : 0.f;
+        cq[k] = (ok && sampled) ? q_row[t] : 0.f;
+      }
+      csync();
+    } else {
+      m = rs->m;
+      if (warp == 1 && lane < m) {
+        czp[lane] = pzp;
+        czq[lane] = pzq;
+        cq[lane] = pq;
+      }
+      for (int k = 32 + tid; k < m; k += kThreads) {  // nodes with more children than a warp has lanes
+        const int t = ktok[k];
+        const bool ok = t >= 0 && t < V;
+        czp[k] = ok ? ld1(zp_row, t) : 0.f;
+        czq[k] = ok ? ld1(zq_row, t) : 0.f;
+        cq[k] = (ok && sampled) ? q_row[t] : 0.f;
+      }
+      status = rs->status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
+      float bk = -INFINITY;
+      if (leaf_race) best_block(bk, kstar);  // its barriers also publish czp / czq / cq
+      else csync();
+    }
     if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
+    // log sum exp(s' / T) over P_beta = M ln 2 + ln S
     const float logS = logf(S);
     const float invS = 1.f / S;
 
@@ -831,32 +1061,32 @@ __global__ void __launch_bounds__(kThreads, 3) score_rows_kernel(const __grid_co
           sh->D = 1.f;
           sh->degen = 0;
           sh->status = status;
-          create_job(sp, s, 1);
+          Job nj;
+          nj.slot = s;
+          nj.J = 1;
+          nj.g = static_cast<int32_t>(g);
+          nj.m = m;
+          nj.status = status;
+          nj.M = M;
+          nj.S = S;
+          nj.Mp = Mp;
+          nj.c = 1.f;  // c_1 = c_0 + D_0
+          nj.alpha = alpha;
+          nj.beta = beta;
+          nj.T = T;
+          create_job(sp, nj);
           accept = -1;
         }
         rs->accept = accept;
       }
-      __syncthreads();
+      csync();
       if (rs->accept == 1) acc = kids[0];
       if (rs->accept == -1) handed_over = true;
     } else {
-      // ---- sampled leaf: the terminal token is drawn from pi_CD,T by the two-level race: a
-      // 1024-token block by its mass 2^(bmax - M) bsum ...
-      float bk = -INFINITY;
-      int bb = INT_MAX;
-      for (int k = tid; k < sp.nblk; k += kThreads) {
-        if (bmax[k] > -INFINITY && bsum[k] > 0.f) {
-          const float key = block_key(p, g, k, lg2(bsum[k]) + (bmax[k] - M));
-          if (key > bk) {
-            bk = key;
-            bb = k;
-          }
-        }
-      }
-      block_argmax(bk, bb, redf, redi);
-      // ... then a token of that block
+      // ---- sampled leaf: the terminal token is drawn from pi_CD,T by the two-level race: the
+      // block kstar won by its mass, then a token of that block
       term = token_race(
-          p, g, bb,
+          p, g, kstar,
           [&](int64_t x) -> float {
             const float z = ld1(zp_row, x);
             const bool in = !masked || (z - Mp >= logb);
@@ -871,10 +1101,10 @@ __global__ void __launch_bounds__(kThreads, 3) score_rows_kernel(const __grid_co
       r.status = status;
       r.reserved = 0;
       p.rec[g] = r;
-      __threadfence();
-      atomicAdd(&sp.hdr->rows_done, 1u);
+      atomicAdd(&sp.hdr->rows_done, 1u);  // only counts: records and outputs are read after the kernel
     }
-    __syncthreads();  // row state in shared memory is rewritten by the next work
+    csync();  // consumer state in shared memory is rewritten by the next work
+    if (tid == 0) mbar_arrive(&dempty[d]);
   }
 }
 
@@ -1003,17 +1233,20 @@ cudaError_t prepare_kernel(int* sms) {
 }
 
 struct Layout {
-  int meta_offset, blk_offset, stage_offset;
+  int meta_offset, chunk_offset, stage_offset;
   size_t total;
 };
 
-Layout layout_for(int N, int nblk, int nst) {
+// Dynamic shared memory: mbarriers, reduction scratch and descriptors; consumer state and the
+// child lists; chunk masses; the ring.
+Layout layout_for(int N, int nchunk, int nst) {
   Layout l;
-  l.meta_offset = 8 * kMaxStages + 64 * 4;
+  const size_t fixed = 8 * (2 * kMaxStages + 2 * kDesc) + 64 * 4 + sizeof(WorkDesc) * kDesc;
+  l.meta_offset = static_cast<int>((fixed + 15) & ~static_cast<size_t>(15));
   const size_t meta_end = static_cast<size_t>(l.meta_offset) + sizeof(RowShared) + static_cast<size_t>(N) * 4 * 5;
-  l.blk_offset = static_cast<int>((meta_end + 15) & ~static_cast<size_t>(15));
-  const size_t blk_end = static_cast<size_t>(l.blk_offset) + static_cast<size_t>(nblk) * 4 * 2;
-  l.stage_offset = static_cast<int>((blk_end + 127) & ~static_cast<size_t>(127));
+  l.chunk_offset = static_cast<int>((meta_end + 15) & ~static_cast<size_t>(15));
+  const size_t chunk_end = static_cast<size_t>(l.chunk_offset) + static_cast<size_t>(nchunk) * 4 * 2;
+  l.stage_offset = static_cast<int>((chunk_end + 127) & ~static_cast<size_t>(127));
   l.total = static_cast<size_t>(l.stage_offset) + static_cast<size_t>(nst) * kStageBytes;
   return l;
 }
@@ -1023,11 +1256,19 @@ Layout layout_for(int N, int nblk, int nst) {
 int tokens_a(int es) { return kStageBytes / (2 * es) / kRaceBlock * kRaceBlock; }
 int tokens_r(int es) { return kStageBytes / (2 * es + 4) / kRaceBlock * kRaceBlock; }
 
-// A warp takes tok / 8 tokens of a stage in groups of 256, and whole warps cover a race block.
+// A warp takes tok / 8 tokens of a stage in groups of 256, whole chunks make a race block, and
+// a piece's chunks fit the chunk arrays.
 bool stage_split_ok(int tok) {
   const int tpw = tok / kWarps;
   return tok > 0 && tok % (kWarps * kSub) == 0 && tpw <= kRaceBlock && kRaceBlock % tpw == 0 &&
-         tok / kRaceBlock <= kThreads;
+         kPieceStages * (tok / kRaceBlock) <= kThreads;
+}
+
+int chunks_per_row(int64_t V, int es) {
+  const int tpw = tokens_a(es) / kWarps;
+  const int64_t rows_chunks = (V + tpw - 1) / tpw;
+  const int piece_chunks = kPieceStages * kWarps;  // csum slots a residual piece uses
+  return static_cast<int>(rows_chunks > piece_chunks ? rows_chunks : piece_chunks);
 }
 
 }  // namespace
@@ -1045,9 +1286,8 @@ size_t slot_bytes(int64_t V, int dtype) {
 RowGeometry row_geometry(const ScoreArgs& a) {
   RowGeometry geo{};
   const int es = a.dtype == DCD_BF16 ? 2 : 4;
-  const int nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
-  const int nst = a.force_stages > 0 ? a.force_stages : 2;
-  const Layout l = layout_for(a.N, nblk, nst);
+  const int nst = a.force_stages > 0 ? a.force_stages : (kStageBytes >= 32768 ? 2 : 65536 / kStageBytes);
+  const Layout l = layout_for(a.N, chunks_per_row(a.V, es), nst);
   const int per_sm = static_cast<int>(kSmemPerSm / (l.total + 1024));
   geo.stages = nst;
   geo.stage_tokens = tokens_a(es);
@@ -1078,31 +1318,43 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.npieces = residual_pieces(a.V, a.dtype);
   sp.bulk = geo.bulk;
   sp.nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
-  const Layout l = layout_for(a.N, sp.nblk, sp.nst);
+  sp.nchunk = chunks_per_row(a.V, es);
+  const Layout l = layout_for(a.N, sp.nchunk, sp.nst);
   sp.meta_offset = l.meta_offset;
-  sp.blk_offset = l.blk_offset;
+  sp.chunk_offset = l.chunk_offset;
   sp.stage_offset = l.stage_offset;
   sp.slot_bytes = static_cast<int32_t>(slot_bytes(a.V, a.dtype));
   sp.hdr = a.hdr;
   sp.jobs = a.jobs;
   sp.slots = a.slots;
-  // the header counters and the job list start every call at zero
-  e = cudaMemsetAsync(a.hdr, 0, kWorkspaceHeader + static_cast<size_t>(R) * sizeof(Job), stream);
+  // the header counters and the part counters start every call at zero
+  e = cudaMemsetAsync(a.hdr, 0, kWorkspaceHeader + part_counter_bytes(static_cast<size_t>(R)), stream);
   if (e != cudaSuccess) return e;
   // a CTA may wait for work queued by another, so all CTAs must be resident at once: the grid is
   // the resident capacity (capped at the row count) and the launch is cooperative
   int per_sm = 0;
-  e = a.dtype == DCD_BF16
-          ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<__nv_bfloat16>, kThreads, geo.smem)
-          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<float>, kThreads, geo.smem);
+  e = a.dtype == DCD_BF16 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<__nv_bfloat16>,
+                                                                          kCtaThreads, geo.smem)
+                          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<float>,
+                                                                          kCtaThreads, geo.smem);
   if (e != cudaSuccess) return e;
   if (per_sm > geo.ctas_per_sm) per_sm = geo.ctas_per_sm;
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
-  int64_t grid = static_cast<int64_t>(sms) * per_sm;
-  if (grid > R) grid = R;
+  const int64_t resident = static_cast<int64_t>(sms) * per_sm;
+  // The last rows (as many as CTAs, or all of a small batch) are streamed in parts of spp
+  // stages each, so the rows still in flight at the end of the step are spread over more CTAs.
+  const int nch_a = static_cast<int>((a.V + sp.tok_a - 1) / sp.tok_a);
+  const int want = nch_a < kMaxParts ? nch_a : kMaxParts;
+  sp.spp = (nch_a + want - 1) / want;
+  sp.parts = (nch_a + sp.spp - 1) / sp.spp;
+  const int64_t tail = sp.parts > 1 ? (R < resident ? R : resident) : 0;
+  sp.r_whole = static_cast<int32_t>(R - tail);
+  sp.items = static_cast<int32_t>(sp.r_whole + tail * sp.parts);
+  int64_t grid = resident;
+  if (grid > sp.items) grid = sp.items;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid));
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kCtaThreads);
   cfg.dynamicSmemBytes = geo.smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];

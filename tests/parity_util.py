@@ -32,8 +32,9 @@ AMB_MASK = 1e-5
 
 
 def records(ws: torch.Tensor, R: int):
-    """Per-row records the kernels leave in the workspace (after the 256-byte header and R jobs)."""
-    off = 256 + 16 * R
+    """Per-row records the kernels leave in the workspace (after the 256-byte header, R 4-byte
+    part counters padded to 16 bytes and R 64-byte residual-pass records)."""
+    off = 256 + (4 * R + 15) // 16 * 16 + 64 * R
     raw = ws[off:off + 16 * R].cpu().numpy().view(np.int32).reshape(R, 4)
     return dict(acc_child=raw[:, 0].copy(), term_token=raw[:, 1].copy(), status=raw[:, 2].view(np.uint32).copy())
 
