@@ -94,6 +94,7 @@ enum { DCD_F32 = 0, DCD_BF16 = 1 };
 #define DCD_DEVERR_NONFINITE 0x4u   /* NaN / +inf reached a row's max or normaliser */
 #define DCD_DEVERR_TIMEOUT 0x8u     /* a bounded wait on an asynchronous copy expired */
 #define DCD_DEVERR_BAD_PARAM 0x10u  /* alpha < 0, beta outside [0, 1], T < 0 or non-finite */
+#define DCD_DEVERR_UNSUPPORTED 0x20u /* fused LM-head call: a node has more than 8 children */
 
 /* Largest tree (nodes per sequence, root included) the library accepts. */
 #define DCD_MAX_NODES 1024
@@ -169,7 +170,7 @@ int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_p
 
 /*
  * Capacity of the scratch array inside the library used by dcd_verify_sample_noalloc:
- * enough for dcd_workspace_bytes(shape) <= 4 MiB, e.g. B * N up to about 6900 rows at
+ * enough for dcd_workspace_bytes(shape) <= 4 MiB, e.g. B * N up to about 11,700 rows at
  * V = 128256 with bf16 logits.
  */
 #define DCD_STATIC_SCRATCH_BYTES (4u * 1024u * 1024u)
@@ -210,6 +211,38 @@ int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_a
                       const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
                       int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
                       dcd_stream_t stream, int stages, int plain_loads);
+
+/*
+ * Greedy CD verification fused with the two models' output projections (LM heads): the
+ * logits z_p = h_exp W_exp^T and z_q = h_ama W_ama^T of Eq. 1 are computed on the tensor
+ * cores tile by tile and reduced in place, never written to memory.  The target is Eq. 1
+ * with beta = 0 (the untruncated target, Sec. 2.1) and the greedy rule (the T -> 0 limit of
+ * Algorithm 1), exactly as dcd_verify_greedy with beta = NULL on the logits
+ * h W^T computed with fp32 accumulation of the bf16 products.
+ *   shape : B, N, V as for dcd_verify_greedy; logits_dtype must be DCD_BF16 (the type of
+ *       h and W); ld_logits and ld_q are not used.
+ *   h_exp : bf16 [B*N, H_exp] row-major, the expert's final hidden state after each node
+ *       (row g = b*N + n, the same row convention as the logits).
+ *   w_exp : bf16 [V, H_exp] row-major, the expert's output embedding (the layout of an
+ *       nn.Linear weight: row v produces logit v).
+ *   h_ama, w_ama : the amateur's, [B*N, H_ama] and [V, H_ama].
+ *   H_exp, H_ama : hidden sizes, >= 1 and multiples of 8 (16-byte rows); every matrix base
+ *       16-byte aligned.
+ *   tokens, parents, alpha, accept_len, accept_path, bonus, cd_logprob, cd_argmax,
+ *       cd_lse : as for dcd_verify_greedy (beta is 0).  A node may have at most 8 children
+ *       (else its sequence reports DCD_DEVERR_UNSUPPORTED and accept_len = 0).
+ *   workspace : device scratch of at least dcd_fused_workspace_bytes(shape), 256-byte
+ *       aligned; about 16 * B * N * ceil(V / 256) bytes.
+ * Returns DCD_ERR_UNSUPPORTED if the driver cannot describe the matrices to the tensor
+ * memory accelerator.  Errors found on the device are read with dcd_get_device_error.
+ */
+size_t dcd_fused_workspace_bytes(const dcd_shape* shape);
+
+int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H_exp, const void* w_exp,
+                            const void* h_ama, int32_t H_ama, const void* w_ama, const int32_t* tokens,
+                            const int32_t* parents, const float* alpha, int32_t* accept_len,
+                            int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
+                            float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream);
 
 /*
  * Synchronises `stream`, then copies the device error word of `workspace` (the OR of

@@ -249,3 +249,33 @@ def margin_fn(zp_row, za_row, alpha: float, beta: float) -> float:
         m = lp.max()
         gap = min(gap, float(np.min(np.abs(lp - m - np.log(beta)))))
     return gap
+
+
+def fused_logits(h, w, chunk: int = 8192) -> np.ndarray:
+    """z = h w^T in fp64 from the exact bf16 values (the fused LM-head variant's logits), h
+    [rows, H] and w [V, H]: a library matrix product, taken over blocks of `chunk` vocabulary
+    rows to bound host memory."""
+    import torch
+    hh = (h.detach().cpu() if isinstance(h, torch.Tensor) else torch.as_tensor(h)).to(torch.float64).numpy()
+    V = w.shape[0]
+    out = np.empty((hh.shape[0], V), dtype=np.float64)
+    for v0 in range(0, V, chunk):
+        v1 = min(V, v0 + chunk)
+        wb = w[v0:v1]
+        wb = (wb.detach().cpu() if isinstance(wb, torch.Tensor) else torch.as_tensor(wb)).to(torch.float64).numpy()
+        out[:, v0:v1] = hh @ wb.T
+    return out
+
+
+def verify_fused_workload(w, nthreads: int = 1, seqs=None) -> dict:
+    """``verify`` of a fused LM-head workload: logits from ``fused_logits`` (fp64), greedy, beta = 0."""
+    B, N = w.B, w.N
+    sel = list(range(B)) if seqs is None else list(seqs)
+    rows = np.concatenate([np.arange(b * N, (b + 1) * N) for b in sel])
+    import torch
+    ridx = torch.as_tensor(rows, device=w.h_exp.device)
+    zp = fused_logits(w.h_exp[ridx], w.w_exp)
+    zq = fused_logits(w.h_ama[ridx], w.w_ama)
+    return verify(B=len(sel), N=N, V=w.V, dtype="f64", z_exp=zp, z_ama=zq,
+                  tokens=w.tokens.cpu()[sel], parents=w.parents.cpu()[sel], alpha=w.alpha.cpu()[sel],
+                  beta=None, temperature=None, nthreads=nthreads, seq_ids=np.asarray(sel))

@@ -186,6 +186,54 @@ int dcd_verify_sample(const dcd_shape* shape, const void* z_exp, const void* z_a
                                                    reinterpret_cast<cudaStream_t>(stream)));
 }
 
+size_t dcd_fused_workspace_bytes(const dcd_shape* s) {
+  if (!s || s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || s->reserved != 0) return 0;
+  if (s->logits_dtype != DCD_BF16) return 0;
+  if (static_cast<int64_t>(s->B) * s->N > INT_MAX / 16) return 0;
+  return dcd::fused_layout(static_cast<int64_t>(s->B) * s->N, s->V).total;
+}
+
+int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H_exp, const void* w_exp,
+                            const void* h_ama, int32_t H_ama, const void* w_ama, const int32_t* tokens,
+                            const int32_t* parents, const float* alpha, int32_t* accept_len,
+                            int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
+                            float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
+  const size_t need = dcd_fused_workspace_bytes(shape);
+  if (need == 0) return DCD_ERR_INVALID_ARG;
+  if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
+  if (shape->B == 0) return DCD_OK;
+  auto al16 = [](const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+  if (!al16(h_exp) || !al16(w_exp) || !al16(h_ama) || !al16(w_ama)) return DCD_ERR_INVALID_ARG;
+  if (H_exp < 1 || H_ama < 1 || H_exp % 8 != 0 || H_ama % 8 != 0) return DCD_ERR_INVALID_ARG;
+  if (!tokens || !parents || !alpha || !accept_len || !accept_path || !bonus) return DCD_ERR_INVALID_ARG;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 || workspace_bytes < need)
+    return DCD_ERR_WORKSPACE;
+  dcd::FusedArgs f;
+  f.B = shape->B;
+  f.N = shape->N;
+  f.V = shape->V;
+  f.H_exp = H_exp;
+  f.H_ama = H_ama;
+  f.h_exp = h_exp;
+  f.w_exp = w_exp;
+  f.h_ama = h_ama;
+  f.w_ama = w_ama;
+  f.tokens = tokens;
+  f.parents = parents;
+  f.alpha = alpha;
+  f.accept_len = accept_len;
+  f.accept_path = accept_path;
+  f.bonus = bonus;
+  f.cd_logprob = cd_logprob;
+  f.cd_argmax = cd_argmax;
+  f.cd_lse = cd_lse;
+  f.workspace = workspace;
+  int status = DCD_OK;
+  const cudaError_t e = dcd::launch_fused(f, stream, &status);
+  if (status != DCD_OK) return status;
+  return cuda_status(e);
+}
+
 int dcd_get_device_error(const void* workspace, dcd_stream_t stream, uint32_t* bits) {
   if (!workspace || !bits) return DCD_ERR_INVALID_ARG;
   uint32_t host = 0;

@@ -67,12 +67,15 @@ def load(build_if_missing: bool = True):
         lib.dcd_score_rows_ex.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P,
                                           ctypes.c_int, ctypes.c_int]
         lib.dcd_tree_walk.argtypes = [SH, P, P, P, P, SZ, P]
+        lib.dcd_fused_workspace_bytes.argtypes = [SH]
+        lib.dcd_fused_workspace_bytes.restype = SZ
+        lib.dcd_verify_fused_lmhead.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
         lib.dcd_get_device_error.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
         lib.dcd_status_string.argtypes = [ctypes.c_int]
         lib.dcd_status_string.restype = ctypes.c_char_p
         lib.dcd_version.restype = ctypes.c_int
         for name in ("dcd_verify_greedy", "dcd_verify_sample", "dcd_score_rows", "dcd_score_rows_ex",
-                     "dcd_tree_walk", "dcd_get_device_error"):
+                     "dcd_tree_walk", "dcd_get_device_error", "dcd_verify_fused_lmhead"):
             getattr(lib, name).restype = I32
         _lib = lib
         return lib
@@ -281,6 +284,49 @@ def dcd_tree_walk(B: int, N: int, V: int, out: dict, workspace, stream=None) -> 
                               _ptr(out["bonus"]), _ptr(workspace), workspace.numel(), _stream(stream))
     _check(st, "dcd_tree_walk")
     return out
+
+
+def fused_workspace_bytes(B: int, N: int, V: int) -> int:
+    sh = make_shape(B, N, V, DCD_BF16)
+    n = load().dcd_fused_workspace_bytes(ctypes.byref(sh))
+    if n == 0:
+        raise ValueError("invalid shape")
+    return int(n)
+
+
+def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, *, out=None, workspace=None,
+                            stream=None) -> dict:
+    """Greedy CD verification fused with the two LM heads (logits h W^T never materialised).
+
+    h_exp [B*N, H_exp], w_exp [V, H_exp], h_ama [B*N, H_ama], w_ama [V, H_ama]: bf16, row-major.
+    Returns accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse (and the workspace).
+    """
+    for t, name in ((h_exp, "h_exp"), (w_exp, "w_exp"), (h_ama, "h_ama"), (w_ama, "w_ama")):
+        _require(t, name, dtype=torch.bfloat16)
+        if t.dim() != 2 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous 2-D tensor")
+    dev = h_exp.device
+    B, N = tokens.shape
+    R, H_exp = h_exp.shape
+    V = w_exp.shape[0]
+    H_ama = h_ama.shape[1]
+    if R != B * N or h_ama.shape[0] != R or tuple(w_exp.shape) != (V, H_exp) or tuple(w_ama.shape) != (V, H_ama):
+        raise ValueError("inconsistent shapes for the fused LM-head call")
+    _require(tokens, "tokens", torch.int32, dev)
+    _require(parents, "parents", torch.int32, dev, (B, N))
+    _require(alpha, "alpha", torch.float32, dev, (B,))
+    sh = make_shape(B, N, V, DCD_BF16)
+    if workspace is None:
+        workspace = torch.empty(fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
+    o = alloc_outputs(B, N, dev) if out is None else out
+    st = load().dcd_verify_fused_lmhead(
+        ctypes.byref(sh), _ptr(h_exp), H_exp, _ptr(w_exp), _ptr(h_ama), H_ama, _ptr(w_ama), _ptr(tokens),
+        _ptr(parents), _ptr(alpha), _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]),
+        _ptr(o.get("cd_logprob")), _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(workspace),
+        workspace.numel(), _stream(stream))
+    _check(st, "dcd_verify_fused_lmhead")
+    o["workspace"] = workspace
+    return o
 
 
 def dcd_get_device_error(workspace: torch.Tensor, stream=None) -> int:

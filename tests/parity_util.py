@@ -68,6 +68,24 @@ def run_gpu(w, *, sampled: bool, residual: bool = False, stages: int = 0, plain:
     return res
 
 
+def fused_records(ws: torch.Tensor, R: int):
+    """Per-row records of the fused LM-head step (after the 256-byte header, 3 x R x 8 child
+    entries of 4 bytes and R 4-byte row statuses padded to 16 bytes)."""
+    off = 256 + 96 * R + (4 * R + 15) // 16 * 16
+    raw = ws[off:off + 16 * R].cpu().numpy().view(np.int32).reshape(R, 4)
+    return dict(acc_child=raw[:, 0].copy(), term_token=raw[:, 1].copy(), status=raw[:, 2].view(np.uint32).copy())
+
+
+def run_fused_gpu(w) -> dict:
+    """The fused LM-head call on workload `w`, results on the host in the layout `compare` takes."""
+    o = dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha)
+    torch.cuda.synchronize()
+    res = {k: v.cpu().numpy() for k, v in o.items() if k != "workspace"}
+    res["records"] = fused_records(o["workspace"], w.B * w.N)
+    res["error_bits"] = dcd.dcd_get_device_error(o["workspace"])
+    return res
+
+
 def compare(w, gpu: dict, ref: dict, seqs=None, check_residual: bool = False, max_amb_frac: float = 0.05):
     """Asserts parity of GPU outputs (all sequences of `w`, or the subset `seqs`) with the oracle's."""
     B, N = w.B, w.N

@@ -116,3 +116,26 @@ def test_binding_refuses_cpu_tensors():
     t = torch.zeros((1, 6), dtype=torch.int32)
     with pytest.raises(ValueError, match="CUDA"):
         dcd.dcd_verify_greedy(z, z, t, t, torch.zeros(1))
+
+
+def test_fused_workspace_and_host_checks(lib):
+    sh = dcd.make_shape(64, 60, 128256, dcd.DCD_BF16)
+    n = lib.dcd_fused_workspace_bytes(ctypes.byref(sh))
+    nvt = (128256 + 255) // 256
+    assert n >= 256 + 3840 * (96 + 16) + 3840 * nvt * 16 and n % 256 == 0
+    f32 = dcd.make_shape(2, 4, 100, dcd.DCD_F32)
+    assert lib.dcd_fused_workspace_bytes(ctypes.byref(f32)) == 0
+    P = _fake(0x10000)
+    sh = dcd.make_shape(2, 4, 100, dcd.DCD_BF16)
+    ws = _fake(0x100000)
+    args = [P, 64, P, P, 64, P, P, P, P, P, P, P, None, None, None]
+    # hidden size not a multiple of 8, misaligned matrix, small workspace: rejected before launch
+    bad = list(args)
+    bad[1] = 60
+    assert lib.dcd_verify_fused_lmhead(ctypes.byref(sh), *bad, ws, 1 << 24, None) == -1
+    bad = list(args)
+    bad[0] = _fake(0x10008)
+    assert lib.dcd_verify_fused_lmhead(ctypes.byref(sh), *bad, ws, 1 << 24, None) == -1
+    assert lib.dcd_verify_fused_lmhead(ctypes.byref(sh), *args, ws, 64, None) == -7
+    empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
+    assert lib.dcd_verify_fused_lmhead(ctypes.byref(empty), *args, ws, 1 << 24, None) == 0

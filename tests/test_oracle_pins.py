@@ -499,3 +499,21 @@ def test_residual_chain_closed_form():
             D = np.maximum(0.0, pi - c * qd).sum()
         np.testing.assert_allclose(closed, ratios, rtol=1e-12, atol=1e-15)
         np.testing.assert_allclose(np.maximum(0.0, pi - c * qd) / D, rm, rtol=0, atol=1e-14)
+
+
+def test_fused_logits_are_h_times_w_transposed():
+    """The fused variant's logits z[r, v] = sum_k h[r, k] w[v, k] (w in the nn.Linear layout
+    [V, H]), checked element by element against the sum written out, in blocks of the vocabulary
+    smaller than V so that the blocking is exercised."""
+    import torch
+    g = torch.Generator().manual_seed(5)
+    h = torch.randn((3, 11), generator=g).to(torch.bfloat16)
+    w = (torch.randn((13, 11), generator=g) * 0.5).to(torch.bfloat16)
+    z = oracle.fused_logits(h, w, chunk=4)
+    hd, wd = h.double().numpy(), w.double().numpy()
+    for r in range(3):
+        for v in range(13):
+            s = 0.0
+            for k in range(11):
+                s += hd[r, k] * wd[v, k]
+            assert abs(z[r, v] - s) < 1e-12
