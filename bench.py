@@ -6,10 +6,16 @@ walk, through the C ABI (dcd_score_rows + dcd_tree_walk, i.e. dcd_verify_sample
 without the test-only residual output), on the batched-serving workload:
 32 sequences x 60-node trees of depth 7 (1920 rows), V = 128256, bf16 logits,
 alpha in {0.05, 0.1, 0.2}, even sequences greedy and odd ones sampled at T = 1.
-Inputs are seeded synthetic data resident in HBM (1.48 GB per step, larger than
-the 126 MB L2, so no flush is needed); each step advances the Philox offset.
+Inputs are seeded synthetic data resident in HBM (1.97 GB, larger than the 129 MB
+L2, so no flush is needed; about 1.05 GB of it is read per step); each step advances
+the Philox offset.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+`--workload fused` times the fused LM-head variant instead (dcd_verify_fused_lmhead:
+64 sequences x 60 nodes = 3840 rows, hidden states of 8192 and 2048, V = 128256,
+bf16, greedy): one step is both output projections on the tensor cores with the CD
+epilogue, the per-row combine and the tree walk.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload batched|fused]
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle on a
 bounded sample of the same workload instead.
@@ -33,6 +39,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOAD = "batched_B32_tree60_V128256_bf16_mixed"
+FUSED_WORKLOAD = "fused_lmhead_B64_tree60_V128256_Hexp8192_Hama2048_bf16_greedy"
 METRIC = "verified draft nodes/sec (CD verification step, 1 GPU)"
 
 
@@ -43,6 +50,16 @@ def _peaks():
         return float(p["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def _bf16_peak():
+    """Sustained dense bf16 TFLOP/s (the fused kernel runs back to back for seconds)."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops_sustained"]), "measured bf16_tflops_sustained"
+    except Exception:
+        return 1700.0, "fallback sustained bf16"
 
 
 def _kernel_source_hash() -> str:
@@ -354,6 +371,142 @@ def run_ours(args):
     return 0
 
 
+def run_fused(args):
+    """The fused LM-head variant: tensor-core bound; roofline in TFLOP/s of the GEMM kernel."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_12913_gb300 import dcd, workloads
+
+    world, rank, local = _dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = workloads.make_fused_torch(device=dev, seed=4 + rank)
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    H_exp, H_ama = w.h_exp.shape[1], w.h_ama.shape[1]
+    flop = 2.0 * R * V * (H_exp + H_ama)
+    out = dcd.alloc_outputs(B, N, dev)
+    ws = torch.empty(dcd.fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    steps = args.steps
+
+    def step(evs=None):
+        dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha, out=out,
+                                    workspace=ws, stream=stream, gemm_events=evs)
+
+    for _ in range(args.warmup):
+        step()
+    if dcd.dcd_get_device_error(ws) != 0:
+        raise RuntimeError("device error bits set during warm-up")
+    sampler = ClockSampler(local)
+    sampler.start()
+    t_soak = time.time()
+    while not args.no_soak and time.time() - t_soak < 1.0:
+        step()
+        torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for e in evs:  # create the events outside the timed region
+        e[0].record(stream)
+        e[1].record(stream)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    start.record(stream)
+    for k in range(steps):
+        step(evs[k])
+    stop.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t_wall1 = time.time()
+    sampler.stop()
+    elapsed_ms = start.elapsed_time(stop)
+    gemm_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    if dcd.dcd_get_device_error(ws) != 0:
+        raise RuntimeError("device error bits set during the timed region")
+    ms_per_step = elapsed_ms / steps
+    value = world * R / (ms_per_step / 1e3)
+    peak, peak_src = _bf16_peak()
+    achieved = flop / (gemm_ms / 1e3) / 1e12
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": None, "kernel": "fused_lmhead_kernel", "peak_source": peak_src,
+                "algorithmic_flops_per_launch": flop, "gemm_kernel_ms": gemm_ms}
+
+    # end to end: the step's hidden states and tree come from pinned host memory (the weights
+    # are the models' resident parameters), the results go back
+    e2e = None
+    if not args.no_e2e:
+        host = {k: getattr(w, k).cpu().pin_memory() for k in ("h_exp", "h_ama", "tokens", "parents", "alpha")}
+        dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
+        res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory() for k in ("accept_len", "accept_path",
+                                                                                     "bonus")}
+        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+        n_e2e = max(3, min(steps, 10))
+
+        def e2e_step():
+            for k in host:
+                dst[k].copy_(host[k], non_blocking=True)
+            o = dcd.dcd_verify_fused_lmhead(dst["h_exp"], w.w_exp, dst["h_ama"], w.w_ama, dst["tokens"],
+                                            dst["parents"], dst["alpha"], out=out, workspace=ws, stream=stream)
+            for k in res_host:
+                res_host[k].copy_(o[k], non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        a, b2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        b2.record(stream)
+        torch.cuda.synchronize()
+        e_ms = a.elapsed_time(b2) / n_e2e
+        if world > 1:
+            t = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e_ms = float(t.item())
+        e2e = {"value": world * R / (e_ms / 1e3), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": FUSED_WORKLOAD, "B": B, "N": N, "V": V, "rows": R, "H_exp": H_exp,
+                       "H_ama": H_ama, "flop_per_step": flop,
+                       "l2": "weights (2.6 GB) larger than L2; no flush",
+                       "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
+            "roofline": roofline,
+            "clocks": sampler.summary(t_wall0, t_wall1),
+            "e2e": e2e,
+            "gpu_launches": 4 * steps,
+        }
+        if not args.no_cpu_baseline:
+            import oracle
+            threads = oracle.max_threads()
+            t0 = time.perf_counter()
+            oracle.verify_fused_workload(w, nthreads=threads, seqs=[0])
+            dt = time.perf_counter() - t0
+            line["cpu_baseline"] = {"value": N / dt, "unit": "nodes/s", "cores": threads, "kind": "oracle",
+                                    "sample": f"sequence 0 of {B} ({N} rows: fp64 logits and the row oracle), "
+                                              f"{dt:.1f} s wall"}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -366,11 +519,16 @@ def main():
     ap.add_argument("--greedy", action="store_true", help="every sequence greedy (profiling case)")
     ap.add_argument("--batch", type=int, default=32,
                     help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
+    ap.add_argument("--workload", choices=("batched", "fused"), default="batched",
+                    help="batched: the streaming step on materialised logits (the headline); fused: the "
+                         "fused LM-head variant")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "fused":
+        return run_fused(args)
     return run_ours(args)
 
 

@@ -245,6 +245,18 @@ int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H
                             float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream);
 
 /*
+ * dcd_verify_fused_lmhead that also records two CUDA events (cudaEvent_t handles, or NULL)
+ * on `stream` immediately before and after the tensor-core kernel, for timing that kernel
+ * alone.  Results equal dcd_verify_fused_lmhead.
+ */
+int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_t H_exp, const void* w_exp,
+                               const void* h_ama, int32_t H_ama, const void* w_ama, const int32_t* tokens,
+                               const int32_t* parents, const float* alpha, int32_t* accept_len,
+                               int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
+                               float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
+                               void* gemm_start, void* gemm_stop);
+
+/*
  * Synchronises `stream`, then copies the device error word of `workspace` (the OR of
  * the DCD_DEVERR_* bits raised by the last call that used it) into *bits.  Returns
  * DCD_OK when the word is zero, DCD_ERR_DEVICE_INPUT when it is not, DCD_ERR_CUDA if

@@ -198,6 +198,17 @@ int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H
                             const int32_t* parents, const float* alpha, int32_t* accept_len,
                             int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
                             float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
+  return dcd_verify_fused_lmhead_ex(shape, h_exp, H_exp, w_exp, h_ama, H_ama, w_ama, tokens, parents, alpha,
+                                    accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse, workspace,
+                                    workspace_bytes, stream, nullptr, nullptr);
+}
+
+int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_t H_exp, const void* w_exp,
+                               const void* h_ama, int32_t H_ama, const void* w_ama, const int32_t* tokens,
+                               const int32_t* parents, const float* alpha, int32_t* accept_len,
+                               int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
+                               float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
+                               void* gemm_start, void* gemm_stop) {
   const size_t need = dcd_fused_workspace_bytes(shape);
   if (need == 0) return DCD_ERR_INVALID_ARG;
   if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
@@ -228,6 +239,8 @@ int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H
   f.cd_argmax = cd_argmax;
   f.cd_lse = cd_lse;
   f.workspace = workspace;
+  f.gemm_start = static_cast<cudaEvent_t>(gemm_start);
+  f.gemm_stop = static_cast<cudaEvent_t>(gemm_stop);
   int status = DCD_OK;
   const cudaError_t e = dcd::launch_fused(f, stream, &status);
   if (status != DCD_OK) return status;

@@ -240,7 +240,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty);
-      if (valid) P.part[static_cast<int64_t>(r) * P.nvt + j] = make_float4(m, ssum, __int_as_float(arg), 0.f);
+      // streaming store: read once by the combine kernel, it should not displace h in L2
+      if (valid) __stcs(&P.part[static_cast<int64_t>(r) * P.nvt + j], make_float4(m, ssum, __int_as_float(arg), 0.f));
     }
   }
 
@@ -455,9 +456,17 @@ cudaError_t launch_fused(const FusedArgs& f, cudaStream_t stream, int* status) {
   int grid = sm_count();
   if (grid <= 0) return cudaErrorInvalidDevice;
   if (grid > P.ntiles) grid = P.ntiles;
+  if (f.gemm_start) {
+    e = cudaEventRecord(f.gemm_start, stream);
+    if (e != cudaSuccess) return e;
+  }
   fused_lmhead_kernel<<<grid, kGemmThreads, kGemmSmem, stream>>>(P);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (f.gemm_stop) {
+    e = cudaEventRecord(f.gemm_stop, stream);
+    if (e != cudaSuccess) return e;
+  }
 
   CombineArgs C;
   C.B = f.B;

@@ -138,6 +138,7 @@ struct FusedArgs {
   int32_t* cd_argmax;
   float* cd_lse;
   void* workspace;
+  cudaEvent_t gemm_start, gemm_stop;  // optional: recorded around the GEMM launch (timing)
 };
 
 // Workspace of the fused step: [WsHeader][child nodes][child tokens][child scores][row status]

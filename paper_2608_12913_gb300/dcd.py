@@ -70,12 +70,15 @@ def load(build_if_missing: bool = True):
         lib.dcd_fused_workspace_bytes.argtypes = [SH]
         lib.dcd_fused_workspace_bytes.restype = SZ
         lib.dcd_verify_fused_lmhead.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
+        lib.dcd_verify_fused_lmhead_ex.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P,
+                                                   P, P]
         lib.dcd_get_device_error.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
         lib.dcd_status_string.argtypes = [ctypes.c_int]
         lib.dcd_status_string.restype = ctypes.c_char_p
         lib.dcd_version.restype = ctypes.c_int
         for name in ("dcd_verify_greedy", "dcd_verify_sample", "dcd_score_rows", "dcd_score_rows_ex",
-                     "dcd_tree_walk", "dcd_get_device_error", "dcd_verify_fused_lmhead"):
+                     "dcd_tree_walk", "dcd_get_device_error", "dcd_verify_fused_lmhead",
+                     "dcd_verify_fused_lmhead_ex"):
             getattr(lib, name).restype = I32
         _lib = lib
         return lib
@@ -295,11 +298,12 @@ def fused_workspace_bytes(B: int, N: int, V: int) -> int:
 
 
 def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, *, out=None, workspace=None,
-                            stream=None) -> dict:
+                            stream=None, gemm_events=None) -> dict:
     """Greedy CD verification fused with the two LM heads (logits h W^T never materialised).
 
     h_exp [B*N, H_exp], w_exp [V, H_exp], h_ama [B*N, H_ama], w_ama [V, H_ama]: bf16, row-major.
     Returns accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse (and the workspace).
+    `gemm_events` = (start, stop) torch.cuda.Event pair recorded around the tensor-core kernel.
     """
     for t, name in ((h_exp, "h_exp"), (w_exp, "w_exp"), (h_ama, "h_ama"), (w_ama, "w_ama")):
         _require(t, name, dtype=torch.bfloat16)
@@ -319,11 +323,17 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
     if workspace is None:
         workspace = torch.empty(fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
     o = alloc_outputs(B, N, dev) if out is None else out
-    st = load().dcd_verify_fused_lmhead(
+    ev0 = ev1 = None
+    if gemm_events is not None:
+        for e in gemm_events:
+            if not e.cuda_event:  # torch creates the event at its first record
+                e.record()
+        ev0, ev1 = (ctypes.c_void_p(e.cuda_event) for e in gemm_events)
+    st = load().dcd_verify_fused_lmhead_ex(
         ctypes.byref(sh), _ptr(h_exp), H_exp, _ptr(w_exp), _ptr(h_ama), H_ama, _ptr(w_ama), _ptr(tokens),
         _ptr(parents), _ptr(alpha), _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]),
         _ptr(o.get("cd_logprob")), _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(workspace),
-        workspace.numel(), _stream(stream))
+        workspace.numel(), _stream(stream), ev0, ev1)
     _check(st, "dcd_verify_fused_lmhead")
     o["workspace"] = workspace
     return o
