@@ -39,7 +39,7 @@
 //  A node without an accepted child draws its terminal token by a two-level exponential
 //  race: a 1024-token block by its mass, then a token of that block (four tokens a thread,
 //  re-read directly).
-// tree_walk_kernel: one thread per sequence follows the accepted children.
+// tree_walk_kernel: one warp per sequence follows the accepted children.
 // terminal_residual_kernel: one block per sequence rebuilds the distribution its bonus
 //   token was drawn from (test output only).
 
@@ -1109,32 +1109,59 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
 }
 
 // ------------------------------------------------------------------------------------------
-__global__ void tree_walk_kernel(int32_t B, int32_t N, const RowRecord* __restrict__ rec, uint32_t* err,
-                                 int32_t* accept_len, int32_t* accept_path, int32_t* bonus) {
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+// One warp per sequence: the N records are read at once into shared memory, then lane 0 follows
+// the accepted children from the root and the warp writes the path.  Launched as a programmatic
+// dependent of the row kernel: it waits for that grid's completion (and its memory) first.
+constexpr int kWalkWarps = 4;
+
+__global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(int32_t B, int32_t N,
+                                                                    const RowRecord* __restrict__ rec, uint32_t* err,
+                                                                    int32_t* accept_len, int32_t* accept_path,
+                                                                    int32_t* bonus) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  extern __shared__ int walk_smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * kWalkWarps + warp;
   if (b >= B) return;
+  int* wacc = walk_smem + warp * 3 * N;
+  int* wterm = wacc + N;
+  int* wpath = wterm + N;
   const RowRecord* r = rec + static_cast<int64_t>(b) * N;
-  int32_t* path = accept_path + static_cast<int64_t>(b) * N;
   uint32_t st = 0u;
-  for (int i = 0; i < N; ++i) st |= r[i].status;
-  int cur = 0, len = 0;
-  path[0] = 0;
+  for (int i = lane; i < N; i += 32) {
+    const RowRecord v = r[i];
+    wacc[i] = v.acc_child;
+    wterm[i] = v.term_token;
+    st |= v.status;
+  }
+  st = __reduce_or_sync(~0u, st);
+  __syncwarp();
+  int32_t* path = accept_path + static_cast<int64_t>(b) * N;
   if (st) {
-    atomicOr(err, st);
-    for (int i = 1; i < N; ++i) path[i] = -1;
-    accept_len[b] = 0;
-    bonus[b] = -1;
+    if (lane == 0) {
+      atomicOr(err, st);
+      accept_len[b] = 0;
+      bonus[b] = -1;
+    }
+    for (int i = lane; i < N; i += 32) path[i] = i == 0 ? 0 : -1;
     return;
   }
-  while (len < N - 1) {
-    const int a = r[cur].acc_child;
-    if (a <= cur || a >= N) break;
-    cur = a;
-    path[++len] = cur;
+  int len = 0;
+  if (lane == 0) {
+    int cur = 0;
+    wpath[0] = 0;
+    while (len < N - 1) {
+      const int a = wacc[cur];
+      if (a <= cur || a >= N) break;
+      cur = a;
+      wpath[++len] = cur;
+    }
+    accept_len[b] = len;
+    bonus[b] = wterm[cur];
   }
-  for (int i = len + 1; i < N; ++i) path[i] = -1;
-  accept_len[b] = len;
-  bonus[b] = r[cur].term_token;
+  len = __shfl_sync(~0u, len, 0);
+  __syncwarp();
+  for (int i = lane; i < N; i += 32) path[i] = i <= len ? wpath[i] : -1;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -1369,10 +1396,19 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
 cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_t* err, int32_t* accept_len,
                              int32_t* accept_path, int32_t* bonus, cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
-  const int threads = 128;
-  tree_walk_kernel<<<(B + threads - 1) / threads, threads, 0, stream>>>(B, N, rec, err, accept_len, accept_path,
-                                                                        bonus);
-  return cudaGetLastError();
+  const size_t smem = static_cast<size_t>(kWalkWarps) * 3 * N * sizeof(int);  // <= 48 KB for N <= 1024
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>((B + kWalkWarps - 1) / kWalkWarps));
+  cfg.blockDim = dim3(kWalkWarps * 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  // launched while the previous kernel in the stream finishes; the kernel waits for it first
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tree_walk_kernel, B, N, rec, err, accept_len, accept_path, bonus);
 }
 
 cudaError_t launch_terminal_residual(const ScoreArgs& a, const int32_t* accept_len, const int32_t* accept_path,
