@@ -163,6 +163,20 @@ def residual_rows_per_step(w, out, ws, stream, offsets) -> float:
     return float(torch.stack(counts).double().mean().item())
 
 
+def max_over_ranks(ms: float, dist, device) -> float:
+    """The slowest rank's time: every rank of the job calls it (a MAX all-reduce)."""
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world: int, units_per_rank: int, ms_per_step: float) -> float:
+    """Whole-job throughput: every rank processes its own batch (weak scaling), so the job's
+    units per step are world x units_per_rank, over the slowest rank's step time."""
+    return world * units_per_rank / (ms_per_step / 1e3)
+
+
 def _dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -286,13 +300,11 @@ def run_ours(args):
     elapsed_ms = start.elapsed_time(stop)
     row_ms = [a.elapsed_time(b) for a, b in evs]
     if world > 1:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+        elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
     if dcd.dcd_get_device_error(ws) != 0:
         raise RuntimeError("device error bits set during the timed region")
     ms_per_step = elapsed_ms / args.steps
-    value = world * R / (ms_per_step / 1e3)
+    value = job_value(world, R, ms_per_step)
 
     # roofline of the dominant kernel (the row kernel) from its own events; the rows that took
     # residual passes are counted on a replay of every 32nd timed offset
@@ -341,10 +353,8 @@ def run_ours(args):
         torch.cuda.synchronize()
         e_ms = a.elapsed_time(b2) / n_e2e
         if world > 1:
-            t = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e_ms = float(t.item())
-        e2e = {"value": world * R / (e_ms / 1e3), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
+            e_ms = max_over_ranks(e_ms, dist, dev)
+        e2e = {"value": job_value(world, R, e_ms), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
         del dst, host
 
@@ -428,13 +438,11 @@ def run_fused(args):
     elapsed_ms = start.elapsed_time(stop)
     gemm_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
     if world > 1:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+        elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
     if dcd.dcd_get_device_error(ws) != 0:
         raise RuntimeError("device error bits set during the timed region")
     ms_per_step = elapsed_ms / steps
-    value = world * R / (ms_per_step / 1e3)
+    value = job_value(world, R, ms_per_step)
     peak, peak_src = _bf16_peak()
     achieved = flop / (gemm_ms / 1e3) / 1e12
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
@@ -471,10 +479,8 @@ def run_fused(args):
         torch.cuda.synchronize()
         e_ms = a.elapsed_time(b2) / n_e2e
         if world > 1:
-            t = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e_ms = float(t.item())
-        e2e = {"value": world * R / (e_ms / 1e3), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
+            e_ms = max_over_ranks(e_ms, dist, dev)
+        e2e = {"value": job_value(world, R, e_ms), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
 
     if rank == 0:

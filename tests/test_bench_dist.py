@@ -1,0 +1,64 @@
+"""The multi-process (replicas) logic of bench.py, on CPU: world-size-2 `gloo` ranks take the
+slowest rank's time, the job value counts every rank's batch, and a non-zero rank of the
+reference arm exits without output."""
+
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        ms = 1.5 + rank  # rank 1 is the slower one
+        worst = bench.max_over_ranks(ms, dist, "cpu")
+        dist.barrier()
+        q.put((rank, worst, bench.job_value(world, 1920, worst)))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_take_the_slowest_time_and_count_both_batches():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    got = sorted(q.get(timeout=10) for _ in range(2))
+    for rank, worst, value in got:
+        assert worst == pytest.approx(2.5)
+        assert value == pytest.approx(2 * 1920 / 2.5e-3)
+
+
+def test_job_value_is_weak_scaling():
+    assert bench.job_value(1, 1920, 0.25) == pytest.approx(1920 / 0.25e-3)
+    assert bench.job_value(4, 1920, 0.25) == pytest.approx(4 * bench.job_value(1, 1920, 0.25))
+
+
+def test_reference_arm_nonzero_rank_exits_quietly():
+    env = dict(os.environ, RANK="1", LOCAL_RANK="1", WORLD_SIZE="2")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "3"], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0
+    assert r.stdout.strip() == ""

@@ -9,7 +9,7 @@ import torch
 
 import oracle
 from paper_2608_12913_gb300 import dcd, workloads
-from tests.parity_util import compare, run_fused_gpu
+from parity_util import compare, run_fused_gpu
 
 pytestmark = pytest.mark.gpu
 

@@ -234,3 +234,12 @@ def test_device_input_errors_are_reported_not_trapped():
     a[0] = -1.0
     o = dcd.dcd_verify_greedy(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, a, wd.beta)
     assert dcd.dcd_get_device_error(o["workspace"]) & 0x10
+
+
+def test_largest_tree_chain_of_max_nodes():
+    # N = 1024 (the largest tree the library accepts): a chain of depth 1023, greedy and sampled
+    for temp in (0.0, 1.0):
+        w = workloads.make_config(0, V=1000, chain_len=1024, B=1, temperatures=(temp,), dtype="f32", seed=21)
+        gpu = run_gpu(w, sampled=temp > 0)
+        ref = oracle.verify_workload(w, nthreads=oracle.max_threads())
+        compare(w, gpu, ref)
