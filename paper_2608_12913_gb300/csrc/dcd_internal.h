@@ -14,7 +14,10 @@ namespace dcd {
 // per part; a slot (SlotHead + one PiecePart per residual piece) holds the chain state of a row
 // whose first sibling was rejected.
 constexpr size_t kWorkspaceHeader = 256;
-constexpr int kMaxParts = 4;  // parts a row may be split into
+#ifndef DCD_MAX_PARTS
+#define DCD_MAX_PARTS 4
+#endif
+constexpr int kMaxParts = DCD_MAX_PARTS;  // parts a row may be split into
 
 inline size_t part_counter_bytes(size_t rows) { return (rows * 4 + 15) & ~static_cast<size_t>(15); }
 

@@ -65,7 +65,17 @@ using namespace dev;
 #endif
 constexpr int kStageBytes = DCD_STAGE_KIB * 1024;  // bytes per ring stage
 constexpr int kMaxStages = 8;
-constexpr int kPieceStages = 4;                    // ring stages per residual piece
+#ifndef DCD_PIECE_STAGES
+#define DCD_PIECE_STAGES 4
+#endif
+#ifndef DCD_PARTS_BELOW
+#define DCD_PARTS_BELOW 2
+#endif
+constexpr int kPieceStages = DCD_PIECE_STAGES;     // ring stages per residual piece
+// Rows are streamed in parts only when the batch has at most this many rows per resident CTA:
+// then whole rows would leave most CTAs idle for part of the step; with more rows than that,
+// dynamic claiming of whole rows balances better than parts (measured).
+constexpr int kPartsBelow = DCD_PARTS_BELOW;
 constexpr int kDesc = 4;                           // work descriptors in flight per CTA
 constexpr int kCtaThreads = kThreads + 32;         // eight consumer warps and one producer warp
 constexpr int kMinCtasPerSm = 3;
@@ -1368,13 +1378,13 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   if (per_sm > geo.ctas_per_sm) per_sm = geo.ctas_per_sm;
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
   const int64_t resident = static_cast<int64_t>(sms) * per_sm;
-  // The last rows (as many as CTAs, or all of a small batch) are streamed in parts of spp
-  // stages each, so the rows still in flight at the end of the step are spread over more CTAs.
+  // A small batch (at most kPartsBelow rows per resident CTA) is streamed in parts of spp stages
+  // each, so that its rows spread over more CTAs.
   const int nch_a = static_cast<int>((a.V + sp.tok_a - 1) / sp.tok_a);
   const int want = nch_a < kMaxParts ? nch_a : kMaxParts;
   sp.spp = (nch_a + want - 1) / want;
   sp.parts = (nch_a + sp.spp - 1) / sp.spp;
-  const int64_t tail = sp.parts > 1 ? (R < resident ? R : resident) : 0;
+  const int64_t tail = (sp.parts > 1 && R <= kPartsBelow * resident) ? R : 0;
   sp.r_whole = static_cast<int32_t>(R - tail);
   sp.items = static_cast<int32_t>(sp.r_whole + tail * sp.parts);
   int64_t grid = resident;
