@@ -103,6 +103,7 @@ struct SParams {
   int32_t parts;         // parts of such a row (stages of the stats pass split in runs of spp)
   int32_t spp;           // stats-pass stages per part
   int32_t items;         // row items: r_whole + (R - r_whole) * parts
+  int32_t keep_internal; // small batch: keep sampled internal rows and pieces in L2 (evict-last)
   WsHeader* hdr;         // counters, zeroed before the launch
   Job* jobs;             // residual passes (zeroed before the launch)
   unsigned char* slots;  // per handed-over row: SlotHead + npieces PieceParts
@@ -355,6 +356,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
   if (warp == kWarps) {
     // ===================================== producer warp
     const uint64_t pol_last = l2_policy_evict_last();
+    const uint64_t pol_normal = l2_policy_evict_normal();
     const uint64_t pol_first = l2_policy_evict_first();
     uint32_t issued = 0;  // ring items issued
 
@@ -481,8 +483,11 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           D.T = meta.T;
           const bool masked = D.beta > 0.f;
           const bool sampled = D.T > 0.f && p.q != nullptr;
-          // a sampled internal row keeps its logits in L2 for residual passes
-          pol = (sampled && meta.m > 0) ? pol_last : pol_first;
+          // In a small batch a sampled internal row keeps its logits in L2 for residual passes,
+          // which are then on the critical path.  In a large batch only about a quarter of those
+          // rows take a pass, and keeping them all crowds L2: every row is streamed evict-first
+          // (measured both ways).
+          pol = (sampled && meta.m > 0 && sp.keep_internal) ? pol_last : pol_first;
           if (meta.part >= 0 && !masked) {
             D.kind = kWorkPart;
             D.piece = meta.part;
@@ -517,7 +522,8 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           const int64_t rem = (V - x_lo + sp.tok_r - 1) / sp.tok_r;
           nitems = static_cast<int>(rem < kPieceStages ? rem : kPieceStages);
           with_q = true;
-          pol = D.J < D.m ? pol_last : pol_first;  // the pass after the last sibling is the last read
+          // a later pass re-reads the piece; the pass after the last sibling is the last read
+          pol = D.J < D.m ? (sp.keep_internal ? pol_last : pol_normal) : pol_first;
         }
       }
       // ---- publish the descriptor
@@ -1386,6 +1392,7 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.parts = (nch_a + sp.spp - 1) / sp.spp;
   const int64_t tail = (sp.parts > 1 && R <= kPartsBelow * resident) ? R : 0;
   sp.r_whole = static_cast<int32_t>(R - tail);
+  sp.keep_internal = R <= kPartsBelow * resident ? 1 : 0;
   sp.items = static_cast<int32_t>(sp.r_whole + tail * sp.parts);
   int64_t grid = resident;
   if (grid > sp.items) grid = sp.items;
