@@ -87,9 +87,10 @@ def _load():
             lib.dcd_oracle_block_uniform.argtypes = [U64, U64, ctypes.c_uint32, I64]
             lib.dcd_oracle_block_uniform.restype = D
             lib.dcd_oracle_row_logpi.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, P, P, P, P, P, P]
-            lib.dcd_oracle_row_chain.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, ctypes.c_int, P, P, P]
+            lib.dcd_oracle_row_chain.argtypes = [I64, ctypes.c_int, P, P, D, D, D, P, ctypes.c_int, P, ctypes.c_int,
+                                                 P, P]
             lib.dcd_oracle_verify.argtypes = [I32, I32, I64, ctypes.c_int, I64, P, P, P, P, P, P, P, P, I64,
-                                              U64, U64, P, ctypes.c_int, P, P, P, P, P, P]
+                                              U64, U64, P, ctypes.c_int, ctypes.c_int, P, P, P, P, P, P]
             lib.dcd_oracle_max_threads.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -165,8 +166,10 @@ def row_logpi(zp, zq, alpha: float, beta: float = 0.0, T: float = 1.0, dtype: st
     return res
 
 
-def row_chain(zp, zq, alpha: float, beta: float, T: float, q, child_tokens, dtype: str = "f64"):
-    """Sibling-rejection chain run to its end: (ratios[m], final residual r_m[V])."""
+def row_chain(zp, zq, alpha: float, beta: float, T: float, q, child_tokens, dtype: str = "f64",
+              distinct: bool = False):
+    """Sibling-rejection chain run to its end: (ratios[m], final residual r_m[V]).  `distinct`:
+    siblings drawn without replacement (each sees q without the earlier siblings' tokens)."""
     zp = _logits(zp, dtype)
     zq = _logits(zq, dtype)
     V = zp.shape[-1]
@@ -175,7 +178,7 @@ def row_chain(zp, zq, alpha: float, beta: float, T: float, q, child_tokens, dtyp
     ratios = np.empty(max(1, len(ct)), dtype=np.float64)
     r = np.empty(V, dtype=np.float64)
     rc = _load().dcd_oracle_row_chain(V, DTYPE_CODE[dtype], _ptr(zp), _ptr(zq), float(alpha), float(beta),
-                                      float(T), _ptr(q), len(ct), _ptr(ct), _ptr(ratios), _ptr(r))
+                                      float(T), _ptr(q), len(ct), _ptr(ct), int(distinct), _ptr(ratios), _ptr(r))
     if rc != 0:
         raise ValueError(f"oracle row_chain failed: {rc}")
     return ratios[: len(ct)], r
@@ -183,7 +186,7 @@ def row_chain(zp, zq, alpha: float, beta: float, T: float, q, child_tokens, dtyp
 
 def verify(*, B: int, N: int, V: int, dtype: str, z_exp, z_ama, tokens, parents, alpha, beta=None,
            temperature=None, q=None, seed: int = 0, offset: int = 0, ld=None, ldq=None,
-           nthreads: int = 1, want_residual: bool = False, seq_ids=None) -> dict:
+           nthreads: int = 1, want_residual: bool = False, seq_ids=None, distinct: bool = False) -> dict:
     """Full verification of B sequences x N nodes (see dcd_oracle_verify in the C source)."""
     zp = _logits(z_exp, dtype)
     zq = _logits(z_ama, dtype)
@@ -217,7 +220,8 @@ def verify(*, B: int, N: int, V: int, dtype: str, z_exp, z_ama, tokens, parents,
     residual = np.zeros((B, V), dtype=np.float64) if want_residual else None
     rc = _load().dcd_oracle_verify(
         B, N, V, DTYPE_CODE[dtype], ld, _ptr(zp), _ptr(zq), _ptr(tok), _ptr(par), _ptr(al), _ptr(be),
-        _ptr(te), _ptr(qq), ldq, seed, offset, _ptr(sid), nthreads, _ptr(accept_len), _ptr(path), _ptr(bonus),
+        _ptr(te), _ptr(qq), ldq, seed, offset, _ptr(sid), int(distinct), nthreads, _ptr(accept_len), _ptr(path),
+        _ptr(bonus),
         _ptr(logprob), _ptr(rows), _ptr(residual))
     if rc != 0:
         raise ValueError(f"oracle verify failed: {rc}")
@@ -225,7 +229,7 @@ def verify(*, B: int, N: int, V: int, dtype: str, z_exp, z_ama, tokens, parents,
                 cd_logprob=logprob.reshape(B, N), rows=rows.reshape(B, N), residual=residual)
 
 
-def verify_workload(w, nthreads: int = 1, want_residual: bool = False, seqs=None) -> dict:
+def verify_workload(w, nthreads: int = 1, want_residual: bool = False, seqs=None, distinct: bool = False) -> dict:
     """Runs ``verify`` on a workloads.Workload (optionally on a subset of its sequences)."""
     import torch
     B, N, V = w.B, w.N, w.V
@@ -237,7 +241,8 @@ def verify_workload(w, nthreads: int = 1, want_residual: bool = False, seqs=None
     return verify(B=len(sel), N=N, V=V, dtype=w.dtype, z_exp=zp, z_ama=zq,
                   tokens=w.tokens.cpu()[sel], parents=w.parents.cpu()[sel], alpha=w.alpha.cpu()[sel],
                   beta=w.beta.cpu()[sel], temperature=w.temperature.cpu()[sel], q=q, seed=w.seed,
-                  offset=w.offset, nthreads=nthreads, want_residual=want_residual, seq_ids=np.asarray(sel))
+                  offset=w.offset, nthreads=nthreads, want_residual=want_residual, seq_ids=np.asarray(sel),
+                  distinct=distinct)
 
 
 def margin_fn(zp_row, za_row, alpha: float, beta: float) -> float:

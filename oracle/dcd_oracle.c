@@ -23,7 +23,10 @@
  *      r_0 = pi_CD, child j (ascending node id) is accepted iff
  *      u_j <= r_{j-1}(t_j) / q(t_j); on rejection r_j = normalise(max(0,
  *      r_{j-1} - q)); if no child is accepted, the row's terminal token is drawn
- *      from the last residual (pi_CD itself at a leaf), "sample y_k ~ P_r";
+ *      from the last residual (pi_CD itself at a leaf), "sample y_k ~ P_r".
+ *      With siblings drawn without replacement ("distinct"), sibling j's proposal
+ *      q_{j-1} is q with the tokens of siblings 1..j-1 removed and renormalised, and it
+ *      takes q's place in both the ratio and the residual step;
  *   7. tree walk: from the root, descend into the accepted child while there is
  *      one; accept_len = number of accepted drafted tokens (the bonus token is
  *      excluded, App. D), the bonus is the terminal token of the last node.
@@ -239,6 +242,31 @@ static double residual_step(int64_t V, double* r, const float* q, double* tmp) {
   return z;
 }
 
+/* The same step against a proposal held in double precision (the renormalised proposal of a
+ * sibling drawn without replacement). */
+static double residual_step_d(int64_t V, double* r, const double* qd, double* tmp) {
+  double z = 0.0;
+  for (int64_t x = 0; x < V; ++x) {
+    const double d = r[x] - qd[x];
+    tmp[x] = d > 0.0 ? d : 0.0;
+    z += tmp[x];
+  }
+  if (z > 0.0)
+    for (int64_t x = 0; x < V; ++x) r[x] = tmp[x] / z;
+  return z;
+}
+
+/* Siblings drawn without replacement: after sibling token t is rejected, the next sibling's
+ * proposal is q with t removed and renormalised.  qd holds the current proposal. */
+static void remove_token(int64_t V, double* qd, int32_t t) {
+  if (qd[t] == 0.0) return; /* already removed (a duplicate sibling) */
+  qd[t] = 0.0;
+  double z = 0.0;
+  for (int64_t x = 0; x < V; ++x) z += qd[x];
+  if (z > 0.0)
+    for (int64_t x = 0; x < V; ++x) qd[x] /= z;
+}
+
 /* Acceptance ratio r(t)/q(t); q(t) = 0 gives +inf if r(t) > 0 and 0 (reject) otherwise. */
 static double accept_ratio(double rt, double qt) {
   if (qt > 0.0) return rt / qt;
@@ -328,29 +356,40 @@ int dcd_oracle_row_logpi(int64_t V, int dtype, const void* zp, const void* zq, d
  * ratios[j] = r_{j}(t_j) / q(t_j) for j = 0..m-1 (r_0 = pi_CD,T), and r_m in r_out[V].
  */
 int dcd_oracle_row_chain(int64_t V, int dtype, const void* zp, const void* zq, double alpha, double beta,
-                         double T, const float* q, int m, const int32_t* child_tokens, double* ratios,
+                         double T, const float* q, int m, const int32_t* child_tokens, int distinct, double* ratios,
                          double* r_out) {
   if (V <= 0 || !zp || !zq || !q || m < 0 || !r_out || T <= 0.0) return ORC_ERR_ARG;
   double* lp = malloc(sizeof(double) * (size_t)V);
   double* lq = malloc(sizeof(double) * (size_t)V);
   double* tmp = malloc(sizeof(double) * (size_t)V);
-  if (!lp || !lq || !tmp) {
+  double* qd = distinct ? malloc(sizeof(double) * (size_t)V) : NULL;
+  if (!lp || !lq || !tmp || (distinct && !qd)) {
     free(lp);
     free(lq);
     free(tmp);
+    free(qd);
     return ORC_ERR_MEM;
   }
   orc_row_target st;
   row_target(V, dtype, zp, zq, alpha, beta, T, lp, lq, r_out, &st);
   for (int64_t x = 0; x < V; ++x) r_out[x] = exp(r_out[x]);
+  if (distinct)
+    for (int64_t x = 0; x < V; ++x) qd[x] = (double)q[x];
   for (int j = 0; j < m; ++j) {
     const int32_t t = child_tokens[j];
-    ratios[j] = accept_ratio(r_out[t], (double)q[t]);
-    residual_step(V, r_out, q, tmp);
+    if (distinct) {
+      ratios[j] = accept_ratio(r_out[t], qd[t]);
+      residual_step_d(V, r_out, qd, tmp);
+      remove_token(V, qd, t);
+    } else {
+      ratios[j] = accept_ratio(r_out[t], (double)q[t]);
+      residual_step(V, r_out, q, tmp);
+    }
   }
   free(lp);
   free(lq);
   free(tmp);
+  free(qd);
   return ORC_OK;
 }
 
@@ -384,8 +423,8 @@ typedef struct {
 int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, const void* zp, const void* zq,
                       const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                       const float* temperature, const float* q, int64_t ldq, uint64_t seed, uint64_t offset,
-                      const int32_t* seq_ids, int nthreads, int32_t* accept_len, int32_t* accept_path, int32_t* bonus,
-                      double* cd_logprob, dcd_oracle_row* rows, double* residual) {
+                      const int32_t* seq_ids, int distinct, int nthreads, int32_t* accept_len, int32_t* accept_path,
+                      int32_t* bonus, double* cd_logprob, dcd_oracle_row* rows, double* residual) {
   if (B < 0 || N < 1 || V < 1 || (dtype < 0 || dtype > 2) || ld < 0 || !zp || !zq || !tokens || !parents ||
       !alpha || !accept_len || !accept_path || !bonus || !cd_logprob || !rows)
     return ORC_ERR_ARG;
@@ -412,8 +451,9 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
     double* lq = malloc(sizeof(double) * (size_t)V);
     double* r = malloc(sizeof(double) * (size_t)V);
     double* tmp = malloc(sizeof(double) * (size_t)V);
+    double* qd = malloc(sizeof(double) * (size_t)V);
     int32_t* kids = malloc(sizeof(int32_t) * (size_t)N);
-    const int have_mem = lp && lq && r && tmp && kids;
+    const int have_mem = lp && lq && r && tmp && qd && kids;
     if (!have_mem) {
 #pragma omp atomic write
       err = ORC_ERR_MEM;
@@ -459,13 +499,16 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
           if (out->acc_child < 0) out->term_token = st.argmax;
           continue;
         }
-        /* sampled rule: r_0 = pi_CD,T */
+        /* sampled rule: r_0 = pi_CD,T; siblings drawn without replacement each see q without
+           the tokens of the siblings rejected before them, renormalised */
         for (int64_t x = 0; x < V; ++x) r[x] = exp(r[x]);
         const float* qr = q + (size_t)(ldq * g);
+        if (distinct)
+          for (int64_t x = 0; x < V; ++x) qd[x] = (double)qr[x];
         for (int k = 0; k < m; ++k) {
           const int32_t c = kids[k];
           const int32_t t = tokens[(int64_t)b * N + c];
-          const double ratio = accept_ratio(r[t], (double)qr[t]);
+          const double ratio = distinct ? accept_ratio(r[t], qd[t]) : accept_ratio(r[t], (double)qr[t]);
           const int64_t sb = seq_ids ? seq_ids[b] : b;
           const double u = dcd_oracle_accept_uniform(seed, offset, (uint32_t)(sb * N + c));
           ++out->n_tests;
@@ -477,7 +520,12 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
             out->acc_child = c;
             break;
           }
-          residual_step(V, r, qr, tmp);
+          if (distinct) {
+            residual_step_d(V, r, qd, tmp);
+            remove_token(V, qd, t);
+          } else {
+            residual_step(V, r, qr, tmp);
+          }
         }
         if (out->acc_child < 0) {
           const int64_t sb = seq_ids ? seq_ids[b] : b;
@@ -489,6 +537,7 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
     free(lq);
     free(r);
     free(tmp);
+    free(qd);
     free(kids);
   }
   if (err) return err;
@@ -517,10 +566,12 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
       double* lp = malloc(sizeof(double) * (size_t)V);
       double* lq = malloc(sizeof(double) * (size_t)V);
       double* tmp = malloc(sizeof(double) * (size_t)V);
-      if (!lp || !lq || !tmp) {
+      double* qd = malloc(sizeof(double) * (size_t)V);
+      if (!lp || !lq || !tmp || !qd) {
         free(lp);
         free(lq);
         free(tmp);
+        free(qd);
         return ORC_ERR_MEM;
       }
       const int64_t g = (int64_t)b * N + cur;
@@ -529,11 +580,20 @@ int dcd_oracle_verify(int32_t B, int32_t N, int64_t V, int dtype, int64_t ld, co
                  alpha[b], beta ? beta[b] : 0.0, T, lp, lq, res, &st);
       for (int64_t x = 0; x < V; ++x) res[x] = exp(res[x]);
       const float* qr = q + (size_t)(ldq * g);
-      for (int32_t c = cur + 1; c < N; ++c)
-        if (parents[(int64_t)b * N + c] == cur) residual_step(V, res, qr, tmp);
+      for (int64_t x = 0; x < V; ++x) qd[x] = (double)qr[x];
+      for (int32_t c = cur + 1; c < N; ++c) {
+        if (parents[(int64_t)b * N + c] != cur) continue;
+        if (distinct) {
+          residual_step_d(V, res, qd, tmp);
+          remove_token(V, qd, tokens[(int64_t)b * N + c]);
+        } else {
+          residual_step(V, res, qr, tmp);
+        }
+      }
       free(lp);
       free(lq);
       free(tmp);
+      free(qd);
     }
   }
   return ORC_OK;

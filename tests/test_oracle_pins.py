@@ -517,3 +517,103 @@ def test_fused_logits_are_h_times_w_transposed():
             for k in range(11):
                 s += hd[r, k] * wd[v, k]
             assert abs(z[r, v] - s) < 1e-12
+
+
+def _emission_from_chain_distinct(zp, zq, alpha, beta, T, q, tokens):
+    ratios, rm = oracle.row_chain(zp, zq, alpha, beta, T, q, tokens, distinct=True)
+    V = len(zp)
+    emit = np.zeros(V)
+    reach = 1.0
+    for t, rho in zip(tokens, ratios):
+        a = min(1.0, rho)
+        emit[t] += reach * a
+        reach *= 1.0 - a
+    emit += reach * rm
+    return emit
+
+
+def _wor_tuples(q64, m):
+    """Every ordered tuple of m distinct draftable tokens with its probability under drawing
+    without replacement from q."""
+    V = len(q64)
+    for tup in itertools.permutations([x for x in range(V) if q64[x] > 0], m):
+        w, rest = 1.0, 1.0
+        for t in tup:
+            w *= q64[t] / rest
+            rest -= q64[t]
+        yield tup, w
+
+
+@pytest.mark.parametrize("m", [1, 2, 3])
+@pytest.mark.parametrize("alpha,beta,T", [(0.1, 0.0, 1.0), (0.5, 0.2, 1.0), (1.0, 0.0, 0.6)])
+def test_lossless_exact_enumeration_siblings_without_replacement(m, alpha, beta, T):
+    """Siblings drawn without replacement from q (distinct tokens): with each sibling tested
+    against q less the earlier siblings' tokens, renormalised, the first emitted token is
+    distributed as pi_CD, to 1e-12, over every ordered tuple of distinct tokens."""
+    rng = np.random.default_rng(m * 37 + int(alpha * 10))
+    V = 5
+    zp, zq = _rows(rng, V, scale=1.0)
+    qd = _dyadic_distribution(special.softmax(zp + rng.standard_normal(V)), zero_last=True)
+    q64 = qd.astype(np.float64)
+    total = np.zeros(V)
+    wsum = 0.0
+    for tup, w in _wor_tuples(q64, m):
+        total += w * _emission_from_chain_distinct(zp, zq, alpha, beta, T, qd, list(tup))
+        wsum += w
+    assert abs(wsum - 1.0) < 1e-12
+    pi = np.exp(oracle.row_logpi(zp, zq, alpha, beta, T)["logpi"])
+    np.testing.assert_allclose(total, pi, rtol=0, atol=1e-12)
+
+
+def test_iid_rule_is_not_lossless_for_distinct_siblings():
+    """The plausible mistake of keeping q unchanged for distinct siblings: the i.i.d. rule on
+    tuples drawn without replacement does not emit pi_CD (so the pin above separates the two)."""
+    rng = np.random.default_rng(7)
+    V = 5
+    zp, zq = _rows(rng, V, scale=1.0)
+    qd = _dyadic_distribution(special.softmax(zp + rng.standard_normal(V)), zero_last=True)
+    q64 = qd.astype(np.float64)
+    total = np.zeros(V)
+    for tup, w in _wor_tuples(q64, 2):
+        total += w * _emission_from_chain(zp, zq, 0.3, 0.0, 1.0, qd, list(tup))
+    pi = np.exp(oracle.row_logpi(zp, zq, 0.3, 0.0, 1.0)["logpi"])
+    assert np.abs(total - pi).max() > 1e-4
+
+
+def test_distinct_rule_equals_iid_rule_for_one_sibling():
+    rng = np.random.default_rng(8)
+    V = 40
+    zp, zq = _rows(rng, V, scale=2.0)
+    q = special.softmax(zp + rng.standard_normal(V)).astype(np.float32)
+    r1, m1 = oracle.row_chain(zp, zq, 0.2, 0.0, 1.0, q, [int(np.argmax(q))])
+    r2, m2 = oracle.row_chain(zp, zq, 0.2, 0.0, 1.0, q, [int(np.argmax(q))], distinct=True)
+    np.testing.assert_array_equal(r1, r2)
+    np.testing.assert_array_equal(m1, m2)
+
+
+def test_lossless_monte_carlo_full_verify_siblings_without_replacement():
+    """Full sampled verification with the distinct-sibling rule (Philox, ratio test, residuals,
+    race) on siblings drawn without replacement from q emits pi_CD."""
+    rng = np.random.default_rng(321)
+    V, B, m = 6, 120000, 3
+    zp, zq = _rows(rng, V, scale=1.0)
+    alpha, T = 0.3, 1.0
+    qd = special.softmax(zp + 0.8 * rng.standard_normal(V)).astype(np.float32)
+    qd = (qd / qd.sum(dtype=np.float64)).astype(np.float32)
+    p64 = qd.astype(np.float64) / qd.sum(dtype=np.float64)
+    N = 1 + m
+    parents = np.tile(np.array([-1, 0, 0, 0], dtype=np.int32), (B, 1))
+    tokens = np.zeros((B, N), dtype=np.int32)
+    # m distinct tokens per sequence, in draw order: Gumbel top-m is sampling without replacement
+    gk = np.log(p64)[None, :] - np.log(-np.log(rng.random((B, V))))
+    tokens[:, 1:] = np.argsort(-gk, axis=1)[:, :m]
+    res = oracle.verify(B=B, N=N, V=V, dtype="f64", z_exp=zp, z_ama=zq, ld=0, tokens=tokens,
+                        parents=parents, alpha=np.full(B, alpha), beta=np.zeros(B),
+                        temperature=np.full(B, T), q=qd, ldq=0, seed=77, offset=3, nthreads=4, distinct=True)
+    first = _first_emitted(res, tokens)
+    counts = np.bincount(first, minlength=V)
+    pi = np.exp(oracle.row_logpi(zp, zq, alpha, 0.0, T)["logpi"])
+    tv = 0.5 * np.abs(counts / B - pi).sum()
+    assert tv < 3.0 * np.sqrt(V / B)
+    chi = stats.chisquare(counts[pi > 0], B * pi[pi > 0])
+    assert chi.pvalue > 1e-4
