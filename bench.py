@@ -147,7 +147,7 @@ def algorithmic_bytes(w, residual_rows: float) -> float:
     return logits + qb + small
 
 
-def residual_rows_per_step(w, out, ws, stream, offsets) -> float:
+def residual_rows_per_step(w, out, ws, stream, offsets, distinct: bool = False) -> float:
     """Mean number of rows handed to residual passes over the given Philox offsets (the
     workspace header's word 4 counts them; the outcome depends only on inputs and offset)."""
     import torch
@@ -157,7 +157,8 @@ def residual_rows_per_step(w, out, ws, stream, offsets) -> float:
     counts = []
     for off in offsets:
         dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q,
-                           temperature=w.temperature, seed=w.seed, offset=off, out=out, workspace=ws, stream=stream)
+                           temperature=w.temperature, seed=w.seed, offset=off, out=out, workspace=ws, stream=stream,
+                           distinct=distinct)
         counts.append(ws[16:20].view(torch.int32).clone())
     torch.cuda.synchronize()
     return float(torch.stack(counts).double().mean().item())
@@ -261,7 +262,8 @@ def run_ours(args):
                                stream=stream)
         else:
             dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q,
-                               temperature=w.temperature, seed=w.seed, offset=i, out=out, workspace=ws, stream=stream)
+                               temperature=w.temperature, seed=w.seed, offset=i, out=out, workspace=ws, stream=stream,
+                               distinct=args.distinct)
         if evs is not None:
             evs[1].record(stream)
         dcd.dcd_tree_walk(B, N, V, out, ws, stream=stream)
@@ -309,7 +311,7 @@ def run_ours(args):
     # roofline of the dominant kernel (the row kernel) from its own events; the rows that took
     # residual passes are counted on a replay of every 32nd timed offset
     replay = [1_000_000 + k for k in range(0, args.steps, 32)]
-    res_rows = residual_rows_per_step(w, out, ws, stream, replay)
+    res_rows = residual_rows_per_step(w, out, ws, stream, replay, args.distinct)
     alg = algorithmic_bytes(w, res_rows)
     row_avg_s = statistics.mean(row_ms) / 1e3
     achieved = alg / row_avg_s / 1e9
@@ -339,7 +341,7 @@ def run_ours(args):
                 dst[k].copy_(host[k], non_blocking=True)
             o = dcd.dcd_verify_sample(dst["z_exp"], dst["z_ama"], dst["q"], dst["tokens"], dst["parents"],
                                       dst["alpha"], dst["temperature"], w.seed, 2_000_000 + i, dst["beta"], out=out,
-                                      workspace=ws, stream=stream)
+                                      workspace=ws, stream=stream, distinct=args.distinct)
             for k in res_host:
                 res_host[k].copy_(o[k], non_blocking=True)
 
@@ -363,7 +365,9 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": WORKLOAD if B == 32 else f"{WORKLOAD} (profiling case, B={B})", "B": B, "N": N, "V": V, "rows": R, "logits": "bf16",
+            "config": {"workload": (WORKLOAD if B == 32 else f"{WORKLOAD} (profiling case, B={B})") +
+                       (" siblings-without-replacement" if args.distinct else ""),
+                       "B": B, "N": N, "V": V, "rows": R, "logits": "bf16",
                        "sampled_sequences": int((w.temperature > 0).sum().item()),
                        "bytes_per_step": alg, "l2": "inputs (1.97 GB resident) larger than L2; no flush",
                        "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
@@ -525,6 +529,8 @@ def main():
     ap.add_argument("--greedy", action="store_true", help="every sequence greedy (profiling case)")
     ap.add_argument("--batch", type=int, default=32,
                     help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
+    ap.add_argument("--distinct", action="store_true",
+                    help="sampled rule for siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)")
     ap.add_argument("--workload", choices=("batched", "fused"), default="batched",
                     help="batched: the streaming step on materialised logits (the headline); fused: the "
                          "fused LM-head variant")

@@ -88,13 +88,25 @@ enum {
 /* Logit element types. */
 enum { DCD_F32 = 0, DCD_BF16 = 1 };
 
+/*
+ * dcd_shape.flags: DCD_SIBLINGS_DISTINCT selects the sampled rule for sibling lists drawn
+ * WITHOUT replacement from q (distinct drafted tokens, EAGLE-style top-k sampling): sibling j
+ * is tested against r_{j-1} with its actual proposal q_{j-1} = q without the tokens of siblings
+ * 1..j-1, renormalised, which also replaces q in the residual step r_j = normalise(max(0,
+ * r_{j-1} - q_{j-1})).  Without the flag siblings are taken as i.i.d. draws from q.  The flag
+ * supports nodes with at most 32 children (more: DCD_DEVERR_UNSUPPORTED for the sequence); the
+ * remaining mass of q is taken as 1 minus the removed tokens' q (q rows sum to 1).
+ */
+#define DCD_SIBLINGS_DISTINCT 0x1
+
 /* Bits of the device error word (dcd_get_device_error). */
 #define DCD_DEVERR_BAD_PARENT 0x1u  /* parents[] violates the ordering rule */
 #define DCD_DEVERR_BAD_TOKEN 0x2u   /* a drafted token is outside [0, V) */
 #define DCD_DEVERR_NONFINITE 0x4u   /* NaN / +inf reached a row's max or normaliser */
 #define DCD_DEVERR_TIMEOUT 0x8u     /* a bounded wait on an asynchronous copy expired */
 #define DCD_DEVERR_BAD_PARAM 0x10u  /* alpha < 0, beta outside [0, 1], T < 0 or non-finite */
-#define DCD_DEVERR_UNSUPPORTED 0x20u /* fused LM-head call: a node has more than 8 children */
+#define DCD_DEVERR_UNSUPPORTED 0x20u /* a node has more children than the call supports (fused
+                                        LM-head: 8; DCD_SIBLINGS_DISTINCT: 32) */
 
 /* Largest tree (nodes per sequence, root included) the library accepts. */
 #define DCD_MAX_NODES 1024
@@ -104,7 +116,7 @@ typedef struct {
   int32_t N;            /* nodes per sequence, root included (1 .. DCD_MAX_NODES) */
   int64_t V;            /* vocabulary size (1 .. 2^31 - 1) */
   int32_t logits_dtype; /* DCD_F32 or DCD_BF16, for z_exp and z_ama */
-  int32_t reserved;     /* must be 0 */
+  int32_t flags;        /* 0, or DCD_SIBLINGS_DISTINCT (sampled calls); other bits must be 0 */
   int64_t ld_logits;    /* row stride of z_exp / z_ama in elements (>= V) */
   int64_t ld_q;         /* row stride of q in fp32 elements (>= V; sampled calls only) */
 } dcd_shape;

@@ -15,7 +15,7 @@ constexpr int kVersion = 10000;  // 1.0.0
 
 bool shape_ok(const dcd_shape* s, bool need_q) {
   if (!s) return false;
-  if (s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || s->reserved != 0) return false;
+  if (s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || (s->flags & ~DCD_SIBLINGS_DISTINCT) != 0) return false;
   if (s->logits_dtype != DCD_F32 && s->logits_dtype != DCD_BF16) return false;
   if (s->ld_logits < s->V) return false;
   if (need_q && s->ld_q < s->V) return false;
@@ -99,6 +99,7 @@ dcd::ScoreArgs make_args(const dcd_shape* s, const void* z_exp, const void* z_am
   a.slots = v.slots;
   a.force_stages = 0;
   a.force_plain = 0;
+  a.distinct = (s->flags & DCD_SIBLINGS_DISTINCT) ? 1 : 0;
   return a;
 }
 
@@ -187,7 +188,7 @@ int dcd_verify_sample(const dcd_shape* shape, const void* z_exp, const void* z_a
 }
 
 size_t dcd_fused_workspace_bytes(const dcd_shape* s) {
-  if (!s || s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || s->reserved != 0) return 0;
+  if (!s || s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || s->flags != 0) return 0;
   if (s->logits_dtype != DCD_BF16) return 0;
   if (static_cast<int64_t>(s->B) * s->N > INT_MAX / 16) return 0;
   return dcd::fused_layout(static_cast<int64_t>(s->B) * s->N, s->V).total;

@@ -69,12 +69,22 @@ static_assert(sizeof(RowPart) == 32, "RowPart layout");
 struct SlotHead {  // chain state of a handed-over row
   int32_t g, m;    // row, children of its node
   float M, S, Mp;  // max CD score, normaliser sum 2^((s' - M) k2), expert max
-  float c, D;      // c_J and D_J of the residual r_J = max(0, pi - c_J q) / D_J last computed
+  float c, D;      // c and mass of the current residual r = max(0, pi - c q) / D (as of the last pass)
   int32_t degen;   // a pass found no residual mass
   uint32_t status;
-  int32_t pad[7];
+  float Z;         // distinct siblings: mass of q not yet removed
+  int32_t nrem;    // distinct siblings: tokens removed (first occurrences), listed after the parts
+  int32_t pad[5];
 };
 static_assert(sizeof(SlotHead) == 64, "SlotHead layout");
+
+// Distinct siblings: a removed token and its frozen residual mass max(0, pi - c q) at the c in
+// effect when it was removed (the residual does not change there afterwards: its proposal is 0).
+struct Removed {
+  int32_t tok;
+  float fz;
+};
+constexpr int kMaxRemoved = 32;
 
 struct PiecePart {  // one piece's share of a residual pass
   float z;          // sum of max(0, pi - c_J q) over the piece
@@ -106,6 +116,7 @@ struct ScoreArgs {
   RowRecord* rec;
   RowPart* parts;   // per row: kMaxParts part statistics
   unsigned char* slots;
+  int32_t distinct;       // 1: siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)
   int32_t force_stages;   // 0 = automatic, else the ring depth to use (tests / tuning)
   int32_t force_plain;    // 1 = plain loads instead of bulk async copies
 };

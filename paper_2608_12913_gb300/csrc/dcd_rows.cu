@@ -165,6 +165,18 @@ __device__ __forceinline__ PiecePart* slot_parts(const SParams& sp, int s) {
   return reinterpret_cast<PiecePart*>(sp.slots + static_cast<size_t>(s) * sp.slot_bytes + sizeof(SlotHead));
 }
 
+// Distinct siblings: the removed tokens of a chain, after its pieces' parts.
+__device__ __forceinline__ Removed* slot_removed(const SParams& sp, int s) {
+  return reinterpret_cast<Removed*>(sp.slots + static_cast<size_t>(s) * sp.slot_bytes + sizeof(SlotHead) +
+                                    static_cast<size_t>(sp.npieces) * sizeof(PiecePart));
+}
+
+__device__ __forceinline__ int find_removed(const Removed* rem, int nrem, int t) {
+  for (int i = 0; i < nrem; ++i)
+    if (rem[i].tok == t) return i;
+  return -1;
+}
+
 // Publishes residual pass `job` (its counters are reset here; one consumer thread).  Passes are
 // published in creation order, so the passes with unclaimed pieces are the window [job_head,
 // jobs_published); the wait for the previous creator spans a few stores and is bounded.
@@ -312,7 +324,9 @@ __device__ __forceinline__ void warp_release(uint64_t* bar) {
 }
 
 // ------------------------------------------------------------------------------------------
-template <typename TIn>
+// kDistinct: siblings drawn without replacement (a separate instantiation, so that the i.i.d.
+// rule's code and registers are untouched by the distinct rule's bookkeeping).
+template <typename TIn, bool kDistinct>
 __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(const __grid_constant__ SParams sp) {
   const ScoreArgs& p = sp.a;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -661,8 +675,22 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           piece_lo + static_cast<int64_t>(tid) * kRaceBlock < V) {
         float mass = 0.f;
         for (int i = 0; i < wpb; ++i) mass += csum[tid * wpb + i];
+        const int kabs = static_cast<int>(piece_lo / kRaceBlock) + tid;
+        if (kDistinct) {
+          // removed siblings' tokens in this block carry their frozen mass, not the streamed one
+          const SlotHead* sh = slot_head(sp, D.slot);
+          const Removed* rem = slot_removed(sp, D.slot);
+          const int nrem = sh->nrem;
+          for (int i = 0; i < nrem; ++i) {
+            const int t = rem[i].tok;
+            if (t / kRaceBlock != kabs) continue;
+            const float z = ld1(zp_row, t);
+            const bool in = !masked || (z - Mp >= logb);
+            const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, t)) - M) * invS : 0.f;
+            mass += rem[i].fz - fmaxf(pit - cJ * q_row[t], 0.f);
+          }
+        }
         if (mass > 0.f) {
-          const int kabs = static_cast<int>(piece_lo / kRaceBlock) + tid;
           bk = block_key(p, g, kabs, lg2(mass));
           bb = kabs;
         }
@@ -695,6 +723,102 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           }
           bool degen = sh->degen != 0;
           float c = sh->c, Dn = sh->D;
+          int acc = -1;
+          bool queued = false, ranked = J == m;
+          if (kDistinct) {
+            // Siblings without replacement.  With the tokens removed so far frozen at their
+            // mass fz, the residual after this pass is max(0, pi - c_J q) elsewhere: its mass is
+            // the streamed sum corrected at the removed tokens.  A pass without mass keeps the
+            // residual it started from.  Then sibling J's token is removed from the proposal
+            // (frozen at the current residual) and the next siblings are tested against r with
+            // the proposal q / Z without the removed tokens.
+            Removed* rem = slot_removed(sp, D.slot);
+            int nrem = sh->nrem;
+            float Z = sh->Z;
+            auto value_at = [&](int t, float& pit, float& qt) {
+              const float z = ld1(zp_row, t);
+              const bool in = !masked || (z - Mp >= logb);
+              pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, t)) - M) * invS : 0.f;
+              qt = q_row[t];
+            };
+            float EJ = DJ;
+            for (int i = 0; i < nrem; ++i) {
+              float pit, qt;
+              value_at(rem[i].tok, pit, qt);
+              EJ += rem[i].fz - fmaxf(pit - cJ * qt, 0.f);
+            }
+            if (EJ > 0.f) {
+              c = cJ;
+              Dn = EJ;
+            } else {
+              ranked = false;  // the pieces ranked blocks of a residual that is not used
+            }
+            auto remove = [&](int t) {
+              if (t < 0 || t >= V || find_removed(rem, nrem, t) >= 0) return;
+              if (nrem >= kMaxRemoved) {
+                st2 |= DCD_DEVERR_UNSUPPORTED;
+                return;
+              }
+              float pit, qt;
+              value_at(t, pit, qt);
+              rem[nrem].tok = t;
+              rem[nrem].fz = fmaxf(pit - c * qt, 0.f);
+              ++nrem;
+              Z -= qt;
+            };
+            remove(ktok[J - 1]);
+            for (int j = J; j < m; ++j) {
+              const int t = ktok[j];
+              float ratio = 0.f;
+              if (t >= 0 && t < V) {
+                const int ri = find_removed(rem, nrem, t);
+                if (ri >= 0) {
+                  ratio = rem[ri].fz > 0.f ? INFINITY : 0.f;  // its proposal is 0
+                } else {
+                  float pit, qt;
+                  value_at(t, pit, qt);
+                  const float rho = fmaxf(pit - c * qt, 0.f);
+                  const float qp = Z > 0.f ? qt / Z : 0.f;
+                  ratio = qp > 0.f ? (rho / Dn) / qp : (rho > 0.f ? INFINITY : 0.f);
+                }
+              }
+              const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[j]);
+              if (u01(philox_block(p.seed, p.offset, G, 0u).x) <= ratio) {
+                acc = kids[j];
+                break;
+              }
+              if (Z > 0.f) {
+                sh->c = c;
+                sh->D = Dn;
+                sh->Z = Z;
+                sh->nrem = nrem;
+                sh->status = st2;
+                Job nj;
+                nj.slot = D.slot;
+                nj.J = j + 1;
+                nj.g = static_cast<int32_t>(g);
+                nj.m = m;
+                nj.status = st2;
+                nj.M = M;
+                nj.S = D.S;
+                nj.Mp = Mp;
+                nj.c = c + Dn / Z;  // the next residual: max(0, r - q / Z) off the removed tokens
+                nj.alpha = alpha;
+                nj.beta = beta;
+                nj.T = T;
+                create_job(sp, nj);
+                queued = true;
+                break;
+              }
+              // every token of q is removed: the proposal is 0 and the residual stays
+              ranked = false;
+              remove(t);
+            }
+            if (!queued) {
+              sh->nrem = nrem;  // the final race reads the removed tokens
+              sh->Z = Z;
+            }
+          } else {
           if (DJ > 0.f) {
             c = cJ;
             Dn = DJ;
@@ -702,8 +826,6 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
             degen = true;  // r_{J-1} == q in exact arithmetic: r_J is taken as q from here on
           }
           // test the remaining siblings; after a pass without residual mass no pass is needed
-          int acc = -1;
-          bool queued = false;
           for (int j = J; j < m; ++j) {
             if (sibling_test<TIn>(p, b, kids[j], ktok[j], zp_row, zq_row, q_row, c1k, ak, masked, Mp, logb, M, invS,
                                   c, Dn, degen)) {
@@ -733,8 +855,9 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
               break;
             }
           }
+          }
           rs->accept = queued ? -2 : acc;
-          rs->term = kstar;  // the winning race block when this pass ranked them
+          rs->term = ranked ? kstar : INT_MAX - 1;  // the winning block when this pass ranked r_m
           rs->status = st2;
           rs->c = c;
           rs->D = Dn;
@@ -749,7 +872,40 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
             const bool degen = rs->degen != 0;
             const float c = rs->c, Dn = rs->D;
             int kstar = rs->term;
-            if (degen) {
+            const Removed* rem = slot_removed(sp, D.slot);
+            const int nrem = kDistinct ? slot_head(sp, D.slot)->nrem : 0;
+            auto rho_at = [&](int64_t x) -> float {  // the final residual's unnormalised mass
+              if (kDistinct) {
+                const int ri = find_removed(rem, nrem, static_cast<int>(x));
+                if (ri >= 0) return rem[ri].fz;
+              }
+              const float z = ld1(zp_row, x);
+              const bool in = !masked || (z - Mp >= logb);
+              const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
+              return fmaxf(pit - c * q_row[x], 0.f);
+            };
+            if (kDistinct && kstar == INT_MAX - 1) {
+              // block masses of the final residual, computed by this CTA alone (rare: the last
+              // pass found no mass, or q was used up)
+              float bk2 = -INFINITY;
+              int bb2 = INT_MAX;
+              for (int kb = warp; kb < sp.nblk; kb += kWarps) {
+                float part = 0.f;
+                for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < V && x < (kb + 1) * kRaceBlock;
+                     x += 32)
+                  part += rho_at(x);
+                const float mass = warp_sum(part);
+                if (lane == 0 && mass > 0.f) {
+                  const float key = block_key(p, g, kb, lg2(mass));
+                  if (key > bk2) {
+                    bk2 = key;
+                    bb2 = kb;
+                  }
+                }
+              }
+              block_argmax(bk2, bb2, redf, redi, csync);
+              kstar = bb2;
+            } else if (degen) {
               // block masses of q, computed by this CTA alone (rare: a residual without mass)
               float bk2 = -INFINITY;
               int bb2 = INT_MAX;
@@ -773,12 +929,8 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
             term = token_race(
                 p, g, kstar,
                 [&](int64_t x) -> float {
-                  const float qe = q_row[x];
-                  if (degen) return qe;
-                  const float z = ld1(zp_row, x);
-                  const bool in = !masked || (z - Mp >= logb);
-                  const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
-                  return fmaxf(pit - c * qe, 0.f) / Dn;
+                  if (degen && !kDistinct) return q_row[x];
+                  return rho_at(x) / Dn;
                 },
                 redf, redi);
           }
@@ -1025,6 +1177,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       else csync();
     }
     if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
+    if (sampled && kDistinct && m > kMaxRemoved) status |= DCD_DEVERR_UNSUPPORTED;
     // log sum exp(s' / T) over P_beta = M ln 2 + ln S
     const float logS = logf(S);
     const float invS = 1.f / S;
@@ -1065,7 +1218,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         const float u = u01(philox_block(p.seed, p.offset, G, 0u).x);
         int accept = u <= ratio ? 1 : 0;
         if (!accept && !(status & (DCD_DEVERR_BAD_PARENT | DCD_DEVERR_BAD_TOKEN | DCD_DEVERR_BAD_PARAM |
-                                   DCD_DEVERR_NONFINITE))) {
+                                   DCD_DEVERR_NONFINITE | DCD_DEVERR_UNSUPPORTED))) {
           const int s = static_cast<int>(atomicAdd(&sp.hdr->nslots, 1u));
           SlotHead* sh = slot_head(sp, s);
           sh->g = static_cast<int32_t>(g);
@@ -1077,6 +1230,8 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           sh->D = 1.f;
           sh->degen = 0;
           sh->status = status;
+          sh->Z = 1.f;  // distinct siblings: nothing removed yet
+          sh->nrem = 0;
           Job nj;
           nj.slot = s;
           nj.J = 1;
@@ -1231,22 +1386,44 @@ __global__ void __launch_bounds__(kThreads) terminal_residual_kernel(const Score
   for (int64_t x = threadIdx.x; x < V; x += kThreads) out[x] *= inv;
   __syncthreads();
   // every child of the terminal node was rejected, in ascending node id
+  __shared__ int removed[kMaxRemoved];
+  __shared__ float zrem;
+  int nrem = 0;
+  if (threadIdx.x == 0) zrem = 1.f;
+  __syncthreads();
   for (int c = cur + 1; c < N; ++c) {
     if (p.parents[static_cast<int64_t>(b) * N + c] != cur) continue;
+    // the proposal of this sibling: q, or (distinct siblings) q without the removed tokens / Z
+    const float Z = zrem;
+    auto prop = [&](int64_t x) -> float {
+      if (!p.distinct) return q[x];
+      for (int i = 0; i < nrem; ++i)
+        if (removed[i] == x) return 0.f;
+      return Z > 0.f ? q[x] / Z : 0.f;
+    };
     float z = 0.f;
-    for (int64_t x = threadIdx.x; x < V; x += kThreads) {
-      const float nv = fmaxf(out[x] - q[x], 0.f);
-      out[x] = nv;
-      z += nv;
-    }
+    for (int64_t x = threadIdx.x; x < V; x += kThreads) z += fmaxf(out[x] - prop(x), 0.f);
     z = block_sum(z, redf);
     if (z > 0.f) {
       const float iz = 1.f / z;
-      for (int64_t x = threadIdx.x; x < V; x += kThreads) out[x] *= iz;
-    } else {
+      for (int64_t x = threadIdx.x; x < V; x += kThreads) out[x] = fmaxf(out[x] - prop(x), 0.f) * iz;
+    } else if (!p.distinct) {
       for (int64_t x = threadIdx.x; x < V; x += kThreads) out[x] = q[x];
-    }
+    }  // distinct siblings: a step without mass leaves the residual as it is
     __syncthreads();
+    if (p.distinct) {
+      const int t = p.tokens[static_cast<int64_t>(b) * N + c];
+      bool seen = t < 0 || t >= V;
+      for (int i = 0; i < nrem; ++i) seen = seen || removed[i] == t;
+      if (!seen && nrem < kMaxRemoved) {
+        if (threadIdx.x == 0) {
+          removed[nrem] = t;
+          zrem = Z - q[t];
+        }
+        ++nrem;
+      }
+      __syncthreads();
+    }
   }
 }
 
@@ -1266,8 +1443,11 @@ cudaError_t prepare_kernel(int* sms) {
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   std::call_once(once[dev], [&] {
     DeviceInfo d;
-    d.err = cudaFuncSetAttribute(score_rows_kernel<TIn>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    d.err = cudaFuncSetAttribute(score_rows_kernel<TIn, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(kSmemMax));
+    if (d.err == cudaSuccess)
+      d.err = cudaFuncSetAttribute(score_rows_kernel<TIn, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   static_cast<int>(kSmemMax));
     if (d.err == cudaSuccess) d.err = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
     info[dev] = d;
   });
@@ -1323,7 +1503,8 @@ int residual_pieces(int64_t V, int dtype) {
 }
 
 size_t slot_bytes(int64_t V, int dtype) {
-  return sizeof(SlotHead) + static_cast<size_t>(residual_pieces(V, dtype)) * sizeof(PiecePart);
+  return sizeof(SlotHead) + static_cast<size_t>(residual_pieces(V, dtype)) * sizeof(PiecePart) +
+         kMaxRemoved * sizeof(Removed);
 }
 
 RowGeometry row_geometry(const ScoreArgs& a) {
@@ -1376,10 +1557,12 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   // a CTA may wait for work queued by another, so all CTAs must be resident at once: the grid is
   // the resident capacity (capped at the row count) and the launch is cooperative
   int per_sm = 0;
-  e = a.dtype == DCD_BF16 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<__nv_bfloat16>,
-                                                                          kCtaThreads, geo.smem)
-                          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_rows_kernel<float>,
-                                                                          kCtaThreads, geo.smem);
+  const void* fn = a.dtype == DCD_BF16
+                       ? (a.distinct ? reinterpret_cast<const void*>(score_rows_kernel<__nv_bfloat16, true>)
+                                     : reinterpret_cast<const void*>(score_rows_kernel<__nv_bfloat16, false>))
+                       : (a.distinct ? reinterpret_cast<const void*>(score_rows_kernel<float, true>)
+                                     : reinterpret_cast<const void*>(score_rows_kernel<float, false>));
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kCtaThreads, geo.smem);
   if (e != cudaSuccess) return e;
   if (per_sm > geo.ctas_per_sm) per_sm = geo.ctas_per_sm;
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
@@ -1406,8 +1589,11 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (a.dtype == DCD_BF16) return cudaLaunchKernelEx(&cfg, score_rows_kernel<__nv_bfloat16>, sp);
-  return cudaLaunchKernelEx(&cfg, score_rows_kernel<float>, sp);
+  if (a.dtype == DCD_BF16)
+    return a.distinct ? cudaLaunchKernelEx(&cfg, score_rows_kernel<__nv_bfloat16, true>, sp)
+                      : cudaLaunchKernelEx(&cfg, score_rows_kernel<__nv_bfloat16, false>, sp);
+  return a.distinct ? cudaLaunchKernelEx(&cfg, score_rows_kernel<float, true>, sp)
+                    : cudaLaunchKernelEx(&cfg, score_rows_kernel<float, false>, sp);
 }
 
 cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_t* err, int32_t* accept_len,

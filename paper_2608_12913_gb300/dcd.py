@@ -29,7 +29,7 @@ _lib = None
 
 class DcdShape(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("N", ctypes.c_int32), ("V", ctypes.c_int64),
-                ("logits_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("logits_dtype", ctypes.c_int32), ("flags", ctypes.c_int32),
                 ("ld_logits", ctypes.c_int64), ("ld_q", ctypes.c_int64)]
 
 
@@ -124,8 +124,12 @@ def _logits_dtype(t: torch.Tensor) -> int:
     raise TypeError(f"logits must be bfloat16 or float32, got {t.dtype}")
 
 
-def make_shape(B: int, N: int, V: int, dtype: int, ld: Optional[int] = None, ldq: Optional[int] = None) -> DcdShape:
-    return DcdShape(B, N, V, dtype, 0, V if ld is None else ld, (V if ldq is None else ldq))
+DCD_SIBLINGS_DISTINCT = 0x1
+
+
+def make_shape(B: int, N: int, V: int, dtype: int, ld: Optional[int] = None, ldq: Optional[int] = None,
+               flags: int = 0) -> DcdShape:
+    return DcdShape(B, N, V, dtype, flags, V if ld is None else ld, (V if ldq is None else ldq))
 
 
 def workspace_bytes(B: int, N: int, V: int, dtype: int = DCD_BF16) -> int:
@@ -159,7 +163,7 @@ def alloc_outputs(B: int, N: int, device, V: Optional[int] = None, residual: boo
 class _Call:
     """Validated arguments of one verification call."""
 
-    def __init__(self, z_exp, z_ama, tokens, parents, alpha, beta, q=None, temperature=None):
+    def __init__(self, z_exp, z_ama, tokens, parents, alpha, beta, q=None, temperature=None, distinct=False):
         _require(z_exp, "z_exp")
         dev = z_exp.device
         if z_exp.dim() != 2 or z_exp.stride(1) != 1:
@@ -190,7 +194,8 @@ class _Call:
             _require(temperature, "temperature", dtype=torch.float32, device=dev, shape=(B,))
         self.device = dev
         self.B, self.N, self.V = B, N, V
-        self.shape = make_shape(B, N, V, _logits_dtype(z_exp), z_exp.stride(0), ldq)
+        self.shape = make_shape(B, N, V, _logits_dtype(z_exp), z_exp.stride(0), ldq,
+                                DCD_SIBLINGS_DISTINCT if distinct else 0)
         self.args = (z_exp, z_ama, q, tokens, parents, alpha, beta, temperature)
 
     def workspace(self, workspace):
@@ -224,9 +229,9 @@ def dcd_verify_greedy(z_exp, z_ama, tokens, parents, alpha, beta=None, *, out=No
 
 
 def dcd_verify_sample(z_exp, z_ama, q, tokens, parents, alpha, temperature, seed: int, offset: int, beta=None, *,
-                      residual: bool = False, out=None, workspace=None, stream=None) -> dict:
+                      residual: bool = False, out=None, workspace=None, stream=None, distinct: bool = False) -> dict:
     """Speculative-sampling CD verification (greedy for sequences with temperature 0)."""
-    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature, distinct=distinct)
     ws = c.workspace(workspace)
     o = c.outputs(out, residual=residual)
     st = load().dcd_verify_sample(
@@ -241,13 +246,13 @@ def dcd_verify_sample(z_exp, z_ama, q, tokens, parents, alpha, temperature, seed
 
 
 def dcd_verify_sample_noalloc(z_exp, z_ama, q, tokens, parents, alpha, temperature, seed: int, offset: int,
-                              beta=None, *, residual: bool = False, out=None, stream=None) -> dict:
+                              beta=None, *, residual: bool = False, out=None, stream=None, distinct: bool = False) -> dict:
     """dcd_verify_sample with the library's built-in scratch instead of a caller workspace.
 
     For callers that cannot allocate device memory (see include/dcd.h).  Calls that overlap on the
     GPU share that scratch and race; the caller serialises them.
     """
-    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature, distinct=distinct)
     o = c.outputs(out, residual=residual)
     st = load().dcd_verify_sample_noalloc(
         ctypes.byref(c.shape), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(tokens), _ptr(parents), _ptr(alpha),
@@ -261,9 +266,9 @@ def dcd_verify_sample_noalloc(z_exp, z_ama, q, tokens, parents, alpha, temperatu
 
 def dcd_score_rows(z_exp, z_ama, tokens, parents, alpha, beta=None, q=None, temperature=None, seed: int = 0,
                    offset: int = 0, *, out=None, workspace=None, stream=None, stages: int = 0,
-                   plain_loads: bool = False) -> dict:
+                   plain_loads: bool = False, distinct: bool = False) -> dict:
     """The per-row step alone (records stay in the workspace); see dcd_tree_walk."""
-    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature)
+    c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature, distinct=distinct)
     ws = c.workspace(workspace)
     o = c.outputs(out)
     lib = load()

@@ -40,7 +40,7 @@ def records(ws: torch.Tensor, R: int):
 
 
 def run_gpu(w, *, sampled: bool, residual: bool = False, stages: int = 0, plain: bool = False, offset=None,
-            out=None, workspace=None):
+            out=None, workspace=None, distinct: bool = False):
     dev = torch.device("cuda")
     wd = w.to(dev)
     off = w.offset if offset is None else offset
@@ -52,12 +52,12 @@ def run_gpu(w, *, sampled: bool, residual: bool = False, stages: int = 0, plain:
             temp = wd.temperature
         o = dcd.dcd_score_rows(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta, q=q, temperature=temp,
                                seed=w.seed, offset=off, stages=stages, plain_loads=plain, out=out,
-                               workspace=workspace)
+                               workspace=workspace, distinct=distinct)
         dcd.dcd_tree_walk(w.B, w.N, w.V, o, o["workspace"])
     elif sampled:
         q = wd.q if wd.q is not None else torch.zeros_like(wd.z_exp, dtype=torch.float32)
         o = dcd.dcd_verify_sample(wd.z_exp, wd.z_ama, q, wd.tokens, wd.parents, wd.alpha, wd.temperature, w.seed, off,
-                                  wd.beta, residual=residual, out=out, workspace=workspace)
+                                  wd.beta, residual=residual, out=out, workspace=workspace, distinct=distinct)
     else:
         o = dcd.dcd_verify_greedy(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta, out=out,
                                   workspace=workspace)
