@@ -92,6 +92,7 @@ def _load():
             lib.dcd_oracle_verify.argtypes = [I32, I32, I64, ctypes.c_int, I64, P, P, P, P, P, P, P, P, I64,
                                               U64, U64, P, ctypes.c_int, ctypes.c_int, P, P, P, P, P, P]
             lib.dcd_oracle_max_threads.restype = ctypes.c_int
+            lib.dcd_oracle_row_diagnostics.argtypes = [I64, ctypes.c_int, P, P, P, ctypes.c_int32, P]
             _lib = lib
     return _lib
 
@@ -284,3 +285,17 @@ def verify_fused_workload(w, nthreads: int = 1, seqs=None) -> dict:
     return verify(B=len(sel), N=N, V=w.V, dtype="f64", z_exp=zp, z_ama=zq,
                   tokens=w.tokens.cpu()[sel], parents=w.parents.cpu()[sel], alpha=w.alpha.cpu()[sel],
                   beta=None, temperature=None, nthreads=nthreads, seq_ids=np.asarray(sel))
+
+
+def row_diagnostics(zp, zq, xstar: int, q=None, dtype: str = "f64") -> dict:
+    """Per-row diagnostics (see dcd_oracle_row_diagnostics): lse_p, lse_q, signal at x*, e_q, and
+    with the drafter's distribution q: e_e and kl_e_p."""
+    zp = _logits(zp, dtype)
+    zq = _logits(zq, dtype)
+    V = zp.shape[-1]
+    qq = None if q is None else np.ascontiguousarray(q, dtype=np.float32)
+    out = np.empty(6, dtype=np.float64)
+    rc = _load().dcd_oracle_row_diagnostics(V, DTYPE_CODE[dtype], _ptr(zp), _ptr(zq), _ptr(qq), int(xstar), _ptr(out))
+    if rc != 0:
+        raise ValueError(f"oracle row_diagnostics failed: {rc}")
+    return dict(zip(("lse_p", "lse_q", "signal", "e_q", "e_e", "kl_e_p"), out))

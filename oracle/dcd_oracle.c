@@ -606,3 +606,49 @@ int dcd_oracle_max_threads(void) {
   return 1;
 #endif
 }
+
+/* ---------------------------------------------------------------- per-row diagnostics */
+
+/*
+ * Diagnostics of one row (the quantities of the paper's signal--proposal-error diagnostic,
+ * Sec. 5.3, and of its alignment-gap estimator, App. E), in fp64 from the exact inputs:
+ *   lse_p, lse_q : log sum_x exp(z_p(x)), log sum_x exp(z_q(x)) (full vocabulary);
+ *   signal       : |log pi_p(x*) - log pi_q(x*)| at the given token x* (the CD argmax);
+ *   e_q          : E_{pi_q}[log pi_p - log pi_q];
+ *   e_e, kl_e_p  : with the drafter's distribution pi_e = q (q may be NULL): E_{pi_e}[log pi_p -
+ *                  log pi_q] and D_KL(pi_e || pi_p), with 0 log 0 = 0.
+ * out[6] = {lse_p, lse_q, signal, e_q, e_e, kl_e_p} (the last two NaN without q).
+ */
+int dcd_oracle_row_diagnostics(int64_t V, int dtype, const void* zp, const void* zq, const float* q, int32_t xstar,
+                               double* out) {
+  if (V <= 0 || !zp || !zq || !out || xstar < 0 || xstar >= V) return ORC_ERR_ARG;
+  double mp = -INFINITY, mq = -INFINITY;
+  for (int64_t x = 0; x < V; ++x) {
+    const double a = logit_at(zp, dtype, x), b = logit_at(zq, dtype, x);
+    if (a > mp) mp = a;
+    if (b > mq) mq = b;
+  }
+  double sp = 0.0, sq = 0.0;
+  for (int64_t x = 0; x < V; ++x) {
+    sp += exp(logit_at(zp, dtype, x) - mp);
+    sq += exp(logit_at(zq, dtype, x) - mq);
+  }
+  const double lse_p = mp + log(sp), lse_q = mq + log(sq);
+  double e_q = 0.0, e_e = 0.0, kl = 0.0;
+  for (int64_t x = 0; x < V; ++x) {
+    const double lp = logit_at(zp, dtype, x) - lse_p, lq = logit_at(zq, dtype, x) - lse_q;
+    e_q += exp(lq) * (lp - lq);
+    if (q) {
+      const double e = (double)q[x];
+      e_e += e * (lp - lq);
+      if (e > 0.0) kl += e * (log(e) - lp);
+    }
+  }
+  out[0] = lse_p;
+  out[1] = lse_q;
+  out[2] = fabs((logit_at(zp, dtype, xstar) - lse_p) - (logit_at(zq, dtype, xstar) - lse_q));
+  out[3] = e_q;
+  out[4] = q ? e_e : NAN;
+  out[5] = q ? kl : NAN;
+  return ORC_OK;
+}

@@ -617,3 +617,29 @@ def test_lossless_monte_carlo_full_verify_siblings_without_replacement():
     assert tv < 3.0 * np.sqrt(V / B)
     chi = stats.chisquare(counts[pi > 0], B * pi[pi > 0])
     assert chi.pvalue > 1e-4
+
+
+def test_row_diagnostics_closed_forms():
+    """The diagnostics against closed forms: lse against scipy's logsumexp; E_{pi_q}[log pi_p -
+    log pi_q] = -KL(pi_q || pi_p) and D_KL(pi_e || pi_p) from scipy's relative entropy; the signal
+    from the log-softmax difference at x*; E_{pi_e} with pi_e = pi_q equals E_{pi_q}; the KL of
+    pi_p from itself is zero."""
+    rng = np.random.default_rng(41)
+    V = 97
+    zp, zq = _rows(rng, V, scale=2.0)
+    lp, lq = special.log_softmax(zp), special.log_softmax(zq)
+    pe = special.softmax(zp + rng.standard_normal(V))
+    x = int(np.argmax(zp))
+    d = oracle.row_diagnostics(zp, zq, x, q=pe.astype(np.float32))
+    assert abs(d["lse_p"] - special.logsumexp(zp)) < 1e-12
+    assert abs(d["lse_q"] - special.logsumexp(zq)) < 1e-12
+    assert abs(d["signal"] - abs(lp[x] - lq[x])) < 1e-12
+    assert abs(d["e_q"] + special.rel_entr(np.exp(lq), np.exp(lp)).sum()) < 1e-12
+    pe32 = pe.astype(np.float32).astype(np.float64)
+    assert abs(d["kl_e_p"] - special.rel_entr(pe32, np.exp(lp)).sum()) < 1e-9
+    assert abs(d["e_e"] - (pe32 * (lp - lq)).sum()) < 1e-12
+    same = oracle.row_diagnostics(zp, zq, x, q=np.exp(lq).astype(np.float32))
+    assert abs(same["e_e"] - d["e_q"]) < 1e-6  # pi_e = pi_q (up to fp32 rounding of q)
+    self_kl = oracle.row_diagnostics(zp, zq, x, q=np.exp(lp).astype(np.float32))["kl_e_p"]
+    assert abs(self_kl) < 1e-6
+    assert np.isnan(oracle.row_diagnostics(zp, zq, x)["e_e"])
