@@ -10,12 +10,16 @@ Inputs are seeded synthetic data resident in HBM (1.97 GB, larger than the 129 M
 L2, so no flush is needed; about 1.05 GB of it is read per step); each step advances
 the Philox offset.
 
+`--workload diagnostics` times the per-row diagnostics pass (dcd_row_diagnostics: the signal
+at the CD argmax and the drafter-alignment terms over the same logits plus an fp32 q row per
+node, 1.97 GB read per step).
+
 `--workload fused` times the fused LM-head variant instead (dcd_verify_fused_lmhead:
 64 sequences x 60 nodes = 3840 rows, hidden states of 8192 and 2048, V = 128256,
 bf16, greedy): one step is both output projections on the tensor cores with the CD
 epilogue, the per-row combine and the tree walk.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload batched|fused]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload batched|fused|diagnostics]
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle on a
 bounded sample of the same workload instead.
@@ -41,6 +45,8 @@ if ROOT not in sys.path:
 WORKLOAD = "batched_B32_tree60_V128256_bf16_mixed"
 FUSED_WORKLOAD = "fused_lmhead_B64_tree60_V128256_Hexp8192_Hama2048_bf16_greedy"
 METRIC = "verified draft nodes/sec (CD verification step, 1 GPU)"
+DIAG_WORKLOAD = "diagnostics_B32_tree60_V128256_bf16_q_f32"
+DIAG_METRIC = "diagnosed rows/sec (per-row CD diagnostics, 1 GPU)"
 
 
 def _peaks():
@@ -62,18 +68,18 @@ def _bf16_peak():
         return 1700.0, "fallback sustained bf16"
 
 
-def _kernel_source_hash() -> str:
+def _kernel_source_hash(files=("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h")) -> str:
     h = hashlib.sha256()
-    for name in ("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h"):
+    for name in files:
         with open(os.path.join(ROOT, "paper_2608_12913_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def _profiled_traffic(kernel_hash: str):
-    """DRAM bytes per launch of the row kernel from the committed ncu summary, if it was taken
-    on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "score_rows_kernel_batched_B32_tree60_V128256.md")
+def _profiled_traffic(kernel_hash: str, summary: str = "score_rows_kernel_batched_B32_tree60_V128256.md"):
+    """DRAM bytes per launch of a kernel from its committed ncu summary, if it was taken on the
+    current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", summary)
     try:
         text = open(path).read()
     except OSError:
@@ -192,6 +198,8 @@ def run_reference(args):
         return 0
     import oracle
     from paper_2608_12913_gb300 import workloads
+    if args.workload == "diagnostics":
+        return run_reference_diagnostics(args, ws)
     w = workloads.make_config(3, B=2)  # sequences 0 (greedy) and 1 (sampled) of the batched workload
     threads = oracle.max_threads()
     for _ in range(args.warmup):
@@ -210,6 +218,43 @@ def run_reference(args):
         "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": threads, "kind": "oracle",
                          "sample": "2 of 32 sequences (120 of 1920 rows) per step"},
         "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def _diag_oracle_rows(w, rows, xstar):
+    """The oracle's diagnostics for the given rows of workload `w` (inputs as stored)."""
+    import oracle
+    R = w.B * w.N
+    zp = w.z_exp.reshape(R, w.V)
+    zq = w.z_ama.reshape(R, w.V)
+    q = w.q.reshape(R, w.V)
+    for g in rows:
+        oracle.row_diagnostics(zp[g].cpu(), zq[g].cpu(), int(xstar[g]), q=q[g].cpu().numpy(), dtype=w.dtype)
+
+
+def run_reference_diagnostics(args, world):
+    from paper_2608_12913_gb300 import workloads
+    w = workloads.make_config(3, B=2)
+    R = w.B * w.N
+    xstar = [(g * 7919) % w.V for g in range(R)]
+    for _ in range(args.warmup):
+        _diag_oracle_rows(w, range(R), xstar)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        _diag_oracle_rows(w, range(R), xstar)
+    dt = (time.perf_counter() - t0) / max(1, args.steps)
+    value = R / dt
+    line = {
+        "impl": "reference", "metric": DIAG_METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": DIAG_WORKLOAD, "sample": "sequences 0-1 of the batch (120 rows) per step",
+                   "V": w.V, "N": w.N},
+        "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                         "sample": "2 of 32 sequences (120 of 1920 rows) per step, one thread"},
+        "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
@@ -517,6 +562,140 @@ def run_fused(args):
     return 0
 
 
+def run_diagnostics(args):
+    """Per-row diagnostics (signal at the CD argmax, alignment terms) over the batched workload's
+    logits and q: a streaming pass bound by HBM; roofline in GB/s of the streaming kernel."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_12913_gb300 import dcd, workloads
+
+    world, rank, local = _dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch)
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    zp, zq, q = w.z_exp.reshape(R, V), w.z_ama.reshape(R, V), w.q.reshape(R, V)
+    stream = torch.cuda.current_stream()
+    o = dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, stream=stream)
+    xstar = o["cd_argmax"].reshape(-1).contiguous()  # the CD argmax of every node
+    ws = torch.empty(dcd.diagnostics_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
+    diag = torch.empty(R, 6, dtype=torch.float32, device=dev)
+    steps = args.steps
+
+    def step(evs=None):
+        dcd.dcd_row_diagnostics(zp, zq, B, N, q=q, xstar=xstar, out=diag, workspace=ws, stream=stream,
+                                pass_events=evs)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
+    t_soak = time.time()
+    while not args.no_soak and time.time() - t_soak < 1.0:
+        for _ in range(32):
+            step()
+        torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for e in evs:  # create the events outside the timed region
+        e[0].record(stream)
+        e[1].record(stream)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    start.record(stream)
+    for k in range(steps):
+        step(evs[k])
+    stop.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t_wall1 = time.time()
+    sampler.stop()
+    elapsed_ms = start.elapsed_time(stop)
+    pass_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+    if world > 1:
+        elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
+    if not torch.isfinite(diag).all():
+        raise RuntimeError("non-finite diagnostics on finite inputs")
+    ms_per_step = elapsed_ms / steps
+    value = job_value(world, R, ms_per_step)
+    alg = float(R * V * (2 * 2 + 4))  # both bf16 logit rows and the fp32 q row of every node
+    peak, peak_kind = _peaks()
+    achieved = alg / (pass_ms / 1e3) / 1e9
+    khash = _kernel_source_hash(("dcd_diag.cu", "dcd_device.cuh", "dcd_internal.h"))
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": _profiled_traffic(khash, "diag_partial_kernel_B32_tree60_V128256.md"),
+                "kernel": "diag_partial_kernel", "peak_source": f"{peak_kind} hbm_gbs",
+                "algorithmic_bytes_per_launch": alg, "pass_kernel_ms": pass_ms, "kernel_source_sha256_16": khash}
+
+    e2e = None
+    if not args.no_e2e:
+        host = {"zp": zp.cpu().pin_memory(), "zq": zq.cpu().pin_memory(), "q": q.cpu().pin_memory(),
+                "xstar": xstar.cpu().pin_memory()}
+        dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
+        res_host = torch.empty((R, 6), dtype=torch.float32).pin_memory()
+        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        d2h = res_host.numel() * 4
+        n_e2e = max(3, min(steps, 10))
+
+        def e2e_step():
+            for k in host:
+                dst[k].copy_(host[k], non_blocking=True)
+            r = dcd.dcd_row_diagnostics(dst["zp"], dst["zq"], B, N, q=dst["q"], xstar=dst["xstar"], out=diag,
+                                        workspace=ws, stream=stream)
+            res_host.copy_(r, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        a, b2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        b2.record(stream)
+        torch.cuda.synchronize()
+        e_ms = a.elapsed_time(b2) / n_e2e
+        if world > 1:
+            e_ms = max_over_ranks(e_ms, dist, dev)
+        e2e = {"value": job_value(world, R, e_ms), "unit": "rows/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
+        del dst, host
+
+    if rank == 0:
+        line = {
+            "metric": DIAG_METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": DIAG_WORKLOAD if B == 32 else f"{DIAG_WORKLOAD} (profiling case, B={B})",
+                       "B": B, "N": N, "V": V, "rows": R, "logits": "bf16", "q": "fp32, every row",
+                       "bytes_per_step": alg, "l2": "inputs (1.97 GB resident) larger than L2; no flush",
+                       "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
+            "roofline": roofline,
+            "clocks": sampler.summary(t_wall0, t_wall1),
+            "e2e": e2e,
+            "gpu_launches": 2 * steps,
+        }
+        if not args.no_cpu_baseline:
+            rows = range(min(R, 240))
+            xs = xstar.cpu().numpy()
+            t0 = time.perf_counter()
+            _diag_oracle_rows(w, rows, xs)
+            dt = time.perf_counter() - t0
+            line["cpu_baseline"] = {"value": len(rows) / dt, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                                    "sample": f"first {len(rows)} of {R} rows, one thread, {dt:.1f} s wall"}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -531,9 +710,9 @@ def main():
                     help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
     ap.add_argument("--distinct", action="store_true",
                     help="sampled rule for siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)")
-    ap.add_argument("--workload", choices=("batched", "fused"), default="batched",
+    ap.add_argument("--workload", choices=("batched", "fused", "diagnostics"), default="batched",
                     help="batched: the streaming step on materialised logits (the headline); fused: the "
-                         "fused LM-head variant")
+                         "fused LM-head variant; diagnostics: the per-row diagnostics pass")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -541,6 +720,8 @@ def main():
         return run_reference(args)
     if args.workload == "fused":
         return run_fused(args)
+    if args.workload == "diagnostics":
+        return run_diagnostics(args)
     return run_ours(args)
 
 

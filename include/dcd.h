@@ -269,6 +269,43 @@ int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_
                                void* gemm_start, void* gemm_stop);
 
 /*
+ * Per-row diagnostics of contrastive verification: the quantities behind the signal versus
+ * proposal-error analysis (Sec. 3.1) and the alignment-gap estimator (App. C).  For every row r
+ * of the B*N rows, with pi_p = softmax(z_exp[r]), pi_q = softmax(z_ama[r]) over the full
+ * vocabulary (no temperature, no plausibility mask) and e = q[r] (the drafter's distribution):
+ *   diag[r][0] = lse_p = log sum_x exp(z_exp[r][x])
+ *   diag[r][1] = lse_q = log sum_x exp(z_ama[r][x])
+ *   diag[r][2] = signal = |log pi_p(x*) - log pi_q(x*)| at x* = xstar[r] (the CD argmax, e.g.
+ *                the cd_argmax output of a verification call); NaN if xstar is NULL or
+ *                xstar[r] is outside [0, V)
+ *   diag[r][3] = E_{pi_q}[log pi_p - log pi_q]   (= -D_KL(pi_q || pi_p))
+ *   diag[r][4] = E_e[log pi_p - log pi_q]         (NaN if q is NULL)
+ *   diag[r][5] = D_KL(e || pi_p), 0 log 0 = 0     (NaN if q is NULL)
+ * The alignment gap of App. C is diag[4] - diag[3] averaged over the rows a caller selects.
+ *   shape : B, N, V, logits_dtype, ld_logits as for the verification calls; ld_q (>= V) when q
+ *       is given; flags must be 0.
+ *   z_exp, z_ama : [B*N, ld_logits] device logits; q : [B*N, ld_q] fp32 device probabilities or
+ *       NULL; xstar : int32 [B*N] device tokens or NULL; diag : fp32 [B*N, 6] device output.
+ *   workspace : device scratch of at least dcd_diagnostics_workspace_bytes(shape) bytes,
+ *       256-byte aligned (about 48 * B * N * ceil(V / 2048) bytes).
+ * Logits must be finite (non-finite inputs give NaN or inf results; no error word is kept).
+ * One pass over the inputs (fp32 accumulation) and a per-row combine, stream-ordered on
+ * `stream`.  Returns DCD_ERR_INVALID_ARG or DCD_ERR_WORKSPACE for bad arguments, DCD_ERR_CUDA
+ * if a launch fails.
+ */
+size_t dcd_diagnostics_workspace_bytes(const dcd_shape* shape);
+
+int dcd_row_diagnostics(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                        const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                        dcd_stream_t stream);
+
+/* dcd_row_diagnostics that also records two CUDA events (cudaEvent_t, or NULL) on `stream`
+ * immediately before and after the streaming pass (the per-row combine follows it). */
+int dcd_row_diagnostics_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                           const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                           dcd_stream_t stream, void* pass_start, void* pass_stop);
+
+/*
  * Synchronises `stream`, then copies the device error word of `workspace` (the OR of
  * the DCD_DEVERR_* bits raised by the last call that used it) into *bits.  Returns
  * DCD_OK when the word is zero, DCD_ERR_DEVICE_INPUT when it is not, DCD_ERR_CUDA if

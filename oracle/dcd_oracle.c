@@ -611,7 +611,7 @@ int dcd_oracle_max_threads(void) {
 
 /*
  * Diagnostics of one row (the quantities of the paper's signal--proposal-error diagnostic,
- * Sec. 5.3, and of its alignment-gap estimator, App. E), in fp64 from the exact inputs:
+ * Sec. 3.1, and of its alignment-gap estimator, App. C), in fp64 from the exact inputs:
  *   lse_p, lse_q : log sum_x exp(z_p(x)), log sum_x exp(z_q(x)) (full vocabulary);
  *   signal       : |log pi_p(x*) - log pi_q(x*)| at the given token x* (the CD argmax);
  *   e_q          : E_{pi_q}[log pi_p - log pi_q];

@@ -248,6 +248,46 @@ int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_
   return cuda_status(e);
 }
 
+size_t dcd_diagnostics_workspace_bytes(const dcd_shape* shape) {
+  if (!shape_ok(shape, false)) return 0;
+  const size_t b = dcd::diag_workspace_bytes(static_cast<int64_t>(shape->B) * shape->N, shape->V);
+  return b ? b : 256;
+}
+
+int dcd_row_diagnostics_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                           const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                           dcd_stream_t stream, void* pass_start, void* pass_stop) {
+  if (!shape_ok(shape, q != nullptr) || shape->flags != 0) return DCD_ERR_INVALID_ARG;
+  const int64_t R = static_cast<int64_t>(shape->B) * shape->N;
+  if (R > 0 && (!z_exp || !z_ama || !diag)) return DCD_ERR_INVALID_ARG;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 ||
+      workspace_bytes < dcd_diagnostics_workspace_bytes(shape))
+    return DCD_ERR_WORKSPACE;
+  dcd::DiagArgs d;
+  d.R = R;
+  d.V = shape->V;
+  d.ld = shape->ld_logits;
+  d.ldq = shape->ld_q;
+  d.dtype = shape->logits_dtype;
+  d.z_exp = z_exp;
+  d.z_ama = z_ama;
+  d.q = q;
+  d.xstar = xstar;
+  d.out = diag;
+  d.part = static_cast<dcd::DiagPart*>(workspace);
+  d.stream = stream;
+  d.start = pass_start;
+  d.stop = pass_stop;
+  return cuda_status(dcd::launch_diagnostics(d));
+}
+
+int dcd_row_diagnostics(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
+                        const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                        dcd_stream_t stream) {
+  return dcd_row_diagnostics_ex(shape, z_exp, z_ama, q, xstar, diag, workspace, workspace_bytes, stream, nullptr,
+                                nullptr);
+}
+
 int dcd_get_device_error(const void* workspace, dcd_stream_t stream, uint32_t* bits) {
   if (!workspace || !bits) return DCD_ERR_INVALID_ARG;
   uint32_t host = 0;

@@ -72,13 +72,17 @@ def load(build_if_missing: bool = True):
         lib.dcd_verify_fused_lmhead.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
         lib.dcd_verify_fused_lmhead_ex.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P,
                                                    P, P]
+        lib.dcd_diagnostics_workspace_bytes.argtypes = [SH]
+        lib.dcd_diagnostics_workspace_bytes.restype = SZ
+        lib.dcd_row_diagnostics.argtypes = [SH, P, P, P, P, P, P, SZ, P]
+        lib.dcd_row_diagnostics_ex.argtypes = [SH, P, P, P, P, P, P, SZ, P, P, P]
         lib.dcd_get_device_error.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
         lib.dcd_status_string.argtypes = [ctypes.c_int]
         lib.dcd_status_string.restype = ctypes.c_char_p
         lib.dcd_version.restype = ctypes.c_int
         for name in ("dcd_verify_greedy", "dcd_verify_sample", "dcd_score_rows", "dcd_score_rows_ex",
                      "dcd_tree_walk", "dcd_get_device_error", "dcd_verify_fused_lmhead",
-                     "dcd_verify_fused_lmhead_ex"):
+                     "dcd_verify_fused_lmhead_ex", "dcd_row_diagnostics", "dcd_row_diagnostics_ex"):
             getattr(lib, name).restype = I32
         _lib = lib
         return lib
@@ -342,6 +346,64 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
     _check(st, "dcd_verify_fused_lmhead")
     o["workspace"] = workspace
     return o
+
+
+DIAG_FIELDS = ("lse_p", "lse_q", "signal", "e_q", "e_e", "kl_e_p")
+
+
+def diagnostics_workspace_bytes(B: int, N: int, V: int) -> int:
+    sh = make_shape(B, N, V, DCD_BF16)
+    n = load().dcd_diagnostics_workspace_bytes(ctypes.byref(sh))
+    if n == 0:
+        raise ValueError("invalid shape")
+    return int(n)
+
+
+def dcd_row_diagnostics(z_exp, z_ama, B: int, N: int, *, q=None, xstar=None, out=None, workspace=None, stream=None,
+                        pass_events=None) -> torch.Tensor:
+    """Per-row diagnostics [B*N, 6] (columns DIAG_FIELDS): lse_p, lse_q, the signal
+    |log pi_p(x*) - log pi_q(x*)| at x* = xstar (the CD argmax), E_{pi_q}[log pi_p - log pi_q],
+    and with the drafter's distribution q: E_q[log pi_p - log pi_q] and D_KL(q || pi_p).
+
+    z_exp, z_ama: [B*N, ld] bf16 or fp32 logits (row stride = their stride); q: [B*N, ldq] fp32
+    or None; xstar: int32 [B*N] or [B, N], or None.  `pass_events` = (start, stop) torch.cuda.Event
+    pair recorded around the streaming pass.
+    """
+    _require(z_exp, "z_exp")
+    dev = z_exp.device
+    _require(z_ama, "z_ama", z_exp.dtype, dev, tuple(z_exp.shape))
+    if z_exp.dim() != 2 or z_exp.stride(1) != 1 or z_ama.stride() != z_exp.stride():
+        raise ValueError("z_exp / z_ama must be 2-D with unit column stride and equal strides")
+    R, V = z_exp.shape
+    if R != B * N:
+        raise ValueError(f"z_exp has {R} rows, expected B*N = {B * N}")
+    ldq = None
+    if q is not None:
+        _require(q, "q", torch.float32, dev)
+        if q.dim() != 2 or q.shape[0] != R or q.shape[1] != V or q.stride(1) != 1:
+            raise ValueError("q must be [B*N, V] with unit column stride")
+        ldq = q.stride(0)
+    if xstar is not None:
+        _require(xstar, "xstar", torch.int32, dev)
+        if xstar.numel() != R or not xstar.is_contiguous():
+            raise ValueError("xstar must be a contiguous int32 tensor of B*N tokens")
+    sh = make_shape(B, N, V, _logits_dtype(z_exp), ld=z_exp.stride(0), ldq=ldq)
+    if workspace is None:
+        workspace = torch.empty(diagnostics_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
+    if out is None:
+        out = torch.empty(R, 6, dtype=torch.float32, device=dev)
+    else:
+        _require(out, "out", torch.float32, dev, (R, 6))
+    ev0 = ev1 = None
+    if pass_events is not None:
+        for e in pass_events:
+            if not e.cuda_event:
+                e.record()
+        ev0, ev1 = (ctypes.c_void_p(e.cuda_event) for e in pass_events)
+    st = load().dcd_row_diagnostics_ex(ctypes.byref(sh), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(xstar), _ptr(out),
+                                       _ptr(workspace), workspace.numel(), _stream(stream), ev0, ev1)
+    _check(st, "dcd_row_diagnostics")
+    return out
 
 
 def dcd_get_device_error(workspace: torch.Tensor, stream=None) -> int:

@@ -139,3 +139,25 @@ def test_fused_workspace_and_host_checks(lib):
     assert lib.dcd_verify_fused_lmhead(ctypes.byref(sh), *args, ws, 64, None) == -7
     empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
     assert lib.dcd_verify_fused_lmhead(ctypes.byref(empty), *args, ws, 1 << 24, None) == 0
+
+
+def test_diagnostics_workspace_and_host_checks(lib):
+    sh = dcd.make_shape(32, 60, 128256, dcd.DCD_BF16)
+    n = lib.dcd_diagnostics_workspace_bytes(ctypes.byref(sh))
+    assert n == (1920 * ((128256 + 2047) // 2048) * 48 + 255) // 256 * 256
+    bad = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, ld=50)
+    assert lib.dcd_diagnostics_workspace_bytes(ctypes.byref(bad)) == 0
+    P = _fake(0x10000)
+    ws = _fake(0x100000)
+    sh = dcd.make_shape(2, 4, 100, dcd.DCD_BF16)
+    # null logits or output, sibling flags, q with a short stride, bad workspace: rejected before launch
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), None, P, None, None, P, ws, 1 << 20, None) == -1
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, None, ws, 1 << 20, None) == -1
+    flagged = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, flags=dcd.DCD_SIBLINGS_DISTINCT)
+    assert lib.dcd_row_diagnostics(ctypes.byref(flagged), P, P, None, None, P, ws, 1 << 20, None) == -1
+    short_q = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, ldq=99)
+    assert lib.dcd_row_diagnostics(ctypes.byref(short_q), P, P, P, None, P, ws, 1 << 20, None) == -1
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, P, _fake(0x100010), 1 << 20, None) == -7
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, P, ws, 16, None) == -7
+    empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
+    assert lib.dcd_row_diagnostics(ctypes.byref(empty), P, P, None, None, P, ws, 1 << 20, None) == 0
