@@ -629,7 +629,7 @@ def run_diagnostics(args):
     alg = float(R * V * (2 * 2 + 4))  # both bf16 logit rows and the fp32 q row of every node
     peak, peak_kind = _peaks()
     achieved = alg / (pass_ms / 1e3) / 1e9
-    khash = _kernel_source_hash(("dcd_diag.cu", "dcd_device.cuh", "dcd_internal.h"))
+    khash = _kernel_source_hash(("dcd_diag.cu", "dcd_diag.h", "dcd_device.cuh"))
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": _profiled_traffic(khash, "diag_partial_kernel_B32_tree60_V128256.md"),
                 "kernel": "diag_partial_kernel", "peak_source": f"{peak_kind} hbm_gbs",

@@ -7,6 +7,7 @@
 #include <climits>
 
 #include "dcd.h"
+#include "dcd_diag.h"
 #include "dcd_internal.h"
 
 namespace {

@@ -22,6 +22,7 @@
 
 #include "dcd.h"
 #include "dcd_device.cuh"
+#include "dcd_diag.h"
 #include "dcd_internal.h"
 
 namespace dcd {

@@ -176,34 +176,4 @@ struct RowGeometry {
 };
 RowGeometry row_geometry(const ScoreArgs& a);
 
-// ---- per-row diagnostics (dcd_diag.cu)
-// Statistics of one chunk of one row's vocabulary (see dcd_diag.cu for their definitions).
-struct alignas(16) DiagPart {
-  float mp, sp, mq, sq, tq, a, e1, ez, h, pad[3];
-};
-constexpr int kDiagMinChunk = 2048;   // tokens per CTA of the streaming pass: at least ...
-constexpr int kDiagMaxChunk = 16384;  // ... and at most
-// Tokens per chunk for R rows of V tokens on a GPU with `sms` SMs (a multiple of kDiagMinChunk).
-int diag_chunk(int64_t R, int64_t V, int sms);
-inline size_t diag_workspace_bytes(int64_t R, int64_t V) {
-  const size_t raw = static_cast<size_t>(R) * static_cast<size_t>((V + kDiagMinChunk - 1) / kDiagMinChunk) *
-                     sizeof(DiagPart);
-  return (raw + 255) & ~static_cast<size_t>(255);
-}
-
-struct DiagArgs {
-  int64_t R, V, ld, ldq;
-  int dtype;
-  const void* z_exp;
-  const void* z_ama;
-  const float* q;        // may be null
-  const int32_t* xstar;  // may be null
-  float* out;            // [R, 6]
-  DiagPart* part;        // workspace
-  cudaStream_t stream;
-  void* start;  // optional cudaEvent_t pair around the streaming pass (timing)
-  void* stop;
-};
-cudaError_t launch_diagnostics(const DiagArgs& d);
-
 }  // namespace dcd
