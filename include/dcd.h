@@ -137,6 +137,10 @@ size_t dcd_workspace_bytes(const dcd_shape* shape);
  *   accept_len [B], accept_path [B, N], bonus [B] : int32 outputs.
  *   cd_logprob [B, N], cd_argmax [B, N], cd_lse [B, N] : optional outputs (NULL skips).
  *   workspace : device scratch of at least dcd_workspace_bytes(shape), 256-byte aligned.
+ * A small call (B*N <= 512 rows and N <= 256: chains and small trees of single-request
+ * decoding) runs as one kernel after a memset of the workspace counters; larger calls run the
+ * streaming kernel and the tree walk (dcd_score_rows + dcd_tree_walk).  Both give the same
+ * accepted paths; the scores differ only by the order of fp32 summation.
  */
 int dcd_verify_greedy(const dcd_shape* shape, const void* z_exp, const void* z_ama, const int32_t* tokens,
                       const int32_t* parents, const float* alpha, const float* beta, int32_t* accept_len,

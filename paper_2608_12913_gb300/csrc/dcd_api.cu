@@ -9,6 +9,7 @@
 #include "dcd.h"
 #include "dcd_diag.h"
 #include "dcd_internal.h"
+#include "dcd_small.h"
 
 namespace {
 
@@ -163,6 +164,19 @@ int dcd_verify_greedy(const dcd_shape* shape, const void* z_exp, const void* z_a
                       void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
   if (!shape_ok(shape, false)) return DCD_ERR_INVALID_ARG;
   if (shape->B > 0 && (!accept_len || !accept_path || !bonus)) return DCD_ERR_INVALID_ARG;
+  if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
+  if (shape->B > 0 && shape->N <= dcd::kSmallMaxNodes &&
+      static_cast<int64_t>(shape->B) * shape->N <= dcd::kSmallMaxRows) {
+    // a small call: rows and tree walk in one launch
+    if (!z_exp || !z_ama || !tokens || !parents || !alpha) return DCD_ERR_INVALID_ARG;
+    const int ws = check_workspace(shape, workspace, workspace_bytes);
+    if (ws != DCD_OK) return ws;
+    const dcd::ScoreArgs a = make_args(shape, z_exp, z_ama, nullptr, tokens, parents, alpha, beta, nullptr, 0, 0,
+                                       cd_logprob, cd_argmax, cd_lse, workspace);
+    if (dcd::greedy_small_ok(a))
+      return cuda_status(dcd::launch_greedy_small(a, accept_len, accept_path, bonus,
+                                                  reinterpret_cast<cudaStream_t>(stream)));
+  }
   int rc = dcd_score_rows(shape, z_exp, z_ama, nullptr, tokens, parents, alpha, beta, nullptr, 0, 0, cd_logprob,
                           cd_argmax, cd_lse, workspace, workspace_bytes, stream);
   if (rc != DCD_OK) return rc;
