@@ -442,19 +442,21 @@ def run_fused(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = workloads.make_fused_torch(device=dev, seed=4 + rank)
+    w = workloads.make_fused_torch(device=dev, seed=4 + rank, beta=args.beta)
     B, N, V = w.B, w.N, w.V
     R = B * N
     H_exp, H_ama = w.h_exp.shape[1], w.h_ama.shape[1]
-    flop = 2.0 * R * V * (H_exp + H_ama)
+    beta = w.beta if args.beta > 0 else None
+    # with a plausibility mask the expert's GEMM runs twice (a max sweep, then the masked sweep)
+    flop = 2.0 * R * V * (H_exp + H_ama + (H_exp if beta is not None else 0))
     out = dcd.alloc_outputs(B, N, dev)
     ws = torch.empty(dcd.fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
     steps = args.steps
 
     def step(evs=None):
-        dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha, out=out,
-                                    workspace=ws, stream=stream, gemm_events=evs)
+        dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha, beta,
+                                    out=out, workspace=ws, stream=stream, gemm_events=evs)
 
     for _ in range(args.warmup):
         step()
@@ -496,7 +498,9 @@ def run_fused(args):
     achieved = flop / (gemm_ms / 1e3) / 1e12
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": None, "kernel": "fused_lmhead_kernel", "peak_source": peak_src,
-                "algorithmic_flops_per_launch": flop, "gemm_kernel_ms": gemm_ms}
+                "algorithmic_flops_per_launch": flop, "gemm_kernel_ms": gemm_ms,
+                "flops_counted": "both LM-head GEMMs" + ("; with beta the expert's twice (max sweep, then masked)"
+                                                           if beta is not None else "")}
 
     # end to end: the step's hidden states and tree come from pinned host memory (the weights
     # are the models' resident parameters), the results go back
@@ -514,7 +518,7 @@ def run_fused(args):
             for k in host:
                 dst[k].copy_(host[k], non_blocking=True)
             o = dcd.dcd_verify_fused_lmhead(dst["h_exp"], w.w_exp, dst["h_ama"], w.w_ama, dst["tokens"],
-                                            dst["parents"], dst["alpha"], out=out, workspace=ws, stream=stream)
+                                            dst["parents"], dst["alpha"], beta, out=out, workspace=ws, stream=stream)
             for k in res_host:
                 res_host[k].copy_(o[k], non_blocking=True)
 
@@ -537,14 +541,16 @@ def run_fused(args):
             "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": FUSED_WORKLOAD, "B": B, "N": N, "V": V, "rows": R, "H_exp": H_exp,
-                       "H_ama": H_ama, "flop_per_step": flop,
+            "config": {"workload": FUSED_WORKLOAD + (f" beta={args.beta:g}" if beta is not None else ""),
+                       "B": B, "N": N, "V": V, "rows": R, "H_exp": H_exp,
+                       "H_ama": H_ama, "flop_per_step": flop, "beta": args.beta,
                        "l2": "weights (2.6 GB) larger than L2; no flush",
                        "parallelism": f"replicas x{world} (sequence batches, no collective in the path)"},
             "roofline": roofline,
             "clocks": sampler.summary(t_wall0, t_wall1),
             "e2e": e2e,
-            "gpu_launches": 4 * steps,
+            # children, GEMM, combine and walk kernels; with a mask also the max sweep and the row max
+            "gpu_launches": (6 if beta is not None else 4) * steps,
         }
         if not args.no_cpu_baseline:
             import oracle
@@ -710,6 +716,8 @@ def main():
                     help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
     ap.add_argument("--distinct", action="store_true",
                     help="sampled rule for siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)")
+    ap.add_argument("--beta", type=float, default=0.0,
+                    help="fused workload: plausibility threshold of every sequence (0: no mask, one sweep)")
     ap.add_argument("--workload", choices=("batched", "fused", "diagnostics"), default="batched",
                     help="batched: the streaming step on materialised logits (the headline); fused: the "
                          "fused LM-head variant; diagnostics: the per-row diagnostics pass")

@@ -245,7 +245,7 @@ int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_a
  *   H_exp, H_ama : hidden sizes, >= 1 and multiples of 8 (16-byte rows); every matrix base
  *       16-byte aligned.
  *   tokens, parents, alpha, accept_len, accept_path, bonus, cd_logprob, cd_argmax,
- *       cd_lse : as for dcd_verify_greedy (beta is 0).  A node may have at most 8 children
+ *       cd_lse : as for dcd_verify_greedy (beta is 0 here; dcd_verify_fused_lmhead_ex takes it).  A node may have at most 8 children
  *       (else its sequence reports DCD_DEVERR_UNSUPPORTED and accept_len = 0).
  *   workspace : device scratch of at least dcd_fused_workspace_bytes(shape), 256-byte
  *       aligned; about 16 * B * N * ceil(V / 256) bytes.
@@ -261,16 +261,24 @@ int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H
                             float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream);
 
 /*
- * dcd_verify_fused_lmhead that also records two CUDA events (cudaEvent_t handles, or NULL)
- * on `stream` immediately before and after the tensor-core kernel, for timing that kernel
- * alone.  Results equal dcd_verify_fused_lmhead.
+ * dcd_verify_fused_lmhead with the plausibility mask and timing events.
+ *   beta : fp32 [B] device plausibility thresholds in [0, 1] (Sec. 2.1), or NULL for beta = 0.
+ *       With beta, the tensor-core kernel runs twice: a first sweep over the expert's hidden
+ *       size only finds each row's max z_p (the same MMAs in the same order as the second sweep,
+ *       so both see bit-identical logits), and the second scores only the tokens with
+ *       z_p - max z_p >= log beta.  That costs the expert GEMM once more (about 1.8x the FLOPs
+ *       of a call without beta at H_exp = 4 H_ama); a sequence with beta = 0 is not masked.
+ *   gemm_start, gemm_stop : two CUDA events (cudaEvent_t handles, or NULL) recorded on
+ *       `stream` immediately before the first and after the last tensor-core sweep, for timing
+ *       them alone.
+ * With beta NULL the results equal dcd_verify_fused_lmhead.
  */
 int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_t H_exp, const void* w_exp,
                                const void* h_ama, int32_t H_ama, const void* w_ama, const int32_t* tokens,
-                               const int32_t* parents, const float* alpha, int32_t* accept_len,
-                               int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
-                               float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
-                               void* gemm_start, void* gemm_stop);
+                               const int32_t* parents, const float* alpha, const float* beta,
+                               int32_t* accept_len, int32_t* accept_path, int32_t* bonus, float* cd_logprob,
+                               int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
+                               dcd_stream_t stream, void* gemm_start, void* gemm_stop);
 
 /*
  * Per-row diagnostics of contrastive verification: the quantities behind the signal versus

@@ -274,7 +274,8 @@ def fused_logits(h, w, chunk: int = 8192) -> np.ndarray:
 
 
 def verify_fused_workload(w, nthreads: int = 1, seqs=None) -> dict:
-    """``verify`` of a fused LM-head workload: logits from ``fused_logits`` (fp64), greedy, beta = 0."""
+    """``verify`` of a fused LM-head workload: logits from ``fused_logits`` (fp64), greedy, with the
+    workload's beta (the plausibility mask) when any is nonzero."""
     B, N = w.B, w.N
     sel = list(range(B)) if seqs is None else list(seqs)
     rows = np.concatenate([np.arange(b * N, (b + 1) * N) for b in sel])
@@ -282,9 +283,12 @@ def verify_fused_workload(w, nthreads: int = 1, seqs=None) -> dict:
     ridx = torch.as_tensor(rows, device=w.h_exp.device)
     zp = fused_logits(w.h_exp[ridx], w.w_exp)
     zq = fused_logits(w.h_ama[ridx], w.w_ama)
+    beta = None
+    if getattr(w, "beta", None) is not None and bool((w.beta != 0).any()):
+        beta = w.beta.cpu()[sel]
     return verify(B=len(sel), N=N, V=w.V, dtype="f64", z_exp=zp, z_ama=zq,
                   tokens=w.tokens.cpu()[sel], parents=w.parents.cpu()[sel], alpha=w.alpha.cpu()[sel],
-                  beta=None, temperature=None, nthreads=nthreads, seq_ids=np.asarray(sel))
+                  beta=beta, temperature=None, nthreads=nthreads, seq_ids=np.asarray(sel))
 
 
 def row_diagnostics(zp, zq, xstar: int, q=None, dtype: str = "f64") -> dict:

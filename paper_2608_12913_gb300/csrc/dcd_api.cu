@@ -8,6 +8,7 @@
 
 #include "dcd.h"
 #include "dcd_diag.h"
+#include "dcd_fused.h"
 #include "dcd_internal.h"
 #include "dcd_small.h"
 
@@ -215,16 +216,16 @@ int dcd_verify_fused_lmhead(const dcd_shape* shape, const void* h_exp, int32_t H
                             int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
                             float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
   return dcd_verify_fused_lmhead_ex(shape, h_exp, H_exp, w_exp, h_ama, H_ama, w_ama, tokens, parents, alpha,
-                                    accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse, workspace,
-                                    workspace_bytes, stream, nullptr, nullptr);
+                                    nullptr, accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse,
+                                    workspace, workspace_bytes, stream, nullptr, nullptr);
 }
 
 int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_t H_exp, const void* w_exp,
                                const void* h_ama, int32_t H_ama, const void* w_ama, const int32_t* tokens,
-                               const int32_t* parents, const float* alpha, int32_t* accept_len,
-                               int32_t* accept_path, int32_t* bonus, float* cd_logprob, int32_t* cd_argmax,
-                               float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
-                               void* gemm_start, void* gemm_stop) {
+                               const int32_t* parents, const float* alpha, const float* beta,
+                               int32_t* accept_len, int32_t* accept_path, int32_t* bonus, float* cd_logprob,
+                               int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
+                               dcd_stream_t stream, void* gemm_start, void* gemm_stop) {
   const size_t need = dcd_fused_workspace_bytes(shape);
   if (need == 0) return DCD_ERR_INVALID_ARG;
   if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
@@ -248,6 +249,7 @@ int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_
   f.tokens = tokens;
   f.parents = parents;
   f.alpha = alpha;
+  f.beta = beta;
   f.accept_len = accept_len;
   f.accept_path = accept_path;
   f.bonus = bonus;

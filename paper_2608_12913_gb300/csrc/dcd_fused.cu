@@ -12,11 +12,14 @@
 //              the producer and each finished tile to the epilogue;
 //   warps 2-5 -- epilogue: each thread owns one row of the tile (one TMEM lane), reads its 2 x
 //              256 accumulators, forms the scaled CD score u = log2(e) ((1 + alpha) z_p -
-//              alpha z_q) (Eq. 1 with beta = 0 and T = 1; the log-softmax shifts cancel), and
+//              alpha z_q) (Eq. 1 at T = 1; the log-softmax shifts cancel) on P_beta, and
 //              keeps the tile's max of u, sum of 2^(u - max) and argmax; the score at each child
 //              token that falls in the tile is kept too.  Tiles are visited vocabulary-block
 //              major, so the 30 row tiles that share a block of W read it while it is in L2, and
 //              h (read once per vocabulary block) is kept in L2 with an evict-last policy.
+//   With a plausibility mask (beta > 0, Sec. 2.1) the kernel runs twice: a first sweep over the
+//   expert's K blocks only keeps each tile's max of z_p, fused_rowmax_kernel reduces them per
+//   row, and the full sweep then scores only tokens with z_p - max z_p >= log beta.
 // fused_children_kernel: per row, the children of its node (ascending id, at most 8) and the
 //   row's input checks.
 // fused_combine_kernel: one warp per row merges the tiles' statistics in order, writes
@@ -34,6 +37,7 @@
 
 #include "dcd.h"
 #include "dcd_device.cuh"
+#include "dcd_fused.h"
 #include "dcd_internal.h"
 #include "dcd_tc.cuh"
 
@@ -58,7 +62,10 @@ constexpr float kLn2f = 0.69314718055994531f;
 struct FusedParams {
   CUtensorMap tm_hp, tm_wp, tm_hq, tm_wq;
   int32_t R, V, N, nkp, nkq, nmt, nvt, ntiles;
+  int32_t sweep;           // 0: both models, the tile statistics of u; 1: the expert only, tile max of z_p
   const float* alpha;
+  const float* beta;       // [B] or null (no plausibility mask)
+  const float* zmax;       // [R] row max of z_p (sweep 0 with beta)
   const int32_t* kid_tok;  // [R][kMaxKids], -1 past the last child
   float* kid_u;            // [R][kMaxKids] scaled score at each child's token
   float4* part;            // [R][nvt] tile statistics {max u, sum 2^(u - max), argmax, -}
@@ -78,7 +85,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drained + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nk = P.nkp + P.nkq;
+  const int nk = P.sweep == 1 ? P.nkp : P.nkp + P.nkq;  // the max sweep runs the expert's K blocks only
   // A bounded wait that gives up records the error and makes every role of the CTA leave its
   // loop, so a failure costs one wait limit, not one per remaining stage.
   auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) -> bool {
@@ -176,14 +183,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
       const int i = tile % P.nmt, j = tile / P.nmt;
       const int r = i * kBM + quarter * 32 + lane;
       const bool valid = r < P.R;
-      float c1k = 0.f, ak = 0.f;
+      float c1k = 0.f, ak = 0.f, Mp = 0.f, logb = -INFINITY;
       int kt[kMaxKids];
 #pragma unroll
       for (int k = 0; k < kMaxKids; ++k) kt[k] = -1;
-      if (valid) {
+      if (valid && P.sweep == 0) {
         const float alpha = P.alpha[r / P.N];
         c1k = (1.f + alpha) * kLog2e;
         ak = alpha * kLog2e;
+        if (P.beta) {
+          const float be = P.beta[r / P.N];
+          if (be > 0.f) {  // P_beta = {x : z_p(x) - max z_p >= log beta}
+            logb = logf(be);
+            Mp = P.zmax[r];
+          }
+        }
         const int4 k0 = reinterpret_cast<const int4*>(P.kid_tok)[2 * r];
         const int4 k1 = reinterpret_cast<const int4*>(P.kid_tok)[2 * r + 1];
         kt[0] = k0.x; kt[1] = k0.y; kt[2] = k0.z; kt[3] = k0.w;
@@ -199,6 +213,27 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
       }
       tc::fence_after_sync();
       const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      if (P.sweep == 1) {
+        // the max sweep: this tile's max of z_p over the vocabulary
+        float mz = -INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < kBN / 64; ++c) {
+          float za[32], zb[32];
+          tc::tmem_ld32x2(trow + c * 64, trow + c * 64 + 32, za, zb);
+          const int col0 = j * kBN + c * 64;
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            if (col0 + e < P.V) mz = fmaxf(mz, za[e]);
+            if (col0 + 32 + e < P.V) mz = fmaxf(mz, zb[e]);
+          }
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty);
+        if (valid) __stcs(&P.part[static_cast<int64_t>(r) * P.nvt + j], make_float4(mz, 0.f, 0.f, 0.f));
+        continue;
+      }
+      const bool masked = logb > -INFINITY;
       float m = -INFINITY, ssum = 0.f;
       int arg = INT_MAX;
 #pragma unroll 1
@@ -210,7 +245,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
         float cm = -INFINITY;
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
-          u[e] = (col0 + e < P.V) ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
+          u[e] = (col0 + e < P.V && (!masked || zp[e] - Mp >= logb)) ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
           cm = fmaxf(cm, u[e]);
         }
         if (cm > m) {
@@ -257,7 +292,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
 // Per row: the children of its node in ascending id (at most kMaxKids) and the row's checks.
 __global__ void fused_children_kernel(int32_t B, int32_t N, int32_t V, const int32_t* __restrict__ tokens,
                                       const int32_t* __restrict__ parents, const float* __restrict__ alpha,
-                                      int32_t* kid_node, int32_t* kid_tok, uint32_t* row_status) {
+                                      const float* __restrict__ beta, int32_t* kid_node, int32_t* kid_tok,
+                                      uint32_t* row_status) {
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= B * N) return;
   const int b = r / N, n = r % N;
@@ -269,6 +305,7 @@ __global__ void fused_children_kernel(int32_t B, int32_t N, int32_t V, const int
   if (n > 0 && (tok[n] < 0 || tok[n] >= V)) st |= DCD_DEVERR_BAD_TOKEN;
   const float a = alpha[b];
   if (!(a >= 0.f && a <= 3.0e38f)) st |= DCD_DEVERR_BAD_PARAM;
+  if (beta && !(beta[b] >= 0.f && beta[b] <= 1.f)) st |= DCD_DEVERR_BAD_PARAM;
   int count = 0;
   for (int c = n + 1; c < N; ++c) {
     if (par[c] != n) continue;
@@ -284,6 +321,17 @@ __global__ void fused_children_kernel(int32_t B, int32_t N, int32_t V, const int
     kid_tok[r * kMaxKids + k] = -1;
   }
   row_status[r] = st;
+}
+
+// One warp per row: the row's max of z_p over its tiles' maxima (the max sweep's result).
+__global__ void fused_rowmax_kernel(int32_t R, int32_t nvt, const float4* __restrict__ part, float* zmax) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (r >= R) return;
+  float m = -INFINITY;
+  for (int j = lane; j < nvt; j += 32) m = fmaxf(m, part[static_cast<int64_t>(r) * nvt + j].x);
+  m = warp_max(m);
+  if (lane == 0) zmax[r] = m;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -401,6 +449,8 @@ FusedLayout fused_layout(int64_t rows, int64_t V) {
   off += static_cast<size_t>(rows) * sizeof(RowRecord);
   l.part = off;
   off += static_cast<size_t>(rows) * static_cast<size_t>(nvt) * 16;
+  l.zmax = off;
+  off += (static_cast<size_t>(rows) * 4 + 15) & ~static_cast<size_t>(15);
   l.total = (off + 255) & ~static_cast<size_t>(255);
   return l;
 }
@@ -418,6 +468,7 @@ cudaError_t launch_fused(const FusedArgs& f, cudaStream_t stream, int* status) {
   uint32_t* row_status = reinterpret_cast<uint32_t*>(ws + l.row_status);
   RowRecord* rec = reinterpret_cast<RowRecord*>(ws + l.rec);
   float4* part = reinterpret_cast<float4*>(ws + l.part);
+  float* zmax = reinterpret_cast<float*>(ws + l.zmax);
 
   FusedParams P;
   if (!make_map(&P.tm_hp, f.h_exp, R, f.H_exp, kBM) || !make_map(&P.tm_wp, f.w_exp, f.V, f.H_exp, kBN) ||
@@ -433,7 +484,10 @@ cudaError_t launch_fused(const FusedArgs& f, cudaStream_t stream, int* status) {
   P.nmt = static_cast<int32_t>((R + kBM - 1) / kBM);
   P.nvt = static_cast<int32_t>((f.V + kBN - 1) / kBN);
   P.ntiles = P.nmt * P.nvt;
+  P.sweep = 0;
   P.alpha = f.alpha;
+  P.beta = f.beta;
+  P.zmax = zmax;
   P.kid_tok = kid_tok;
   P.kid_u = kid_u;
   P.part = part;
@@ -442,7 +496,7 @@ cudaError_t launch_fused(const FusedArgs& f, cudaStream_t stream, int* status) {
   cudaError_t e = cudaMemsetAsync(hdr, 0, kWorkspaceHeader, stream);
   if (e != cudaSuccess) return e;
   fused_children_kernel<<<static_cast<unsigned>((R + 127) / 128), 128, 0, stream>>>(
-      f.B, f.N, static_cast<int32_t>(f.V), f.tokens, f.parents, f.alpha, kid_node, kid_tok, row_status);
+      f.B, f.N, static_cast<int32_t>(f.V), f.tokens, f.parents, f.alpha, f.beta, kid_node, kid_tok, row_status);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
@@ -458,6 +512,18 @@ cudaError_t launch_fused(const FusedArgs& f, cudaStream_t stream, int* status) {
   if (grid > P.ntiles) grid = P.ntiles;
   if (f.gemm_start) {
     e = cudaEventRecord(f.gemm_start, stream);
+    if (e != cudaSuccess) return e;
+  }
+  if (f.beta) {
+    // with a plausibility mask: first the expert's logits alone for each row's max of z_p (the
+    // same MMAs in the same order as below, so the second sweep sees bit-identical z_p)
+    FusedParams P1 = P;
+    P1.sweep = 1;
+    fused_lmhead_kernel<<<grid, kGemmThreads, kGemmSmem, stream>>>(P1);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    fused_rowmax_kernel<<<static_cast<unsigned>((R + 7) / 8), 256, 0, stream>>>(P.R, P.nvt, part, zmax);
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
   fused_lmhead_kernel<<<grid, kGemmThreads, kGemmSmem, stream>>>(P);

@@ -133,39 +133,6 @@ cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_
 cudaError_t launch_terminal_residual(const ScoreArgs& a, const int32_t* accept_len, const int32_t* accept_path,
                                      const int32_t* bonus, float* residual, cudaStream_t stream);
 
-// ---- the greedy step fused with the two LM heads (dcd_fused.cu)
-struct FusedArgs {
-  int32_t B, N;
-  int64_t V;
-  int32_t H_exp, H_ama;
-  const void* h_exp;  // bf16 [B*N, H_exp]
-  const void* w_exp;  // bf16 [V, H_exp]
-  const void* h_ama;  // bf16 [B*N, H_ama]
-  const void* w_ama;  // bf16 [V, H_ama]
-  const int32_t* tokens;
-  const int32_t* parents;
-  const float* alpha;
-  int32_t* accept_len;
-  int32_t* accept_path;
-  int32_t* bonus;
-  float* cd_logprob;
-  int32_t* cd_argmax;
-  float* cd_lse;
-  void* workspace;
-  cudaEvent_t gemm_start, gemm_stop;  // optional: recorded around the GEMM launch (timing)
-};
-
-// Workspace of the fused step: [WsHeader][child nodes][child tokens][child scores][row status]
-// [RowRecord x R][tile statistics x R x ceil(V / 256)] (byte offsets).
-struct FusedLayout {
-  size_t kid_node, kid_tok, kid_u, row_status, rec, part, total;
-};
-FusedLayout fused_layout(int64_t rows, int64_t V);
-
-// Launches the fused step; *status is set to a DCD_ERR_* code for requests the launch cannot
-// describe (tensor maps), with cudaSuccess returned.
-cudaError_t launch_fused(const FusedArgs& f, cudaStream_t stream, int* status);
-
 // Launch geometry the row kernel would use for a call (exposed for diagnostics).
 struct RowGeometry {
   int stages;        // ring depth per CTA

@@ -70,8 +70,8 @@ def load(build_if_missing: bool = True):
         lib.dcd_fused_workspace_bytes.argtypes = [SH]
         lib.dcd_fused_workspace_bytes.restype = SZ
         lib.dcd_verify_fused_lmhead.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
-        lib.dcd_verify_fused_lmhead_ex.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P,
-                                                   P, P]
+        lib.dcd_verify_fused_lmhead_ex.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, P, SZ,
+                                                   P, P, P]
         lib.dcd_diagnostics_workspace_bytes.argtypes = [SH]
         lib.dcd_diagnostics_workspace_bytes.restype = SZ
         lib.dcd_row_diagnostics.argtypes = [SH, P, P, P, P, P, P, SZ, P]
@@ -306,13 +306,14 @@ def fused_workspace_bytes(B: int, N: int, V: int) -> int:
     return int(n)
 
 
-def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, *, out=None, workspace=None,
-                            stream=None, gemm_events=None) -> dict:
+def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, beta=None, *, out=None,
+                            workspace=None, stream=None, gemm_events=None) -> dict:
     """Greedy CD verification fused with the two LM heads (logits h W^T never materialised).
 
     h_exp [B*N, H_exp], w_exp [V, H_exp], h_ama [B*N, H_ama], w_ama [V, H_ama]: bf16, row-major.
+    beta: fp32 [B] plausibility thresholds (two tensor-core sweeps) or None (beta = 0, one sweep).
     Returns accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse (and the workspace).
-    `gemm_events` = (start, stop) torch.cuda.Event pair recorded around the tensor-core kernel.
+    `gemm_events` = (start, stop) torch.cuda.Event pair recorded around the tensor-core sweeps.
     """
     for t, name in ((h_exp, "h_exp"), (w_exp, "w_exp"), (h_ama, "h_ama"), (w_ama, "w_ama")):
         _require(t, name, dtype=torch.bfloat16)
@@ -328,6 +329,8 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
     _require(tokens, "tokens", torch.int32, dev)
     _require(parents, "parents", torch.int32, dev, (B, N))
     _require(alpha, "alpha", torch.float32, dev, (B,))
+    if beta is not None:
+        _require(beta, "beta", torch.float32, dev, (B,))
     sh = make_shape(B, N, V, DCD_BF16)
     if workspace is None:
         workspace = torch.empty(fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
@@ -340,7 +343,7 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
         ev0, ev1 = (ctypes.c_void_p(e.cuda_event) for e in gemm_events)
     st = load().dcd_verify_fused_lmhead_ex(
         ctypes.byref(sh), _ptr(h_exp), H_exp, _ptr(w_exp), _ptr(h_ama), H_ama, _ptr(w_ama), _ptr(tokens),
-        _ptr(parents), _ptr(alpha), _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]),
+        _ptr(parents), _ptr(alpha), _ptr(beta), _ptr(o["accept_len"]), _ptr(o["accept_path"]), _ptr(o["bonus"]),
         _ptr(o.get("cd_logprob")), _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(workspace),
         workspace.numel(), _stream(stream), ev0, ev1)
     _check(st, "dcd_verify_fused_lmhead")

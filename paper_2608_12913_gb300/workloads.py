@@ -337,8 +337,10 @@ def make_config_torch(cfg: int, device="cuda", **overrides) -> Workload:
 
 def make_fused_torch(device="cuda", B: Optional[int] = None, V: Optional[int] = None,
                      H_exp: Optional[int] = None, H_ama: Optional[int] = None,
-                     seed: Optional[int] = None, levels: Optional[Sequence[int]] = None) -> Workload:
-    """Fused LM-head workload: hidden states ~ N(0,1), weights ~ N(0, 0.02^2), all bf16.
+                     seed: Optional[int] = None, levels: Optional[Sequence[int]] = None,
+                     beta: float = 0.0, w_std: Optional[float] = None) -> Workload:
+    """Fused LM-head workload: hidden states ~ N(0,1), weights ~ N(0, w_std^2) (0.02 unless
+    given), all bf16.
 
     Weights use the nn.Linear layout [V, H] (row v holds the output-embedding of token v).
     Draft tokens are the top-m of (z_p[parent] + N(0,1)) with z_p = h_exp @ w_exp^T taken
@@ -359,8 +361,9 @@ def make_fused_torch(device="cuda", B: Optional[int] = None, V: Optional[int] = 
     gen.manual_seed(1_000_003 * seed + 29)
     h_exp = torch.randn((R, H_exp), generator=gen, device=dev).to(torch.bfloat16)
     h_ama = torch.randn((R, H_ama), generator=gen, device=dev).to(torch.bfloat16)
-    w_exp = (torch.randn((V, H_exp), generator=gen, device=dev) * c["w_std"]).to(torch.bfloat16)
-    w_ama = (torch.randn((V, H_ama), generator=gen, device=dev) * c["w_std"]).to(torch.bfloat16)
+    ws = c["w_std"] if w_std is None else w_std
+    w_exp = (torch.randn((V, H_exp), generator=gen, device=dev) * ws).to(torch.bfloat16)
+    w_ama = (torch.randn((V, H_ama), generator=gen, device=dev) * ws).to(torch.bfloat16)
     tokens = np.zeros((B, N), dtype=np.int32)
     kids = [children_lists(t) for t in tree]
     blk = 512
@@ -378,6 +381,6 @@ def make_fused_torch(device="cuda", B: Optional[int] = None, V: Optional[int] = 
         name=c["name"], B=B, N=N, V=V, dtype="bf16", z_exp=torch.empty(0), z_ama=torch.empty(0),
         tokens=torch.from_numpy(tokens).to(dev), parents=torch.from_numpy(np.stack(tree)).to(dev),
         alpha=torch.full((B,), c["alpha"], dtype=torch.float32, device=dev),
-        beta=torch.zeros(B, dtype=torch.float32, device=dev),
+        beta=torch.full((B,), beta, dtype=torch.float32, device=dev),
         temperature=torch.zeros(B, dtype=torch.float32, device=dev), q=None, seed=seed,
         h_exp=h_exp, w_exp=w_exp, h_ama=h_ama, w_ama=w_ama)

@@ -68,6 +68,19 @@ def run_gpu(w, *, sampled: bool, residual: bool = False, stages: int = 0, plain:
     return res
 
 
+# The fused LM-head forms its logits itself: bf16 products accumulated in fp32 over K = H (8192
+# at full size).  That rounding is about sqrt(K / 16) * 2^-24 * sum_k |h_k w_k| ~ 1.4e-4 of a
+# logit at full size (sum |h w| ~ 100), against the oracle's exact fp64 logits.
+# * FUSED_AMB_MASK: margin to the plausibility threshold within which the two may mask a token
+#   differently;
+# * FUSED_SCORE_TOL: the score bar of a masked fused row.  With beta > 0 few tokens make up P_beta
+#   and the normaliser follows the GEMM's rounding of one or two logits, (1 + 2 alpha) x 1.4e-4
+#   at alpha = 0.1, where an unmasked row's normaliser averages it over many tokens (those keep
+#   the 1e-4 bar).
+FUSED_AMB_MASK = 2e-4
+FUSED_SCORE_TOL = 3e-4
+
+
 def fused_records(ws: torch.Tensor, R: int):
     """Per-row records of the fused LM-head step (after the 256-byte header, 3 x R x 8 child
     entries of 4 bytes and R 4-byte row statuses padded to 16 bytes)."""
@@ -76,9 +89,10 @@ def fused_records(ws: torch.Tensor, R: int):
     return dict(acc_child=raw[:, 0].copy(), term_token=raw[:, 1].copy(), status=raw[:, 2].view(np.uint32).copy())
 
 
-def run_fused_gpu(w) -> dict:
-    """The fused LM-head call on workload `w`, results on the host in the layout `compare` takes."""
-    o = dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha)
+def run_fused_gpu(w, beta=None) -> dict:
+    """The fused LM-head call on workload `w` (with the plausibility thresholds `beta`, a tensor
+    [B], or none), results on the host in the layout `compare` takes."""
+    o = dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha, beta)
     torch.cuda.synchronize()
     res = {k: v.cpu().numpy() for k, v in o.items() if k != "workspace"}
     res["records"] = fused_records(o["workspace"], w.B * w.N)
@@ -86,29 +100,42 @@ def run_fused_gpu(w) -> dict:
     return res
 
 
-def compare(w, gpu: dict, ref: dict, seqs=None, check_residual: bool = False, max_amb_frac: float = 0.05):
-    """Asserts parity of GPU outputs (all sequences of `w`, or the subset `seqs`) with the oracle's."""
+def compare(w, gpu: dict, ref: dict, seqs=None, check_residual: bool = False, max_amb_frac: float = 0.05,
+            amb_mask: float = AMB_MASK, score_tol: float = SCORE_TOL):
+    """Asserts parity of GPU outputs (all sequences of `w`, or the subset `seqs`) with the oracle's.
+
+    `amb_mask` is the margin to the plausibility threshold below which a row's mask is taken as
+    unresolved.  With materialised logits both sides test the same values and AMB_MASK covers
+    fp32 against fp64 evaluation; the fused LM-head forms the logits itself in fp32, so its
+    callers pass the GEMM's rounding instead.  Such a row's scores are not compared either (one
+    token on the other side of the threshold moves its normaliser)."""
     B, N = w.B, w.N
     sel = np.arange(B) if seqs is None else np.asarray(seqs)
     rows_ref = ref["rows"]  # [len(sel), N]
     gsel = (sel[:, None] * N + np.arange(N)[None, :]).reshape(-1)
     rr = rows_ref.reshape(-1)
+    mask_amb = rr["gap_mask"] < amb_mask
     amb = ((rr["gap_argmax"] < AMB_ARGMAX) | (rr["gap_accept"] < AMB_ACCEPT) | (rr["gap_race"] < AMB_RACE) |
-           (rr["gap_mask"] < AMB_MASK))
+           mask_amb)
     assert gpu["error_bits"] == 0, f"device error bits {gpu['error_bits']:#x}"
     assert np.all(gpu["records"]["status"][gsel] == 0)
 
-    # Eq. 1 scores, within tolerance everywhere
+    # Eq. 1 scores, within tolerance everywhere the mask is resolved
     lse_g = gpu["cd_lse"].reshape(-1)[gsel].astype(np.float64)
-    lse_err = np.abs(lse_g - rr["cd_lse"])
-    assert lse_err.max() <= SCORE_TOL, f"cd_lse max error {lse_err.max():.3g}"
+    lse_err = np.where(mask_amb, 0.0, np.abs(lse_g - rr["cd_lse"]))
+    assert lse_err.max() <= score_tol, f"cd_lse max error {lse_err.max():.3g}"
     lp_g = gpu["cd_logprob"][sel].astype(np.float64)
     lp_r = ref["cd_logprob"]
+    # a node's score comes from its parent's row
+    par = w.parents.cpu().numpy()[sel] if hasattr(w.parents, "cpu") else np.asarray(w.parents)[sel]
+    row_amb = mask_amb.reshape(len(sel), N)
+    node_amb = np.zeros_like(row_amb)
+    node_amb[:, 1:] = np.take_along_axis(row_amb, np.clip(par[:, 1:], 0, N - 1), axis=1)
     both_inf = np.isneginf(lp_g) & np.isneginf(lp_r)
-    assert np.array_equal(np.isneginf(lp_g), np.isneginf(lp_r)), "plausibility masks differ"
+    assert np.array_equal(np.isneginf(lp_g) & ~node_amb, np.isneginf(lp_r) & ~node_amb), "plausibility masks differ"
     with np.errstate(invalid="ignore"):
-        lp_err = np.where(both_inf, 0.0, np.abs(lp_g - lp_r))
-    assert lp_err.max() <= SCORE_TOL, f"cd_logprob max error {lp_err.max():.3g}"
+        lp_err = np.where(both_inf | node_amb, 0.0, np.abs(lp_g - lp_r))
+    assert lp_err.max() <= score_tol, f"cd_logprob max error {lp_err.max():.3g}"
 
     # integer decisions per row: bit-exact where the margin is resolvable in fp32
     arg_g = gpu["cd_argmax"].reshape(-1)[gsel]
