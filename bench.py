@@ -291,7 +291,7 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     # weak scaling: every rank verifies its own full batch
-    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch,
+    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch or 32,
                                     temperatures=(0.0,) if args.greedy else (0.0, 1.0))
     B, N, V = w.B, w.N, w.V
     R = B * N
@@ -442,7 +442,7 @@ def run_fused(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = workloads.make_fused_torch(device=dev, seed=4 + rank, beta=args.beta)
+    w = workloads.make_fused_torch(device=dev, seed=4 + rank, beta=args.beta, B=args.batch)
     B, N, V = w.B, w.N, w.V
     R = B * N
     H_exp, H_ama = w.h_exp.shape[1], w.h_ama.shape[1]
@@ -541,7 +541,8 @@ def run_fused(args):
             "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": FUSED_WORKLOAD + (f" beta={args.beta:g}" if beta is not None else ""),
+            "config": {"workload": FUSED_WORKLOAD + (f" beta={args.beta:g}" if beta is not None else "") +
+                       (f" (profiling case, B={B})" if B != 64 else ""),
                        "B": B, "N": N, "V": V, "rows": R, "H_exp": H_exp,
                        "H_ama": H_ama, "flop_per_step": flop, "beta": args.beta,
                        "l2": "weights (2.6 GB) larger than L2; no flush",
@@ -581,7 +582,7 @@ def run_diagnostics(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch)
+    w = workloads.make_config_torch(3, device=dev, seed=3 + rank, B=args.batch or 32)
     B, N, V = w.B, w.N, w.V
     R = B * N
     zp, zq, q = w.z_exp.reshape(R, V), w.z_ama.reshape(R, V), w.q.reshape(R, V)
@@ -712,8 +713,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
     ap.add_argument("--no-soak", action="store_true", help="skip the 1 s clock soak (profiling runs)")
     ap.add_argument("--greedy", action="store_true", help="every sequence greedy (profiling case)")
-    ap.add_argument("--batch", type=int, default=32,
-                    help="sequences per GPU; the benchmark workload is 32 (smaller values are profiling cases)")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="sequences per GPU; the benchmark workloads use 32 (batched, diagnostics) and 64 "
+                         "(fused); other values are profiling cases")
     ap.add_argument("--distinct", action="store_true",
                     help="sampled rule for siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)")
     ap.add_argument("--beta", type=float, default=0.0,

@@ -6,15 +6,17 @@
 // columns x 128 lanes: the whole of it).  Per CTA:
 //   warp 0  -- TMA producer: for every K block of 64 it loads the 128 x 64 bf16 tile of h and the
 //              256 x 64 bf16 tile of W (128-byte swizzle) into a 4-stage shared-memory ring,
-//              first the expert's K blocks, then the amateur's;
+//              first the amateur's K blocks, then the expert's;
 //   warp 1  -- allocates tensor memory, and its lane 0 issues tcgen05.mma (M = 128, N = 256,
-//              K = 16; bf16 in, fp32 accumulate) into z_p then z_q, committing each stage back to
+//              K = 16; bf16 in, fp32 accumulate) into z_q then z_p, committing each stage back to
 //              the producer and each finished tile to the epilogue;
-//   warps 2-5 -- epilogue: each thread owns one row of the tile (one TMEM lane), reads its 2 x
-//              256 accumulators, forms the scaled CD score u = log2(e) ((1 + alpha) z_p -
-//              alpha z_q) (Eq. 1 at T = 1; the log-softmax shifts cancel) on P_beta, and
-//              keeps the tile's max of u, sum of 2^(u - max) and argmax; the score at each child
-//              token that falls in the tile is kept too.  Tiles are visited vocabulary-block
+//   warps 2-5 -- epilogue: each thread owns one row of the tile (one TMEM lane).  Phase 1 reads
+//              both accumulators 64 columns at a time, forms the scaled CD score u = log2(e)
+//              ((1 + alpha) z_p - alpha z_q) (Eq. 1 at T = 1; the log-softmax shifts cancel) on
+//              P_beta, keeps the score at each child token of the tile, and stores u over z_p;
+//              the z_q columns then go back to the MMA warp, which starts the next tile's amateur
+//              blocks.  Phase 2 reduces u to the tile's max, sum of 2^(u - max) and argmax while
+//              those MMAs run, then hands back the z_p columns.  Tiles are visited vocabulary-block
 //              major, so the 30 row tiles that share a block of W read it while it is in L2, and
 //              h (read once per vocabulary block) is kept in L2 with an evict-last policy.
 //   With a plausibility mask (beta > 0, Sec. 2.1) the kernel runs twice: a first sweep over the
@@ -80,12 +82,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kGStages * kGStageBytes);
   uint64_t* empty = full + kGStages;
   uint64_t* tfull = empty + kGStages;  // accumulators of a tile complete
-  uint64_t* tempty = tfull + 1;        // accumulators read by the epilogue
-  uint64_t* drained = tempty + 1;      // every MMA issued has completed (before tensor memory is freed)
+  uint64_t* qfree = tfull + 1;         // the z_q columns read by the epilogue (u is in the z_p columns)
+  uint64_t* pfree = qfree + 1;         // the z_p columns (holding u) read by the epilogue
+  uint64_t* drained = pfree + 1;       // every MMA issued has completed (before tensor memory is freed)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drained + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nk = P.sweep == 1 ? P.nkp : P.nkp + P.nkq;  // the max sweep runs the expert's K blocks only
+  const int qblocks = P.sweep == 1 ? 0 : P.nkq;          // K blocks of the amateur, issued first
   // A bounded wait that gives up records the error and makes every role of the CTA leave its
   // loop, so a failure costs one wait limit, not one per remaining stage.
   auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) -> bool {
@@ -102,7 +106,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
       mbar_init(&empty[s], 1);
     }
     mbar_init(tfull, 1);
-    mbar_init(tempty, 4);
+    mbar_init(qfree, 4);
+    mbar_init(pfree, 4);
     mbar_init(drained, 1);
     fence_mbar_init();
     tc::prefetch_tensormap(&P.tm_hp);
@@ -130,12 +135,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
           unsigned char* a = smem + s * kGStageBytes;
           unsigned char* b = a + kABytes;
           mbar_arrive_expect_tx(&full[s], kGStageBytes);
-          if (kb < P.nkp) {
-            tc::tma_load_2d(a, &P.tm_hp, kb * kBK, i * kBM, &full[s], pol_h);
-            tc::tma_load_2d(b, &P.tm_wp, kb * kBK, j * kBN, &full[s]);
+          if (kb < qblocks) {  // the amateur's K blocks first
+            tc::tma_load_2d(a, &P.tm_hq, kb * kBK, i * kBM, &full[s], pol_h);
+            tc::tma_load_2d(b, &P.tm_wq, kb * kBK, j * kBN, &full[s]);
           } else {
-            tc::tma_load_2d(a, &P.tm_hq, (kb - P.nkp) * kBK, i * kBM, &full[s], pol_h);
-            tc::tma_load_2d(b, &P.tm_wq, (kb - P.nkp) * kBK, j * kBN, &full[s]);
+            tc::tma_load_2d(a, &P.tm_hp, (kb - qblocks) * kBK, i * kBM, &full[s], pol_h);
+            tc::tma_load_2d(b, &P.tm_wp, (kb - qblocks) * kBK, j * kBN, &full[s]);
           }
         }
       }
@@ -152,23 +157,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
       constexpr uint32_t idesc = tc::idesc_bf16_f32(kBM, kBN);
       uint32_t it = 0, tcount = 0;
       for (int tile = blockIdx.x; tile < P.ntiles && !*abort_flag; tile += gridDim.x, ++tcount) {
-        // the epilogue has read the previous tile's accumulators
-        if (!wait_or_abort(tempty, (tcount & 1u) ^ 1u)) break;
-        tc::fence_after_sync();
+        // The amateur's blocks go to the z_q columns as soon as the epilogue has read the last
+        // tile's z_q (it keeps that tile's scores u in the z_p columns); the expert's blocks wait
+        // until it has read those too.  The epilogue's reductions overlap the amateur's MMAs.
+        bool ok = true;
         for (int kb = 0; kb < nk; ++kb, ++it) {
+          if (kb == 0 && qblocks > 0) {
+            if (!wait_or_abort(qfree, (tcount & 1u) ^ 1u)) { ok = false; break; }
+            tc::fence_after_sync();
+          }
+          if (kb == qblocks) {
+            if (!wait_or_abort(pfree, (tcount & 1u) ^ 1u)) { ok = false; break; }
+            tc::fence_after_sync();
+          }
           const int s = static_cast<int>(it % kGStages);
-          if (!wait_or_abort(&full[s], (it / kGStages) & 1u)) break;
+          if (!wait_or_abort(&full[s], (it / kGStages) & 1u)) { ok = false; break; }
           tc::fence_after_sync();
           const unsigned char* a = smem + s * kGStageBytes;
           const uint64_t ad = tc::sw128_kmajor_desc(a), bd = tc::sw128_kmajor_desc(a + kABytes);
-          const uint32_t d = tmem + (kb < P.nkp ? 0u : static_cast<uint32_t>(kBN));
-          const bool first = kb == 0 || kb == P.nkp;
+          const uint32_t d = tmem + (kb < qblocks ? static_cast<uint32_t>(kBN) : 0u);
+          const bool first = kb == 0 || kb == qblocks;
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k)  // K = 16 per MMA: 32 bytes along the swizzled row
             tc::mma_bf16(d, ad + 2 * k, bd + 2 * k, idesc, !(first && k == 0));
           tc::mma_commit(&empty[s]);
         }
-        if (*abort_flag) break;
+        if (!ok || *abort_flag) break;
         tc::mma_commit(tfull);
       }
       tc::mma_commit(drained);
@@ -229,52 +243,69 @@ __global__ void __launch_bounds__(kGemmThreads, 1) fused_lmhead_kernel(const __g
         }
         tc::fence_before_sync();
         __syncwarp();
-        if (lane == 0) mbar_arrive(tempty);
+        if (lane == 0) {
+          mbar_arrive(qfree);
+          mbar_arrive(pfree);
+        }
         if (valid) __stcs(&P.part[static_cast<int64_t>(r) * P.nvt + j], make_float4(mz, 0.f, 0.f, 0.f));
         continue;
       }
       const bool masked = logb > -INFINITY;
+      // phase 1: u = log2(e) ((1 + alpha) z_p - alpha z_q) on P_beta, written over z_p; the scores at
+      // the children's tokens; then the z_q columns go back to the MMA warp
+#pragma unroll 1
+      for (int c = 0; c < kBN / 64; ++c) {
+        float zp[64], zq[64];
+        tc::tmem_ld64x2(trow + c * 64, trow + kBN + c * 64, zp, zq);
+        const int col0 = j * kBN + c * 64;
+#pragma unroll
+        for (int e = 0; e < 64; ++e)  // u in place of z_p
+          zp[e] = (col0 + e < P.V && (!masked || zp[e] - Mp >= logb)) ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxKids; ++k) {
+          const unsigned d = static_cast<unsigned>(kt[k] - col0);
+          if (d < 64u) {  // rare: this child's token is in the chunk
+            float v = 0.f;
+#pragma unroll
+            for (int e = 0; e < 64; ++e) v = (d == static_cast<unsigned>(e)) ? zp[e] : v;
+            P.kid_u[r * kMaxKids + k] = v;
+          }
+        }
+        tc::tmem_st64(trow + c * 64, zp);
+      }
+      tc::tmem_st_wait();
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(qfree);
+      // phase 2 (while the next tile's amateur MMAs run): the tile's max of u, sum of 2^(u - max)
+      // and argmax, from the z_p columns
       float m = -INFINITY, ssum = 0.f;
       int arg = INT_MAX;
 #pragma unroll 1
-      for (int c = 0; c < kBN / 32; ++c) {
-        float zp[32], zq[32];
-        tc::tmem_ld32x2(trow + c * 32, trow + kBN + c * 32, zp, zq);
-        const int col0 = j * kBN + c * 32;
-        float u[32];
+      for (int c = 0; c < kBN / 64; ++c) {
+        float u[64];
+        tc::tmem_ld32x2(trow + c * 64, trow + c * 64 + 32, u, u + 32);
+        const int col0 = j * kBN + c * 64;
         float cm = -INFINITY;
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          u[e] = (col0 + e < P.V && (!masked || zp[e] - Mp >= logb)) ? fmaf(c1k, zp[e], -ak * zq[e]) : -INFINITY;
-          cm = fmaxf(cm, u[e]);
-        }
+        for (int e = 0; e < 64; ++e) cm = fmaxf(cm, u[e]);
         if (cm > m) {
           ssum = m > -INFINITY ? ssum * ex2(m - cm) : 0.f;
           m = cm;
 #pragma unroll
-          for (int e = 31; e >= 0; --e)
+          for (int e = 63; e >= 0; --e)
             if (u[e] == cm) arg = col0 + e;
         }
         if (m > -INFINITY) {
           float acc = 0.f;
 #pragma unroll
-          for (int e = 0; e < 32; ++e) acc += ex2(u[e] - m);
+          for (int e = 0; e < 64; ++e) acc += ex2(u[e] - m);
           ssum += acc;
-        }
-#pragma unroll
-        for (int k = 0; k < kMaxKids; ++k) {
-          const unsigned d = static_cast<unsigned>(kt[k] - col0);
-          if (d < 32u) {  // rare: this child's token is in the chunk
-            float v = 0.f;
-#pragma unroll
-            for (int e = 0; e < 32; ++e) v = (d == static_cast<unsigned>(e)) ? u[e] : v;
-            P.kid_u[r * kMaxKids + k] = v;
-          }
         }
       }
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty);
+      if (lane == 0) mbar_arrive(pfree);
       // streaming store: read once by the combine kernel, it should not displace h in L2
       if (valid) __stcs(&P.part[static_cast<int64_t>(r) * P.nvt + j], make_float4(m, ssum, __int_as_float(arg), 0.f));
     }
