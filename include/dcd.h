@@ -186,7 +186,7 @@ int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_p
 
 /*
  * Capacity of the scratch array inside the library used by dcd_verify_sample_noalloc:
- * enough for dcd_workspace_bytes(shape) <= 4 MiB, e.g. B * N up to about 11,700 rows at
+ * enough for dcd_workspace_bytes(shape) <= 4 MiB, e.g. B * N up to 6,354 rows at
  * V = 128256 with bf16 logits.
  */
 #define DCD_STATIC_SCRATCH_BYTES (4u * 1024u * 1024u)
