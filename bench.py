@@ -19,7 +19,7 @@ node, 1.97 GB read per step).
 bf16, greedy): one step is both output projections on the tensor cores with the CD
 epilogue, the per-row combine and the tree walk.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload batched|fused|diagnostics]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload batched|fused|diagnostics|small]
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle on a
 bounded sample of the same workload instead.
@@ -715,6 +715,117 @@ def run_diagnostics(args):
     return 0
 
 
+def run_small(args):
+    """Latency of one small verification call (BASELINE configs 0-2: a 6-node chain at V = 32000,
+    or a 60-node tree at V = 128256, greedy or sampled), through the public API.  The device time
+    per call is taken from CUDA-graph replays of 64 calls (the host's launch cost left out); the
+    eager per-call time is reported beside it."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_12913_gb300 import dcd, workloads
+
+    world, rank, local = _dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg = args.config
+    w = workloads.make_config_torch(cfg, device=dev, seed=cfg + rank)
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    sampled = w.q is not None
+    out = dcd.alloc_outputs(B, N, dev)
+    ws = dcd.alloc_workspace(B, N, V, dev, dtype=dcd.DCD_F32 if w.dtype == "f32" else dcd.DCD_BF16)
+
+    def call(i, stream):
+        if sampled:
+            dcd.dcd_verify_sample(w.z_exp, w.z_ama, w.q, w.tokens, w.parents, w.alpha, w.temperature, w.seed, i,
+                                  w.beta, out=out, workspace=ws, stream=stream)
+        else:
+            dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, out=out, workspace=ws,
+                                  stream=stream)
+
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        for i in range(max(args.warmup, 3)):
+            call(i, stream)
+    stream.synchronize()
+    if dcd.dcd_get_device_error(ws, stream) != 0:
+        raise RuntimeError("device error bits set during warm-up")
+    per_graph = 64
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for i in range(per_graph):
+            call(i, stream)
+    graph.replay()
+    torch.cuda.synchronize()
+    reps = max(1, args.steps // per_graph)
+    sampler = ClockSampler(local)
+    sampler.start()
+    t_soak = time.time()
+    while not args.no_soak and time.time() - t_soak < 1.0:
+        graph.replay()
+        torch.cuda.synchronize()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    start.record()
+    for _ in range(reps):
+        graph.replay()
+    stop.record()
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    sampler.stop()
+    steps = reps * per_graph
+    ms_per_step = start.elapsed_time(stop) / steps
+    if world > 1:
+        ms_per_step = max_over_ranks(ms_per_step, dist, dev)
+    # eager calls, the host's launch cost included
+    with torch.cuda.stream(stream):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(steps):
+            call(i, stream)
+        b.record(stream)
+    torch.cuda.synchronize()
+    eager_ms = a.elapsed_time(b) / steps
+    if dcd.dcd_get_device_error(ws, stream) != 0:
+        raise RuntimeError("device error bits set during the timed region")
+    es = 4 if w.dtype == "f32" else 2
+    alg = float(R * V * 2 * es)  # both logit rows of every node (q: only at children unless rejected)
+    peak, peak_kind = _peaks()
+    achieved = alg / (ms_per_step / 1e3) / 1e9
+    path = "one launch (greedy_small_kernel)" if not sampled and R <= 512 else "persistent row kernel + tree walk"
+    if rank == 0:
+        line = {
+            "metric": METRIC + ", small call", "value": job_value(world, R, ms_per_step), "unit": "nodes/s",
+            "n_gpus": world, "steps": steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "B": B, "N": N, "V": V, "rows": R, "logits": w.dtype,
+                       "path": path, "timing": f"CUDA-graph replays of {per_graph} calls",
+                       "eager_ms_per_call": eager_ms,
+                       "l2": "inputs smaller than L2 and re-read every call: latency, not bandwidth",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None, "kernel": "whole call (latency-bound)",
+                         "peak_source": f"{peak_kind} hbm_gbs", "algorithmic_bytes_per_launch": alg},
+            "clocks": sampler.summary(t_wall0, t_wall1),
+            "e2e": {"value": job_value(world, R, eager_ms), "unit": "nodes/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0, "ms_per_step": eager_ms,
+                    "note": "eager calls on device-resident inputs (the host's launch cost included)"},
+            "gpu_launches": (1 if path.startswith("one") else 2) * steps,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -732,9 +843,13 @@ def main():
                     help="sampled rule for siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)")
     ap.add_argument("--beta", type=float, default=0.0,
                     help="fused workload: plausibility threshold of every sequence (0: no mask, one sweep)")
-    ap.add_argument("--workload", choices=("batched", "fused", "diagnostics"), default="batched",
+    ap.add_argument("--workload", choices=("batched", "fused", "diagnostics", "small"), default="batched",
                     help="batched: the streaming step on materialised logits (the headline); fused: the "
-                         "fused LM-head variant; diagnostics: the per-row diagnostics pass")
+                         "fused LM-head variant; diagnostics: the per-row diagnostics pass; small: the "
+                         "latency of one small call (--config)")
+    ap.add_argument("--config", type=int, choices=(0, 1, 2), default=0,
+                    help="small workload: 0 = 6-node chain (fp32, V 32000, greedy), 1 = 60-node tree "
+                         "(bf16, V 128256, greedy), 2 = the same tree sampled at T = 1")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -744,6 +859,8 @@ def main():
         return run_fused(args)
     if args.workload == "diagnostics":
         return run_diagnostics(args)
+    if args.workload == "small":
+        return run_small(args)
     return run_ours(args)
 
 
