@@ -30,7 +30,7 @@ size_t workspace_bytes_for(const dcd_shape* s) {
   const size_t rows = static_cast<size_t>(s->B) * static_cast<size_t>(s->N);
   const size_t raw = dcd::kWorkspaceHeader + dcd::part_counter_bytes(rows) +
                      rows * (sizeof(dcd::Job) + sizeof(dcd::RowRecord) + dcd::kMaxParts * sizeof(dcd::RowPart) +
-                             dcd::slot_bytes(s->V, s->logits_dtype));
+                             dcd::slot_bytes(s->V, s->logits_dtype, static_cast<int64_t>(rows)));
   return (raw + 255) & ~static_cast<size_t>(255);
 }
 

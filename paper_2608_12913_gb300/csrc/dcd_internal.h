@@ -121,9 +121,10 @@ struct ScoreArgs {
   int32_t force_plain;    // 1 = plain loads instead of bulk async copies
 };
 
-// Residual pieces per pass and slot bytes per row for a vocabulary of V tokens.
-int residual_pieces(int64_t V, int dtype);
-size_t slot_bytes(int64_t V, int dtype);
+// Residual pieces per pass and slot bytes per row for a vocabulary of V tokens in a call of
+// `rows` rows (small calls use smaller pieces).
+int residual_pieces(int64_t V, int dtype, int64_t rows);
+size_t slot_bytes(int64_t V, int dtype, int64_t rows);
 
 cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream);
 

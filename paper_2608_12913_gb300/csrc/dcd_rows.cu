@@ -71,7 +71,19 @@ constexpr int kMaxStages = 8;
 #ifndef DCD_PARTS_BELOW
 #define DCD_PARTS_BELOW 2
 #endif
-constexpr int kPieceStages = DCD_PIECE_STAGES;     // ring stages per residual piece
+constexpr int kPieceStages = DCD_PIECE_STAGES;     // ring stages per residual piece (at most)
+#ifndef DCD_SMALL_PIECE_ROWS
+#define DCD_SMALL_PIECE_ROWS 256
+#endif
+#ifndef DCD_SMALL_PIECE_STAGES
+#define DCD_SMALL_PIECE_STAGES 2
+#endif
+// A call with at most kSmallPieceRows rows splits residual passes into pieces of
+// kSmallPieceStages stages: its chains of passes are on the critical path, and smaller pieces
+// spread each pass over more CTAs (measured: 4% faster at 120 rows, neutral at 480; one-stage
+// pieces were slower at 480 rows).
+constexpr int64_t kSmallPieceRows = DCD_SMALL_PIECE_ROWS;
+constexpr int kSmallPieceStages = DCD_SMALL_PIECE_STAGES;
 // Rows are streamed in parts only when the batch has at most this many rows per resident CTA:
 // then whole rows would leave most CTAs idle for part of the step; with more rows than that,
 // dynamic claiming of whole rows balances better than parts (measured).
@@ -92,6 +104,7 @@ struct SParams {
   int32_t tok_a;         // tokens per stage in row passes (z_p, then z_q)
   int32_t tok_r;         // tokens per stage in residual pieces (z_p, z_q, then q)
   int32_t npieces;       // pieces per residual pass
+  int32_t piece_stages;  // ring stages per residual piece
   int32_t bulk;          // 1: bulk asynchronous copies, 0: plain loads
   int32_t nblk;          // race blocks per row, ceil(V / 1024)
   int32_t nchunk;        // warp chunks per row in the stats pass, ceil(V / (tok_a / 8))
@@ -532,9 +545,9 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           D.J = __shfl_sync(~0u, D.J, 0);
           D.m = __shfl_sync(~0u, D.m, 0);
           tok = sp.tok_r;
-          x_lo = static_cast<int64_t>(piece) * kPieceStages * sp.tok_r;
+          x_lo = static_cast<int64_t>(piece) * sp.piece_stages * sp.tok_r;
           const int64_t rem = (V - x_lo + sp.tok_r - 1) / sp.tok_r;
-          nitems = static_cast<int>(rem < kPieceStages ? rem : kPieceStages);
+          nitems = static_cast<int>(rem < sp.piece_stages ? rem : sp.piece_stages);
           with_q = true;
           // a later pass re-reads the piece; the pass after the last sibling is the last read
           pol = D.J < D.m ? (sp.keep_internal ? pol_last : pol_normal) : pol_first;
@@ -641,9 +654,9 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       // a warp takes tok_r / 8 consecutive tokens of each stage (a chunk); `wpb` chunks make a
       // race block
       const int tpw = sp.tok_r / kWarps, wpb = kRaceBlock / tpw;
-      const int64_t piece_lo = static_cast<int64_t>(piece) * kPieceStages * sp.tok_r;
+      const int64_t piece_lo = static_cast<int64_t>(piece) * sp.piece_stages * sp.tok_r;
       const int64_t rem = (V - piece_lo + sp.tok_r - 1) / sp.tok_r;
-      const int nst_piece = static_cast<int>(rem < kPieceStages ? rem : kPieceStages);
+      const int nst_piece = static_cast<int>(rem < sp.piece_stages ? rem : sp.piece_stages);
       float zl = 0.f;
       for (int L = 0; L < nst_piece; ++L, ++seq) {
         const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(sp.nst)), sp.tok_r);
@@ -1496,14 +1509,16 @@ int chunks_per_row(int64_t V, int es) {
 
 }  // namespace
 
-int residual_pieces(int64_t V, int dtype) {
+int piece_stages_for(int64_t rows) { return rows <= kSmallPieceRows ? kSmallPieceStages : kPieceStages; }
+
+int residual_pieces(int64_t V, int dtype, int64_t rows) {
   const int es = dtype == DCD_BF16 ? 2 : 4;
-  const int64_t tok = static_cast<int64_t>(tokens_r(es)) * kPieceStages;
+  const int64_t tok = static_cast<int64_t>(tokens_r(es)) * piece_stages_for(rows);
   return static_cast<int>((V + tok - 1) / tok);
 }
 
-size_t slot_bytes(int64_t V, int dtype) {
-  return sizeof(SlotHead) + static_cast<size_t>(residual_pieces(V, dtype)) * sizeof(PiecePart) +
+size_t slot_bytes(int64_t V, int dtype, int64_t rows) {
+  return sizeof(SlotHead) + static_cast<size_t>(residual_pieces(V, dtype, rows)) * sizeof(PiecePart) +
          kMaxRemoved * sizeof(Removed);
 }
 
@@ -1539,7 +1554,8 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.nst = geo.stages;
   sp.tok_a = tokens_a(es);
   sp.tok_r = tokens_r(es);
-  sp.npieces = residual_pieces(a.V, a.dtype);
+  sp.npieces = residual_pieces(a.V, a.dtype, R);
+  sp.piece_stages = piece_stages_for(R);
   sp.bulk = geo.bulk;
   sp.nblk = static_cast<int>((a.V + kRaceBlock - 1) / kRaceBlock);
   sp.nchunk = chunks_per_row(a.V, es);
@@ -1547,7 +1563,7 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.meta_offset = l.meta_offset;
   sp.chunk_offset = l.chunk_offset;
   sp.stage_offset = l.stage_offset;
-  sp.slot_bytes = static_cast<int32_t>(slot_bytes(a.V, a.dtype));
+  sp.slot_bytes = static_cast<int32_t>(slot_bytes(a.V, a.dtype, R));
   sp.hdr = a.hdr;
   sp.jobs = a.jobs;
   sp.slots = a.slots;
