@@ -708,7 +708,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
           bb = kabs;
         }
       }
-      block_argmax(bk, bb, redf, redi, csync);
+      if (race) block_argmax(bk, bb, redf, redi, csync);  // CTA-uniform; other passes rank no blocks
       if (tid == 0) {
         PiecePart pp;
         pp.z = zsum;
