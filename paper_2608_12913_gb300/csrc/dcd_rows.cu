@@ -723,17 +723,27 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       if (rs->last) {
         // ================= the pass is complete: next sibling test, next pass or terminal race
         if (warp == 0) list_children(p, b, n, kids, ktok);
-        if (tid == 0) {
-          SlotHead* sh = slot_head(sp, D.slot);
+        if (warp == 1 && lane == 0) {
+          // the pieces' partial sums and race keys, read while warp 0 lists the children
           const PiecePart* parts = slot_parts(sp, D.slot);
           float DJ = 0.f, K = -INFINITY;
           int kstar = INT_MAX;
           uint32_t st2 = D.status;
-          for (int k = 0; k < sp.npieces; ++k) {
+          for (int k = 0; k < sp.npieces; ++k) {  // a fixed order
             DJ += parts[k].z;
             argmax_merge(K, kstar, parts[k].key, parts[k].blk);
             if (parts[k].timed_out) st2 |= DCD_DEVERR_TIMEOUT;
           }
+          rs->D = DJ;
+          rs->term = kstar;
+          rs->status = st2;
+        }
+        csync();
+        if (tid == 0) {
+          SlotHead* sh = slot_head(sp, D.slot);
+          const float DJ = rs->D;
+          const int kstar = rs->term;
+          uint32_t st2 = rs->status;
           bool degen = sh->degen != 0;
           float c = sh->c, Dn = sh->D;
           int acc = -1;
