@@ -502,8 +502,14 @@ def run_fused(args):
     value = job_value(world, R, ms_per_step)
     peak, peak_src = _bf16_peak()
     achieved = flop / (gemm_ms / 1e3) / 1e12
+    khash = _kernel_source_hash(("dcd_fused.cu", "dcd_fused.h", "dcd_tc.cuh", "dcd_device.cuh"))
+    # DRAM bytes of one tensor-core launch from the committed launch list (the unmasked call; the
+    # masked call runs two sweeps of different traffic, not captured)
+    traffic = (_profiled_traffic(khash, "fused_lmhead_kernel_B64_tree60_V128256_H8192_2048.md")
+               if beta is None and B == 64 else None)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": None, "kernel": "fused_lmhead_kernel", "peak_source": peak_src,
+                "traffic": traffic, "kernel": "fused_lmhead_kernel", "peak_source": peak_src,
+                "kernel_source_sha256_16": khash,
                 "algorithmic_flops_per_launch": flop, "gemm_kernel_ms": gemm_ms,
                 "flops_counted": "both LM-head GEMMs" + ("; with beta the expert's twice (max sweep, then masked)"
                                                            if beta is not None else "")}
