@@ -147,7 +147,15 @@ struct RowShared {
   int32_t last;     // this CTA finished a pass's last piece
   int32_t degen;    // a pass found no residual mass left
   float c, D;
+  // Distinct siblings: a chain's removed tokens, their frozen masses, and pi and q at them (then
+  // at siblings J - 1 and J), read by two warps in parallel before a pass's sibling step
+  int32_t rn;
+  int32_t rtok[kMaxRemoved + 2];
+  float rfz[kMaxRemoved + 2];
+  float rpit[kMaxRemoved + 2];
+  float rq[kMaxRemoved + 2];
 };
+static_assert(kMaxRemoved <= 32, "one lane a removed token");
 
 template <typename TIn>
 struct Stage {
@@ -722,7 +730,33 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       csync();
       if (rs->last) {
         // ================= the pass is complete: next sibling test, next pass or terminal race
-        if (warp == 0) list_children(p, b, n, kids, ktok);
+        // pi at token t (0 outside P_beta) and q there, as every sibling step computes them
+        auto value_at = [&](int t, float& pit, float& qt) {
+          const float z = ld1(zp_row, t);
+          const bool in = !masked || (z - Mp >= logb);
+          pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, t)) - M) * invS : 0.f;
+          qt = q_row[t];
+        };
+        if (warp == 0) {
+          const int cnt = list_children(p, b, n, kids, ktok);
+          if (kDistinct && lane < 2) {  // the values at siblings J - 1 (removed now) and J (tested next)
+            const int j = J - 1 + lane;
+            const int t = j < cnt ? ktok[j] : -1;
+            const bool ok = t >= 0 && t < V;
+            rs->rtok[kMaxRemoved + lane] = ok ? t : -1;
+            if (ok) value_at(t, rs->rpit[kMaxRemoved + lane], rs->rq[kMaxRemoved + lane]);
+          }
+        }
+        if (kDistinct && warp == 2) {  // the removed tokens so far and the values at them
+          const int nr = slot_head(sp, D.slot)->nrem;
+          if (lane < nr) {
+            const Removed r = slot_removed(sp, D.slot)[lane];
+            rs->rtok[lane] = r.tok;
+            rs->rfz[lane] = r.fz;
+            value_at(r.tok, rs->rpit[lane], rs->rq[lane]);
+          }
+          if (lane == 0) rs->rn = nr;
+        }
         if (warp == 1 && lane == 0) {
           // the pieces' partial sums and race keys, read while warp 0 lists the children
           const PiecePart* parts = slot_parts(sp, D.slot);
@@ -756,20 +790,31 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
             // (frozen at the current residual) and the next siblings are tested against r with
             // the proposal q / Z without the removed tokens.
             Removed* rem = slot_removed(sp, D.slot);
-            int nrem = sh->nrem;
+            int nrem = rs->rn;
             float Z = sh->Z;
-            auto value_at = [&](int t, float& pit, float& qt) {
-              const float z = ld1(zp_row, t);
-              const bool in = !masked || (z - Mp >= logb);
-              pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, t)) - M) * invS : 0.f;
-              qt = q_row[t];
+            // the values read before the barrier; a token not among them is loaded here
+            auto value_of = [&](int t, float& pit, float& qt) {
+              for (int i = 0; i < nrem; ++i)
+                if (rs->rtok[i] == t) {
+                  pit = rs->rpit[i];
+                  qt = rs->rq[i];
+                  return;
+                }
+              for (int i = kMaxRemoved; i < kMaxRemoved + 2; ++i)
+                if (rs->rtok[i] == t) {
+                  pit = rs->rpit[i];
+                  qt = rs->rq[i];
+                  return;
+                }
+              value_at(t, pit, qt);
+            };
+            auto removed_index = [&](int t) {
+              for (int i = 0; i < nrem; ++i)
+                if (rs->rtok[i] == t) return i;
+              return -1;
             };
             float EJ = DJ;
-            for (int i = 0; i < nrem; ++i) {
-              float pit, qt;
-              value_at(rem[i].tok, pit, qt);
-              EJ += rem[i].fz - fmaxf(pit - cJ * qt, 0.f);
-            }
+            for (int i = 0; i < nrem; ++i) EJ += rs->rfz[i] - fmaxf(rs->rpit[i] - cJ * rs->rq[i], 0.f);
             if (EJ > 0.f) {
               c = cJ;
               Dn = EJ;
@@ -777,15 +822,20 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
               ranked = false;  // the pieces ranked blocks of a residual that is not used
             }
             auto remove = [&](int t) {
-              if (t < 0 || t >= V || find_removed(rem, nrem, t) >= 0) return;
+              if (t < 0 || t >= V || removed_index(t) >= 0) return;
               if (nrem >= kMaxRemoved) {
                 st2 |= DCD_DEVERR_UNSUPPORTED;
                 return;
               }
               float pit, qt;
-              value_at(t, pit, qt);
+              value_of(t, pit, qt);
+              const float fz = fmaxf(pit - c * qt, 0.f);
               rem[nrem].tok = t;
-              rem[nrem].fz = fmaxf(pit - c * qt, 0.f);
+              rem[nrem].fz = fz;
+              rs->rtok[nrem] = t;
+              rs->rfz[nrem] = fz;
+              rs->rpit[nrem] = pit;
+              rs->rq[nrem] = qt;
               ++nrem;
               Z -= qt;
             };
@@ -794,12 +844,12 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
               const int t = ktok[j];
               float ratio = 0.f;
               if (t >= 0 && t < V) {
-                const int ri = find_removed(rem, nrem, t);
+                const int ri = removed_index(t);
                 if (ri >= 0) {
-                  ratio = rem[ri].fz > 0.f ? INFINITY : 0.f;  // its proposal is 0
+                  ratio = rs->rfz[ri] > 0.f ? INFINITY : 0.f;  // its proposal is 0
                 } else {
                   float pit, qt;
-                  value_at(t, pit, qt);
+                  value_of(t, pit, qt);
                   const float rho = fmaxf(pit - c * qt, 0.f);
                   const float qp = Z > 0.f ? qt / Z : 0.f;
                   ratio = qp > 0.f ? (rho / Dn) / qp : (rho > 0.f ? INFINITY : 0.f);
