@@ -28,11 +28,12 @@
 //    sum_x max(0, pi(x) - c_j q(x)) (induction on j from r_j = normalise(max(0, r_{j-1} -
 //    q))), so a pass needs only two scalars from the one before.  A row that needs a pass is
 //    handed to a job list; the pass is split into pieces of four ring stages (16384 tokens for
-//    bf16 logits) that any CTA's producer claims before taking a new row.  Each piece writes
-//    its partial sum (and, in the pass after the last sibling, its best race key) to its own
-//    slot; the CTA that finishes a pass's last piece (an atomic ticket, no waiting) sums the
-//    slots in a fixed order, tests the next sibling, and either queues the next pass or runs
-//    the terminal race.  A producer with no row left polls for pieces until every row's record
+//    bf16 logits; two stages in a call of at most 256 rows) that any CTA's producer claims
+//    before taking a new row.  Each piece writes its partial sum (and, in the pass after the
+//    last sibling, its best race key) to its own slot; the CTA that finishes a pass's last piece
+//    (an atomic ticket, no waiting) sums the slots in a fixed order while it lists the node's
+//    children, tests the next sibling, and either queues the next pass or runs the terminal
+//    race.  A producer with no row left polls for pieces until every row's record
 //    is written (bounded; all CTAs are co-resident under a cooperative launch), so the passes
 //    of late chains still spread over the GPU.
 //
