@@ -31,6 +31,14 @@ def test_distinct_full_vocabulary_sampled():
     compare(w, g, _oracle(w, residual=True), check_residual=True)
 
 
+@pytest.mark.parametrize("beta", [0.1, 0.5])
+def test_distinct_with_plausibility_mask(beta):
+    # the distinct rule on masked rows (rows read whole, a max pass first), residual output included
+    w = workloads.make_config(2, V=4099, B=6, beta=beta, seed=33, margin_fn=oracle.margin_fn)
+    g = run_gpu(w, sampled=True, residual=True, distinct=True)
+    compare(w, g, _oracle(w, residual=True), check_residual=True)
+
+
 def test_distinct_mixed_batch_and_split_steps():
     w = workloads.make_config(3, B=6, V=20000, margin_fn=oracle.margin_fn)
     ref = _oracle(w)

@@ -14,7 +14,7 @@ from scipy import special, stats
 
 import oracle
 from paper_2608_12913_gb300 import dcd, workloads
-from parity_util import compare, run_gpu
+from parity_util import AMB_MASK, compare, run_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -62,14 +62,17 @@ def test_config3_full_size_sampled_sequences():
     compare(w, g, r, seqs=seqs, max_amb_frac=0.25)
 
 
-@pytest.mark.parametrize("beta", [1e-3, 0.1, 0.5])
+@pytest.mark.parametrize("beta", [1e-3, 0.1, 0.5, 1.0])
 @pytest.mark.parametrize("sampled", [False, True])
 def test_plausibility_mask(beta, sampled):
+    # beta = 1 keeps only the expert's argmax set: pi_CD is a point mass there.  Its mask test,
+    # z_p - max z_p >= log 1 = 0, is exact in fp32 and fp64 alike (0 for the max token, nonzero for
+    # any other), so the max token's zero distance to the threshold is no ambiguity.
     cfg = 2 if sampled else 1
     w = workloads.make_config(cfg, B=3, V=9001, beta=beta, seed=40 + int(beta * 100), margin_fn=oracle.margin_fn)
     g = run_gpu(w, sampled=sampled, residual=sampled)
     r = _oracle(w, residual=sampled)
-    compare(w, g, r, check_residual=sampled)
+    compare(w, g, r, check_residual=sampled, amb_mask=0.0 if beta == 1.0 else AMB_MASK)
 
 
 @pytest.mark.parametrize("stages", [2, 3, 4, 6])
