@@ -455,37 +455,59 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         int item = 0, piece = 0;
         kind = kWorkNone;
         Job job_rec;  // lane 0: the claimed pass
-        if (lane == 0) {
+        {
+          const uint32_t np_u = static_cast<uint32_t>(sp.npieces);
           const long long t0 = clock64();
           for (int poll = 0;; ++poll) {
-            // a piece of the oldest published pass that still has one (the first look uses the
-            // state read during the last issue).  The scan reaches pass k only after finding every
-            // pass between the head and k without pieces, so whoever claims the last piece of k
-            // may move the head past it.
-            const uint32_t pub = poll ? ld_volatile(&sp.hdr->jobs_published) : pub_seen;
-            for (uint32_t k = poll ? ld_volatile(&sp.hdr->job_head) : head_seen; k < pub; ++k) {
-              const uint32_t pc = atomicAdd(&sp.jobs[k].next_piece, 1u);
-              if (pc < static_cast<uint32_t>(sp.npieces)) {
-                if (pc + 1u == static_cast<uint32_t>(sp.npieces)) atomicMax(&sp.hdr->job_head, k + 1u);
-                kind = kWorkPiece;
-                item = static_cast<int>(k);
-                piece = static_cast<int>(pc);
-                __threadfence();  // the record was written before the pass was published
-                job_rec = load_job(&sp.jobs[k]);
-                break;
+            uint32_t pub = 0u, k0 = 0u;
+            if (lane == 0) {
+              pub = poll ? ld_volatile(&sp.hdr->jobs_published) : pub_seen;
+              k0 = poll ? ld_volatile(&sp.hdr->job_head) : head_seen;
+            }
+            pub = __shfl_sync(~0u, pub, 0);
+            k0 = __shfl_sync(~0u, k0, 0);
+            // a piece of the oldest published pass that still has one: the lanes look at 32
+            // passes at once and only a pass seen open is claimed from (one atomic), so a stale
+            // view of the list costs one round of loads, not an atomic per drained pass.  Every
+            // pass before the claimed one was seen drained, so whoever claims the last piece of a
+            // pass may move the head past it.
+            for (; k0 < pub && kind == kWorkNone; k0 += 32u) {
+              const uint32_t k = k0 + static_cast<uint32_t>(lane);
+              const bool open = k < pub && ld_volatile(&sp.jobs[k].next_piece) < np_u;
+              for (unsigned avail = __ballot_sync(~0u, open); avail != 0u; avail &= avail - 1u) {
+                const uint32_t kc = k0 + static_cast<uint32_t>(__ffs(avail) - 1);
+                uint32_t pc = 0u;
+                if (lane == 0) pc = atomicAdd(&sp.jobs[kc].next_piece, 1u);
+                pc = __shfl_sync(~0u, pc, 0);
+                if (pc < np_u) {
+                  kind = kWorkPiece;
+                  item = static_cast<int>(kc);
+                  piece = static_cast<int>(pc);
+                  if (lane == 0) {
+                    if (pc + 1u == np_u) atomicMax(&sp.hdr->job_head, kc + 1u);
+                    __threadfence();  // the record was written before the pass was published
+                    job_rec = load_job(&sp.jobs[kc]);
+                  }
+                  break;
+                }
               }
             }
             if (kind != kWorkNone) break;
             if (meta.g >= 0) {
               kind = kWorkRow;
-              nr = static_cast<int>(atomicAdd(&sp.hdr->work, 1u));  // its result is read after the next issue
+              if (lane == 0) nr = static_cast<int>(atomicAdd(&sp.hdr->work, 1u));  // read after the next issue
               break;
             }
-            if (poll && ld_volatile(&sp.hdr->rows_done) >= static_cast<uint32_t>(R)) break;
-            if (clock64() - t0 > kWaitCycles) {
-              atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
-              break;
+            int stop = 0;
+            if (lane == 0) {
+              if (poll && ld_volatile(&sp.hdr->rows_done) >= static_cast<uint32_t>(R)) {
+                stop = 1;
+              } else if (clock64() - t0 > kWaitCycles) {
+                atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
+                stop = 1;
+              }
             }
+            if (__shfl_sync(~0u, stop, 0)) break;
             if (poll) __nanosleep(256);
           }
         }
