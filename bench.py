@@ -379,18 +379,18 @@ def run_ours(args):
     e2e = None
     if not args.no_e2e:
         host = {k: getattr(w, k).cpu().pin_memory() for k in ("z_exp", "z_ama", "q", "tokens", "parents", "alpha",
-                                                               "beta", "temperature")}
+                                                               "beta", "temperature") if getattr(w, k) is not None}
         dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
         res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory() for k in ("accept_len", "accept_path",
                                                                                      "bonus")}
-        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        # q is copied only for the sampled sequences: the verification reads no other row of it
+        h2d = dcd.upload_inputs(host, dst, N, stream)
         d2h = sum(v.numel() * v.element_size() for v in res_host.values())
         n_e2e = max(3, min(args.steps, 10))
 
         def e2e_step(i):
-            for k in host:
-                dst[k].copy_(host[k], non_blocking=True)
-            o = dcd.dcd_verify_sample(dst["z_exp"], dst["z_ama"], dst["q"], dst["tokens"], dst["parents"],
+            dcd.upload_inputs(host, dst, N, stream)
+            o = dcd.dcd_verify_sample(dst["z_exp"], dst["z_ama"], dst.get("q"), dst["tokens"], dst["parents"],
                                       dst["alpha"], dst["temperature"], w.seed, 2_000_000 + i, dst["beta"], out=out,
                                       workspace=ws, stream=stream, distinct=args.distinct)
             for k in res_host:

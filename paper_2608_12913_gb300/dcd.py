@@ -420,3 +420,37 @@ def dcd_get_device_error(workspace: torch.Tensor, stream=None) -> int:
 
 def version() -> int:
     return int(load().dcd_version())
+
+
+def sampled_row_ranges(temperature: torch.Tensor, N: int) -> list:
+    """Row ranges [start, stop) of the sequences with a positive temperature (sequence b owns rows
+    b*N .. b*N+N-1), adjacent sequences merged.  The kernels read q only in these rows."""
+    t = temperature.detach().to("cpu").reshape(-1)
+    ranges = []
+    for b in range(t.numel()):
+        if float(t[b]) > 0.0:
+            if ranges and ranges[-1][1] == b * N:
+                ranges[-1][1] = (b + 1) * N
+            else:
+                ranges.append([b * N, (b + 1) * N])
+    return [tuple(r) for r in ranges]
+
+
+def upload_inputs(host: dict, dst: dict, N: int, stream=None) -> int:
+    """Copies one call's inputs from host tensors (pinned, for asynchronous copies) into the
+    matching device tensors on `stream`, and returns the bytes copied.  Every tensor is copied whole
+    except ``q``, of which only the rows of sampled sequences are copied: the verification reads
+    no other row of q, so the rows of greedy sequences may hold anything on the device.  `host`
+    must hold ``temperature`` when it holds ``q``."""
+    stream = stream if stream is not None else torch.cuda.current_stream()
+    nbytes = 0
+    with torch.cuda.stream(stream):
+        for k, h in host.items():
+            if k == "q" and h is not None:
+                for r0, r1 in sampled_row_ranges(host["temperature"], N):
+                    dst[k][r0:r1].copy_(h[r0:r1], non_blocking=True)
+                    nbytes += (r1 - r0) * h.shape[1] * h.element_size()
+            elif h is not None:
+                dst[k].copy_(h, non_blocking=True)
+                nbytes += h.numel() * h.element_size()
+    return nbytes

@@ -161,3 +161,11 @@ def test_diagnostics_workspace_and_host_checks(lib):
     assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, P, ws, 16, None) == -7
     empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
     assert lib.dcd_row_diagnostics(ctypes.byref(empty), P, P, None, None, P, ws, 1 << 20, None) == 0
+
+
+def test_sampled_row_ranges_merges_adjacent_sequences():
+    import torch
+    from paper_2608_12913_gb300 import dcd
+    t = torch.tensor([0.0, 1.0, 0.7, 0.0, 2.0])
+    assert dcd.sampled_row_ranges(t, 4) == [(4, 12), (16, 20)]
+    assert dcd.sampled_row_ranges(torch.zeros(3), 4) == []
