@@ -55,8 +55,13 @@
  *   16384 vocabulary tokens (bf16 logits; 8192 for fp32), rounded up to 256; its
  *   contents need no initialisation).  Calls are asynchronous and ordered on
  *   `stream`; host-side argument checks return a negative status before anything is
- *   launched.  Two
- *   calls that share a workspace must not overlap on the device.
+ *   launched.  Two calls that share a workspace must not overlap on the device.
+ * - Vocabulary limit: the streaming kernel keeps 8 bytes per 1024 vocabulary tokens
+ *   (per 512 with fp32 logits) of the row in flight in shared memory, next to its
+ *   64 KB ring.  A shape for which that does not fit in a CTA's 227 KB -- V above
+ *   about 18 million tokens with bf16 logits, 9 million with fp32, at N = 1024; a
+ *   little more for smaller trees -- returns DCD_ERR_UNSUPPORTED (the one-launch
+ *   greedy path of small calls has no such limit).
  * - Thread safety: entry points may be called from several host threads, each with
  *   its own workspace.
  */
@@ -114,7 +119,7 @@ enum { DCD_F32 = 0, DCD_BF16 = 1 };
 typedef struct {
   int32_t B;            /* sequences (>= 0) */
   int32_t N;            /* nodes per sequence, root included (1 .. DCD_MAX_NODES) */
-  int64_t V;            /* vocabulary size (1 .. 2^31 - 1) */
+  int64_t V;            /* vocabulary size (1 .. 2^31 - 1; see the shared-memory limit below) */
   int32_t logits_dtype; /* DCD_F32 or DCD_BF16, for z_exp and z_ama */
   int32_t flags;        /* 0, or DCD_SIBLINGS_DISTINCT (sampled calls); other bits must be 0 */
   int64_t ld_logits;    /* row stride of z_exp / z_ama in elements (>= V) */

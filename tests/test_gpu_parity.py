@@ -52,6 +52,28 @@ def test_config3_reduced_mixed_batch():
     compare(w, g, r, check_residual=True)
 
 
+def test_wide_vocabulary_mixed_batch():
+    # a 262K vocabulary (ragged: not a multiple of a stage, a race block or a residual piece)
+    w = workloads.make_config(3, B=2, V=262147, seed=43, margin_fn=oracle.margin_fn)
+    g = run_gpu(w, sampled=True, residual=True)
+    r = _oracle(w, residual=True)
+    compare(w, g, r, check_residual=True)
+
+
+def test_vocabulary_beyond_shared_memory_is_unsupported():
+    # the row kernel keeps 8 bytes per 1024 vocabulary tokens of a row in shared memory; a
+    # vocabulary past that returns DCD_ERR_UNSUPPORTED before any launch
+    V = 1 << 25
+    z = torch.zeros((2, V), dtype=torch.bfloat16, device="cuda")
+    q = torch.full((2, V), 1.0 / V, dtype=torch.float32, device="cuda")
+    tokens = torch.tensor([[0, 1]], dtype=torch.int32, device="cuda")
+    parents = torch.tensor([[-1, 0]], dtype=torch.int32, device="cuda")
+    one = torch.ones(1, dtype=torch.float32, device="cuda")
+    with pytest.raises(dcd.DcdError) as e:
+        dcd.dcd_verify_sample(z, z, q, tokens, parents, one * 0.1, one, 1, 0)
+    assert e.value.status == -3
+
+
 def test_config3_full_size_sampled_sequences():
     """The 32 x 60-node, V = 128256 batch in the launch configuration the benchmark times;
     the oracle recomputes 8 of its sequences (4 greedy, 4 sampled) one by one."""
