@@ -51,9 +51,10 @@
  *   s'(x) / T_eff - cd_lse[g]); T_eff = T, or 1 for greedy sequences.
  * - Memory: every array pointer is a DEVICE pointer owned by the caller.  The
  *   library allocates nothing per call; scratch lives in the caller's workspace
- *   (dcd_workspace_bytes: 256 bytes plus, per row, 96 bytes and 16 bytes per
- *   16384 vocabulary tokens (bf16 logits; 8192 for fp32), rounded up to 256; its
- *   contents need no initialisation).  Calls are asynchronous and ordered on
+ *   (dcd_workspace_bytes: 256 bytes plus, per row, 532 bytes and 16 bytes per
+ *   residual piece -- a piece covers 16384 vocabulary tokens with bf16 logits, 8192
+ *   with fp32, half that in calls of at most 256 rows -- rounded up to 256; 660 bytes
+ *   a row at V = 128256 in bf16; its contents need no initialisation).  Calls are asynchronous and ordered on
  *   `stream`; host-side argument checks return a negative status before anything is
  *   launched.  Two calls that share a workspace must not overlap on the device.
  * - Vocabulary limit: the streaming kernel keeps 8 bytes per 1024 vocabulary tokens
