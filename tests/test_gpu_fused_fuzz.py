@@ -1,0 +1,44 @@
+"""A seeded sweep of random shapes for the fused LM-head step against the oracle (which forms
+the logits h W^T in fp64).  Each case draws from its own fixed seed the batch (every fourth case
+30-50 sequences, several row tiles), the tree, a vocabulary of 8 to 20000 tokens (ragged tiles),
+the hidden sizes (multiples of 8 up to 2048 and 1024: K tails), per-sequence alpha and, in half
+the cases, a plausibility threshold.  Bars as in test_gpu_fused.py."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_12913_gb300 import workloads
+from parity_util import FUSED_AMB_MASK, FUSED_SCORE_TOL, compare, run_fused_gpu
+
+pytestmark = pytest.mark.gpu
+
+N_CASES = 24
+
+
+def _case(i):
+    rng = np.random.default_rng(11000 + i)
+    levels = tuple([1] + [int(rng.integers(1, 9)) for _ in range(int(rng.integers(1, 5)))])
+    B = int(rng.integers(30, 51)) if i % 4 == 3 else int(rng.integers(1, 7))
+    V = int(rng.choice([8, 255, 256, 257, 4099, int(rng.integers(8, 20001))]))
+    beta = float(rng.choice([0.0, 0.1, 0.5])) if i % 2 else 0.0
+    spec = dict(B=B, V=V, H_exp=8 * int(rng.integers(1, 257)), H_ama=8 * int(rng.integers(1, 129)),
+                seed=12000 + i, levels=levels, beta=beta, w_std=0.12 if beta > 0 else None)
+    alphas = rng.choice([0.0, 0.05, 0.1, 0.5, 1.0], size=B).astype(np.float32)
+    return spec, alphas
+
+
+@pytest.mark.parametrize("i", range(N_CASES))
+def test_random_fused_case_matches_oracle(i):
+    spec, alphas = _case(i)
+    w = workloads.make_fused_torch(**spec)
+    w.alpha = torch.from_numpy(alphas).to(w.h_exp.device)
+    if spec["beta"] > 0:
+        gpu = run_fused_gpu(w, beta=w.beta)
+        ref = oracle.verify_fused_workload(w, nthreads=oracle.max_threads())
+        compare(w, gpu, ref, amb_mask=FUSED_AMB_MASK, max_amb_frac=0.5, score_tol=FUSED_SCORE_TOL)
+    else:
+        gpu = run_fused_gpu(w)
+        ref = oracle.verify_fused_workload(w, nthreads=oracle.max_threads())
+        compare(w, gpu, ref, max_amb_frac=0.34)
