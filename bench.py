@@ -335,7 +335,11 @@ def run_ours(args):
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    # The row kernel's own duration is sampled on every 16th step: an event between the two
+    # launches breaks the tree walk's programmatic dependent launch, so the other steps run as a
+    # user's back-to-back calls do.
+    sampled_steps = list(range(0, args.steps, 16))
+    evs = {k: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for k in sampled_steps}
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
@@ -343,7 +347,7 @@ def run_ours(args):
     t_wall0 = time.time()
     start.record(stream)
     for k in range(args.steps):
-        step(1_000_000 + k, evs[k])
+        step(1_000_000 + k, evs.get(k))
     stop.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -351,7 +355,7 @@ def run_ours(args):
     t_wall1 = time.time()
     sampler.stop()
     elapsed_ms = start.elapsed_time(stop)
-    row_ms = [a.elapsed_time(b) for a, b in evs]
+    row_ms = [a.elapsed_time(b) for a, b in evs.values()]
     if world > 1:
         elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
     if dcd.dcd_get_device_error(ws) != 0:
@@ -368,11 +372,12 @@ def run_ours(args):
     achieved = alg / row_avg_s / 1e9
     peak, peak_kind = _peaks()
     khash = _kernel_source_hash()
-    traffic = _profiled_traffic(khash)
+    # the profile covers the default workload (32 sequences, mixed, i.i.d. siblings) only
+    traffic = _profiled_traffic(khash) if B == 32 and not args.greedy and not args.distinct else None
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": traffic, "kernel": "score_rows_kernel", "peak_source": f"{peak_kind} hbm_gbs",
                 "algorithmic_bytes_per_launch": alg, "residual_rows_per_step": res_rows,
-                "row_kernel_ms": row_avg_s * 1e3,
+                "row_kernel_ms": row_avg_s * 1e3, "row_kernel_samples": len(row_ms),
                 "kernel_source_sha256_16": khash}
 
     # end to end through the public API: pinned host inputs -> device, verify, results -> host
@@ -625,8 +630,12 @@ def run_diagnostics(args):
         for _ in range(32):
             step()
         torch.cuda.synchronize()
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-    for e in evs:  # create the events outside the timed region
+    # the pass's own duration is sampled on every 16th step: events between the pass and the
+    # combine break the combine's programmatic dependent launch, so the other steps run as a
+    # user's back-to-back calls do
+    evs = {k: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for k in range(0, steps, 16)}
+    for e in evs.values():  # create the events outside the timed region
         e[0].record(stream)
         e[1].record(stream)
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -636,7 +645,7 @@ def run_diagnostics(args):
     t_wall0 = time.time()
     start.record(stream)
     for k in range(steps):
-        step(evs[k])
+        step(evs.get(k))
     stop.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -644,7 +653,7 @@ def run_diagnostics(args):
     t_wall1 = time.time()
     sampler.stop()
     elapsed_ms = start.elapsed_time(stop)
-    pass_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+    pass_ms = statistics.mean(a.elapsed_time(b) for a, b in evs.values())
     if world > 1:
         elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
     if not torch.isfinite(diag).all():
@@ -656,9 +665,11 @@ def run_diagnostics(args):
     achieved = alg / (pass_ms / 1e3) / 1e9
     khash = _kernel_source_hash(("dcd_diag.cu", "dcd_diag.h", "dcd_device.cuh"))
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                "traffic": _profiled_traffic(khash, "diag_partial_kernel_B32_tree60_V128256.md"),
+                "traffic": (_profiled_traffic(khash, "diag_partial_kernel_B32_tree60_V128256.md")
+                            if B == 32 else None),
                 "kernel": "diag_partial_kernel", "peak_source": f"{peak_kind} hbm_gbs",
-                "algorithmic_bytes_per_launch": alg, "pass_kernel_ms": pass_ms, "kernel_source_sha256_16": khash}
+                "algorithmic_bytes_per_launch": alg, "pass_kernel_ms": pass_ms,
+                "pass_kernel_samples": len(evs), "kernel_source_sha256_16": khash}
 
     e2e = None
     if not args.no_e2e:
