@@ -422,32 +422,44 @@ def version() -> int:
     return int(load().dcd_version())
 
 
-def sampled_row_ranges(temperature: torch.Tensor, N: int) -> list:
-    """Row ranges [start, stop) of the sequences with a positive temperature (sequence b owns rows
-    b*N .. b*N+N-1), adjacent sequences merged.  The kernels read q only in these rows."""
+def sampled_row_ranges(temperature: torch.Tensor, N: int, parents: Optional[torch.Tensor] = None) -> list:
+    """Row ranges [start, stop), adjacent rows merged, of the rows whose q the kernels read: the
+    rows of sequences with a positive temperature (sequence b owns rows b*N .. b*N+N-1), and of
+    those, when `parents` [B, N] is given, only the rows of nodes with at least one child (a
+    leaf draws its terminal token from pi_CD alone)."""
     t = temperature.detach().to("cpu").reshape(-1)
+    par = None if parents is None else parents.detach().to("cpu").reshape(t.numel(), N)
     ranges = []
     for b in range(t.numel()):
-        if float(t[b]) > 0.0:
-            if ranges and ranges[-1][1] == b * N:
-                ranges[-1][1] = (b + 1) * N
+        if not float(t[b]) > 0.0:
+            continue
+        if par is None:
+            rows = range(b * N, (b + 1) * N)
+        else:
+            has_child = torch.zeros(N, dtype=torch.bool)
+            p = par[b, 1:].long()
+            has_child[p[(p >= 0) & (p < N)]] = True
+            rows = (b * N + n for n in range(N) if bool(has_child[n]))
+        for g in rows:
+            if ranges and ranges[-1][1] == g:
+                ranges[-1][1] = g + 1
             else:
-                ranges.append([b * N, (b + 1) * N])
+                ranges.append([g, g + 1])
     return [tuple(r) for r in ranges]
 
 
 def upload_inputs(host: dict, dst: dict, N: int, stream=None) -> int:
     """Copies one call's inputs from host tensors (pinned, for asynchronous copies) into the
     matching device tensors on `stream`, and returns the bytes copied.  Every tensor is copied whole
-    except ``q``, of which only the rows of sampled sequences are copied: the verification reads
-    no other row of q, so the rows of greedy sequences may hold anything on the device.  `host`
-    must hold ``temperature`` when it holds ``q``."""
+    except ``q``, of which only the rows the verification reads are copied (sampled_row_ranges:
+    rows of sampled sequences whose node has a child); the other rows may hold anything on the
+    device.  `host` must hold ``temperature`` and ``parents`` when it holds ``q``."""
     stream = stream if stream is not None else torch.cuda.current_stream()
     nbytes = 0
     with torch.cuda.stream(stream):
         for k, h in host.items():
             if k == "q" and h is not None:
-                for r0, r1 in sampled_row_ranges(host["temperature"], N):
+                for r0, r1 in sampled_row_ranges(host["temperature"], N, host["parents"]):
                     dst[k][r0:r1].copy_(h[r0:r1], non_blocking=True)
                     nbytes += (r1 - r0) * h.shape[1] * h.element_size()
             elif h is not None:

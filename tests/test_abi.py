@@ -169,3 +169,7 @@ def test_sampled_row_ranges_merges_adjacent_sequences():
     t = torch.tensor([0.0, 1.0, 0.7, 0.0, 2.0])
     assert dcd.sampled_row_ranges(t, 4) == [(4, 12), (16, 20)]
     assert dcd.sampled_row_ranges(torch.zeros(3), 4) == []
+    # with the tree: only nodes that have a child (node 0 of every sequence; node 1 in sequence 1;
+    # node 2 in sequences 2 and 4)
+    par = torch.tensor([[-1, 0, 0, 0], [-1, 0, 1, 1], [-1, 0, 0, 2], [-1, 0, 1, 2], [-1, 0, 0, 2]])
+    assert dcd.sampled_row_ranges(t, 4, par) == [(4, 6), (8, 9), (10, 11), (16, 17), (18, 19)]

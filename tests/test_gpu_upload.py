@@ -1,6 +1,6 @@
-"""The end-to-end upload copies q only for sampled sequences (dcd.upload_inputs).  The kernels
-never read q in the rows of greedy sequences: with those rows NaN on the device, every output
-equals that of a call on fully copied inputs, bit for bit."""
+"""The end-to-end upload copies q only in the rows the verification reads (dcd.upload_inputs:
+rows of sampled sequences whose node has a child).  With every other row NaN on the device,
+every output equals that of a call on fully copied inputs, bit for bit."""
 
 import numpy as np
 import pytest
@@ -21,9 +21,9 @@ def test_upload_copies_only_read_rows_of_q(distinct):
     part = {k: torch.empty_like(v, device="cuda") for k, v in host.items()}
     part["q"].fill_(float("nan"))
     nbytes = dcd.upload_inputs(host, part, w.N)
-    sampled = int((w.temperature > 0).sum())
     expect = sum(v.numel() * v.element_size() for k, v in host.items() if k != "q")
-    assert nbytes == expect + sampled * w.N * w.V * 4
+    read_rows = w.sampled_rows_with_children()  # the rows whose q the rules read
+    assert nbytes == expect + read_rows * w.V * 4
 
     def run(d):
         o = dcd.dcd_verify_sample(d["z_exp"], d["z_ama"], d["q"], d["tokens"], d["parents"], d["alpha"],
