@@ -164,6 +164,30 @@ def alloc_outputs(B: int, N: int, device, V: Optional[int] = None, residual: boo
     return out
 
 
+def _check_outputs(o: dict, B: int, N: int, V: int, device) -> dict:
+    """A caller's output tensors: each must have the dtype, device and shape the library writes, and
+    be contiguous (the library writes them as dense arrays)."""
+    specs = {"accept_len": (torch.int32, (B,)), "accept_path": (torch.int32, (B, N)), "bonus": (torch.int32, (B,)),
+             "cd_logprob": (torch.float32, (B, N)), "cd_argmax": (torch.int32, (B, N)),
+             "cd_lse": (torch.float32, (B, N)), "residual": (torch.float32, (B, V))}
+    for k in ("accept_len", "accept_path", "bonus"):
+        if k not in o:
+            raise ValueError(f"out must hold {k!r}")
+    for k, t in o.items():
+        if k in specs:
+            dtype, shape = specs[k]
+            _require(t, f"out[{k!r}]", dtype, device, shape)
+            if not t.is_contiguous():
+                raise ValueError(f"out[{k!r}] must be contiguous")
+    return o
+
+
+def _require_vec(t, name, B: int, device):
+    _require(t, name, torch.float32, device, (B,))
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
 class _Call:
     """Validated arguments of one verification call."""
 
@@ -185,9 +209,9 @@ class _Call:
         _require(parents, "parents", dtype=torch.int32, device=dev, shape=(B, N))
         if not parents.is_contiguous():
             raise ValueError("parents must be contiguous")
-        _require(alpha, "alpha", dtype=torch.float32, device=dev, shape=(B,))
+        _require_vec(alpha, "alpha", B, dev)
         if beta is not None:
-            _require(beta, "beta", dtype=torch.float32, device=dev, shape=(B,))
+            _require_vec(beta, "beta", B, dev)
         ldq = None
         if q is not None:
             _require(q, "q", dtype=torch.float32, device=dev)
@@ -195,7 +219,7 @@ class _Call:
                 raise ValueError("q must be a [B*N, V] float32 tensor with unit stride along the vocabulary")
             ldq = q.stride(0)
         if temperature is not None:
-            _require(temperature, "temperature", dtype=torch.float32, device=dev, shape=(B,))
+            _require_vec(temperature, "temperature", B, dev)
         self.device = dev
         self.B, self.N, self.V = B, N, V
         self.shape = make_shape(B, N, V, _logits_dtype(z_exp), z_exp.stride(0), ldq,
@@ -214,7 +238,7 @@ class _Call:
     def outputs(self, out, residual=False):
         if out is None:
             return alloc_outputs(self.B, self.N, self.device, self.V, residual)
-        return out
+        return _check_outputs(out, self.B, self.N, self.V, self.device)
 
 
 def dcd_verify_greedy(z_exp, z_ama, tokens, parents, alpha, beta=None, *, out=None, workspace=None,
@@ -315,11 +339,12 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
     Returns accept_len, accept_path, bonus, cd_logprob, cd_argmax, cd_lse (and the workspace).
     `gemm_events` = (start, stop) torch.cuda.Event pair recorded around the tensor-core sweeps.
     """
+    _require(h_exp, "h_exp", dtype=torch.bfloat16)
+    dev = h_exp.device
     for t, name in ((h_exp, "h_exp"), (w_exp, "w_exp"), (h_ama, "h_ama"), (w_ama, "w_ama")):
-        _require(t, name, dtype=torch.bfloat16)
+        _require(t, name, dtype=torch.bfloat16, device=dev)
         if t.dim() != 2 or not t.is_contiguous():
             raise ValueError(f"{name} must be a contiguous 2-D tensor")
-    dev = h_exp.device
     B, N = tokens.shape
     R, H_exp = h_exp.shape
     V = w_exp.shape[0]
@@ -327,14 +352,18 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
     if R != B * N or h_ama.shape[0] != R or tuple(w_exp.shape) != (V, H_exp) or tuple(w_ama.shape) != (V, H_ama):
         raise ValueError("inconsistent shapes for the fused LM-head call")
     _require(tokens, "tokens", torch.int32, dev)
+    if tokens.dim() != 2 or not tokens.is_contiguous():
+        raise ValueError("tokens must be a contiguous [B, N] int32 tensor")
     _require(parents, "parents", torch.int32, dev, (B, N))
-    _require(alpha, "alpha", torch.float32, dev, (B,))
+    if not parents.is_contiguous():
+        raise ValueError("parents must be contiguous")
+    _require_vec(alpha, "alpha", B, dev)
     if beta is not None:
-        _require(beta, "beta", torch.float32, dev, (B,))
+        _require_vec(beta, "beta", B, dev)
     sh = make_shape(B, N, V, DCD_BF16)
     if workspace is None:
         workspace = torch.empty(fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
-    o = alloc_outputs(B, N, dev) if out is None else out
+    o = alloc_outputs(B, N, dev) if out is None else _check_outputs(out, B, N, V, dev)
     ev0 = ev1 = None
     if gemm_events is not None:
         for e in gemm_events:
@@ -397,6 +426,8 @@ def dcd_row_diagnostics(z_exp, z_ama, B: int, N: int, *, q=None, xstar=None, out
         out = torch.empty(R, 6, dtype=torch.float32, device=dev)
     else:
         _require(out, "out", torch.float32, dev, (R, 6))
+        if not out.is_contiguous():
+            raise ValueError("out must be contiguous")
     ev0 = ev1 = None
     if pass_events is not None:
         for e in pass_events:

@@ -268,3 +268,26 @@ def test_largest_tree_chain_of_max_nodes():
         gpu = run_gpu(w, sampled=temp > 0)
         ref = oracle.verify_workload(w, nthreads=oracle.max_threads())
         compare(w, gpu, ref)
+
+
+def test_binding_rejects_outputs_and_vectors_it_cannot_write_or_read():
+    # checked on the host, before any launch: a wrong output shape would let a kernel write past
+    # the caller's tensor, a strided parameter vector would be read as dense
+    w = workloads.make_config(1, B=2, V=1000, seed=51).to("cuda")
+    out = dcd.alloc_outputs(w.B, w.N, "cuda")
+    bad = dict(out, accept_path=torch.empty((w.B, w.N - 1), dtype=torch.int32, device="cuda"))
+    with pytest.raises(ValueError):
+        dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, out=bad)
+    bad = dict(out, cd_lse=torch.empty((w.B, w.N), dtype=torch.float64, device="cuda"))
+    with pytest.raises(TypeError):
+        dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, out=bad)
+    bad = {k: v for k, v in out.items() if k != "bonus"}
+    with pytest.raises(ValueError):
+        dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, out=bad)
+    strided = torch.zeros(2 * w.B, dtype=torch.float32, device="cuda")[::2]
+    with pytest.raises(ValueError):
+        dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, strided, w.beta, out=out)
+    o = dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, out=out)
+    torch.cuda.synchronize()
+    assert o["accept_len"] is out["accept_len"]
+
