@@ -223,6 +223,27 @@ int dcd_verify_sample_noalloc(const dcd_shape* shape, const void* z_exp, const v
                               int32_t* cd_argmax, float* cd_lse, float* residual, dcd_stream_t stream);
 
 /*
+ * Staging of a sampled call's draft distributions from host memory: copies into q_dev the
+ * rows of q_host that dcd_verify_sample reads -- the rows of sequences with a positive
+ * temperature whose node has at least one child (the sibling test reads q at the
+ * children's tokens and a residual pass the whole row, Algorithm 1; a leaf draws its
+ * terminal token from pi_CD alone).  Every other row of q_dev keeps its contents.
+ *   shape       : B, N, V and ld_q (the row stride, in floats, of both q_host and q_dev;
+ *                 >= V); logits_dtype and ld_logits as for dcd_verify_sample.
+ *   q_host      : fp32 [B*N, ld_q] in page-locked host memory mapped into the device's
+ *                 address space (cudaHostAlloc, or cudaHostRegister with the mapped flag);
+ *                 the GPU reads it directly, in one launch, at the host link's rate.
+ *   q_dev       : fp32 [B*N, ld_q] device memory.
+ *   parents, temperature : the call's DEVICE arrays as for dcd_verify_sample (already on
+ *                 the device: the copy is ordered after them on `stream`).
+ * Returns DCD_ERR_INVALID_ARG for a bad shape, a null pointer, or a q_host whose first or
+ * last element is not mapped page-locked host memory (nothing is launched).  Asynchronous
+ * on `stream`; the caller keeps q_host unchanged until the copy completes.
+ */
+int dcd_upload_q_rows(const dcd_shape* shape, const float* q_host, float* q_dev, const int32_t* parents,
+                      const float* temperature, dcd_stream_t stream);
+
+/*
  * dcd_score_rows with an explicit launch geometry, for tests and tuning: `stages` is
  * the depth of each CTA's ring of shared-memory stages (0 = automatic, else 2 .. 8)
  * and `plain_loads` = 1 stages rows with ordinary loads instead of bulk asynchronous

@@ -203,6 +203,26 @@ int dcd_verify_sample(const dcd_shape* shape, const void* z_exp, const void* z_a
                                                    reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int dcd_upload_q_rows(const dcd_shape* shape, const float* q_host, float* q_dev, const int32_t* parents,
+                      const float* temperature, dcd_stream_t stream) {
+  if (!shape_ok(shape, true)) return DCD_ERR_INVALID_ARG;
+  if (shape->B == 0) return DCD_OK;
+  if (!q_host || !q_dev || !parents || !temperature) return DCD_ERR_INVALID_ARG;
+  // the first and the last element read must be page-locked host memory mapped into the device
+  const int64_t R = static_cast<int64_t>(shape->B) * shape->N;
+  const float* last = q_host + (R - 1) * shape->ld_q + (shape->V - 1);
+  cudaPointerAttributes a0, a1;
+  if (cudaPointerGetAttributes(&a0, q_host) != cudaSuccess || cudaPointerGetAttributes(&a1, last) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return DCD_ERR_INVALID_ARG;
+  }
+  if (a0.type != cudaMemoryTypeHost || a1.type != cudaMemoryTypeHost || !a0.devicePointer || !a1.devicePointer)
+    return DCD_ERR_INVALID_ARG;
+  return cuda_status(dcd::launch_upload_q_rows(shape->B, shape->N, shape->V, shape->ld_q,
+                                               static_cast<const float*>(a0.devicePointer), q_dev, parents,
+                                               temperature, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 size_t dcd_fused_workspace_bytes(const dcd_shape* s) {
   if (!s || s->B < 0 || s->N < 1 || s->V < 1 || s->V > INT_MAX || s->flags != 0) return 0;
   if (s->logits_dtype != DCD_BF16) return 0;

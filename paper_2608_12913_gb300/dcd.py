@@ -67,6 +67,8 @@ def load(build_if_missing: bool = True):
         lib.dcd_score_rows_ex.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P,
                                           ctypes.c_int, ctypes.c_int]
         lib.dcd_tree_walk.argtypes = [SH, P, P, P, P, SZ, P]
+        lib.dcd_upload_q_rows.argtypes = [SH, P, P, P, P, P]
+        lib.dcd_upload_q_rows.restype = I32
         lib.dcd_fused_workspace_bytes.argtypes = [SH]
         lib.dcd_fused_workspace_bytes.restype = SZ
         lib.dcd_verify_fused_lmhead.argtypes = [SH, P, I32, P, P, I32, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
@@ -489,11 +491,24 @@ def upload_inputs(host: dict, dst: dict, N: int, stream=None) -> int:
     nbytes = 0
     with torch.cuda.stream(stream):
         for k, h in host.items():
-            if k == "q" and h is not None:
-                for r0, r1 in sampled_row_ranges(host["temperature"], N, host["parents"]):
-                    dst[k][r0:r1].copy_(h[r0:r1], non_blocking=True)
-                    nbytes += (r1 - r0) * h.shape[1] * h.element_size()
-            elif h is not None:
+            if k != "q" and h is not None:
                 dst[k].copy_(h, non_blocking=True)
                 nbytes += h.numel() * h.element_size()
+    h = host.get("q")
+    if h is not None:
+        ranges = sampled_row_ranges(host["temperature"], N, host["parents"])
+        nbytes += sum(r1 - r0 for r0, r1 in ranges) * h.shape[1] * h.element_size()
+        d = dst["q"]
+        if h.is_pinned() and h.dim() == 2 and h.stride(1) == 1 and d.stride() == h.stride():
+            # one launch: the SMs read the rows through the pinned buffer's device mapping (after
+            # parents and temperature, copied above on the same stream)
+            B = host["temperature"].numel()
+            sh = make_shape(B, N, h.shape[1], DCD_BF16, ldq=h.stride(0))
+            st = load().dcd_upload_q_rows(ctypes.byref(sh), ctypes.c_void_p(h.data_ptr()), _ptr(d),
+                                          _ptr(dst["parents"]), _ptr(dst["temperature"]), _stream(stream))
+            _check(st, "dcd_upload_q_rows")
+        else:
+            with torch.cuda.stream(stream):
+                for r0, r1 in ranges:
+                    d[r0:r1].copy_(h[r0:r1], non_blocking=True)
     return nbytes

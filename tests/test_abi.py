@@ -108,6 +108,12 @@ def test_host_checks_reject_before_launch(lib):
     # empty batch is a no-op
     empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
     assert lib.dcd_verify_greedy(ctypes.byref(empty), *base, ws_ok, 1 << 20, None) == 0
+    # q staging: null pointers, a short row stride, an empty batch
+    assert lib.dcd_upload_q_rows(ctypes.byref(sh), None, P, P, P, None) == -1
+    assert lib.dcd_upload_q_rows(ctypes.byref(sh), P, P, None, P, None) == -1
+    short = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, ldq=50)
+    assert lib.dcd_upload_q_rows(ctypes.byref(short), P, P, P, P, None) == -1
+    assert lib.dcd_upload_q_rows(ctypes.byref(empty), P, P, P, P, None) == 0
 
 
 def test_binding_refuses_cpu_tensors():
