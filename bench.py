@@ -335,10 +335,10 @@ def run_ours(args):
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
-    # The row kernel's own duration is sampled on every 16th step: an event between the two
-    # launches breaks the tree walk's programmatic dependent launch, so the other steps run as a
-    # user's back-to-back calls do.
-    sampled_steps = list(range(0, args.steps, 16))
+    # The row kernel's own duration is sampled on every 8th step (the median is reported): an
+    # event between the two launches breaks the tree walk's programmatic dependent launch, so the
+    # other steps run as a user's back-to-back calls do.
+    sampled_steps = list(range(0, args.steps, 8))
     evs = {k: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for k in sampled_steps}
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
@@ -368,7 +368,7 @@ def run_ours(args):
     replay = [1_000_000 + k for k in range(0, args.steps, 32)]
     res_rows = residual_rows_per_step(w, out, ws, stream, replay, args.distinct)
     alg = algorithmic_bytes(w, res_rows)
-    row_avg_s = statistics.mean(row_ms) / 1e3
+    row_avg_s = statistics.median(row_ms) / 1e3
     achieved = alg / row_avg_s / 1e9
     peak, peak_kind = _peaks()
     khash = _kernel_source_hash()
@@ -630,11 +630,11 @@ def run_diagnostics(args):
         for _ in range(32):
             step()
         torch.cuda.synchronize()
-    # the pass's own duration is sampled on every 16th step: events between the pass and the
-    # combine break the combine's programmatic dependent launch, so the other steps run as a
-    # user's back-to-back calls do
+    # the pass's own duration is sampled on every 8th step (the median is reported): events between
+    # the pass and the combine break the combine's programmatic dependent launch, so the other
+    # steps run as a user's back-to-back calls do
     evs = {k: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for k in range(0, steps, 16)}
+           for k in range(0, steps, 8)}
     for e in evs.values():  # create the events outside the timed region
         e[0].record(stream)
         e[1].record(stream)
@@ -653,7 +653,7 @@ def run_diagnostics(args):
     t_wall1 = time.time()
     sampler.stop()
     elapsed_ms = start.elapsed_time(stop)
-    pass_ms = statistics.mean(a.elapsed_time(b) for a, b in evs.values())
+    pass_ms = statistics.median(a.elapsed_time(b) for a, b in evs.values())
     if world > 1:
         elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
     if not torch.isfinite(diag).all():

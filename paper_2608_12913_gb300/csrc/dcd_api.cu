@@ -10,6 +10,7 @@
 #include "dcd_diag.h"
 #include "dcd_fused.h"
 #include "dcd_internal.h"
+#include "dcd_upload.h"
 #include "dcd_small.h"
 
 namespace {

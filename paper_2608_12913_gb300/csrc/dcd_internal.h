@@ -128,9 +128,6 @@ size_t slot_bytes(int64_t V, int dtype, int64_t rows);
 
 cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream);
 
-cudaError_t launch_upload_q_rows(int32_t B, int32_t N, int64_t V, int64_t ldq, const float* src_dev_view, float* dst,
-                                 const int32_t* parents, const float* temperature, cudaStream_t stream);
-
 cudaError_t launch_tree_walk(int32_t B, int32_t N, const RowRecord* rec, uint32_t* err, int32_t* accept_len,
                              int32_t* accept_path, int32_t* bonus, cudaStream_t stream);
 

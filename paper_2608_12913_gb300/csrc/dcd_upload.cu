@@ -11,7 +11,7 @@
 #include <stdint.h>
 
 #include "dcd.h"
-#include "dcd_internal.h"
+#include "dcd_upload.h"
 
 namespace dcd {
 namespace {
