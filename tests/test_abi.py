@@ -179,3 +179,21 @@ def test_sampled_row_ranges_merges_adjacent_sequences():
     # node 2 in sequences 2 and 4)
     par = torch.tensor([[-1, 0, 0, 0], [-1, 0, 1, 1], [-1, 0, 0, 2], [-1, 0, 1, 2], [-1, 0, 0, 2]])
     assert dcd.sampled_row_ranges(t, 4, par) == [(4, 6), (8, 9), (10, 11), (16, 17), (18, 19)]
+
+
+def test_header_is_plain_c(tmp_path):
+    """include/dcd.h is a C header: a C99 translation unit using it compiles with -pedantic."""
+    import shutil
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "use_dcd.c"
+    src.write_text('#include "dcd.h"\n'
+                   "int main(void) {\n"
+                   "  dcd_shape s = {1, 6, 32000, DCD_F32, 0, 32000, 32000};\n"
+                   "  return dcd_workspace_bytes(&s) == 0;\n"
+                   "}\n")
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", inc, "-fsyntax-only",
+                        str(src)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
