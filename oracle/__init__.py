@@ -92,7 +92,8 @@ def _load():
             lib.dcd_oracle_verify.argtypes = [I32, I32, I64, ctypes.c_int, I64, P, P, P, P, P, P, P, P, I64,
                                               U64, U64, P, ctypes.c_int, ctypes.c_int, P, P, P, P, P, P]
             lib.dcd_oracle_max_threads.restype = ctypes.c_int
-            lib.dcd_oracle_row_diagnostics.argtypes = [I64, ctypes.c_int, P, P, P, ctypes.c_int32, P]
+            lib.dcd_oracle_row_diagnostics.argtypes = [I64, ctypes.c_int, P, P, P, ctypes.c_int32, ctypes.c_double,
+                                                       P]
             _lib = lib
     return _lib
 
@@ -291,15 +292,18 @@ def verify_fused_workload(w, nthreads: int = 1, seqs=None) -> dict:
                   beta=beta, temperature=None, nthreads=nthreads, seq_ids=np.asarray(sel))
 
 
-def row_diagnostics(zp, zq, xstar: int, q=None, dtype: str = "f64") -> dict:
-    """Per-row diagnostics (see dcd_oracle_row_diagnostics): lse_p, lse_q, signal at x*, e_q, and
-    with the drafter's distribution q: e_e and kl_e_p."""
+def row_diagnostics(zp, zq, xstar: int, q=None, dtype: str = "f64", alpha=None) -> dict:
+    """Per-row diagnostics (see dcd_oracle_row_diagnostics): lse_p, lse_q, signal at x*, e_q,
+    kl_p_q = D_KL(pi_p || pi_q); with the drafter's distribution q: e_e and kl_e_p; with the
+    contrast strength alpha: kl_p_cd = D_KL(pi_p || pi_CD) of the untruncated T = 1 target."""
     zp = _logits(zp, dtype)
     zq = _logits(zq, dtype)
     V = zp.shape[-1]
     qq = None if q is None else np.ascontiguousarray(q, dtype=np.float32)
-    out = np.empty(6, dtype=np.float64)
-    rc = _load().dcd_oracle_row_diagnostics(V, DTYPE_CODE[dtype], _ptr(zp), _ptr(zq), _ptr(qq), int(xstar), _ptr(out))
+    out = np.empty(8, dtype=np.float64)
+    a = -1.0 if alpha is None else float(alpha)
+    rc = _load().dcd_oracle_row_diagnostics(V, DTYPE_CODE[dtype], _ptr(zp), _ptr(zq), _ptr(qq), int(xstar), a,
+                                            _ptr(out))
     if rc != 0:
         raise ValueError(f"oracle row_diagnostics failed: {rc}")
-    return dict(zip(("lse_p", "lse_q", "signal", "e_q", "e_e", "kl_e_p"), out))
+    return dict(zip(("lse_p", "lse_q", "signal", "e_q", "e_e", "kl_e_p", "kl_p_q", "kl_p_cd"), out))

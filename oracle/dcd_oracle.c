@@ -611,16 +611,21 @@ int dcd_oracle_max_threads(void) {
 
 /*
  * Diagnostics of one row (the quantities of the paper's signal--proposal-error diagnostic,
- * Sec. 3.1, and of its alignment-gap estimator, App. C), in fp64 from the exact inputs:
+ * Sec. 3.1, of its alignment-gap estimator, App. C, and of the KL decomposition of App. B), in
+ * fp64 from the exact inputs:
  *   lse_p, lse_q : log sum_x exp(z_p(x)), log sum_x exp(z_q(x)) (full vocabulary);
  *   signal       : |log pi_p(x*) - log pi_q(x*)| at the given token x* (the CD argmax);
  *   e_q          : E_{pi_q}[log pi_p - log pi_q];
  *   e_e, kl_e_p  : with the drafter's distribution pi_e = q (q may be NULL): E_{pi_e}[log pi_p -
- *                  log pi_q] and D_KL(pi_e || pi_p), with 0 log 0 = 0.
- * out[6] = {lse_p, lse_q, signal, e_q, e_e, kl_e_p} (the last two NaN without q).
+ *                  log pi_q] and D_KL(pi_e || pi_p), with 0 log 0 = 0;
+ *   kl_p_q       : D_KL(pi_p || pi_q) = E_{pi_p}[log pi_p - log pi_q];
+ *   kl_p_cd      : D_KL(pi_p || pi_CD) for the untruncated, untempered target of Eq. 1,
+ *                  pi_CD proportional to pi_p^(1 + alpha) pi_q^(-alpha) over the whole vocabulary,
+ *                  summed term by term from that definition (NaN when alpha < 0: not requested).
+ * out[8] = {lse_p, lse_q, signal, e_q, e_e, kl_e_p, kl_p_q, kl_p_cd} (e_e, kl_e_p NaN without q).
  */
 int dcd_oracle_row_diagnostics(int64_t V, int dtype, const void* zp, const void* zq, const float* q, int32_t xstar,
-                               double* out) {
+                               double alpha, double* out) {
   if (V <= 0 || !zp || !zq || !out || xstar < 0 || xstar >= V) return ORC_ERR_ARG;
   double mp = -INFINITY, mq = -INFINITY;
   for (int64_t x = 0; x < V; ++x) {
@@ -634,14 +639,37 @@ int dcd_oracle_row_diagnostics(int64_t V, int dtype, const void* zp, const void*
     sq += exp(logit_at(zq, dtype, x) - mq);
   }
   const double lse_p = mp + log(sp), lse_q = mq + log(sq);
-  double e_q = 0.0, e_e = 0.0, kl = 0.0;
+  double e_q = 0.0, e_e = 0.0, kl = 0.0, kl_pq = 0.0;
   for (int64_t x = 0; x < V; ++x) {
     const double lp = logit_at(zp, dtype, x) - lse_p, lq = logit_at(zq, dtype, x) - lse_q;
     e_q += exp(lq) * (lp - lq);
+    kl_pq += exp(lp) * (lp - lq);
     if (q) {
       const double e = (double)q[x];
       e_e += e * (lp - lq);
       if (e > 0.0) kl += e * (log(e) - lp);
+    }
+  }
+  double kl_cd = NAN;
+  if (alpha >= 0.0) {
+    /* log pi_CD(x) = (1 + alpha) lp(x) - alpha lq(x) - log Z_CD (Eq. 1 with beta = 0, T = 1) */
+    double ms = -INFINITY;
+    for (int64_t x = 0; x < V; ++x) {
+      const double lp = logit_at(zp, dtype, x) - lse_p, lq = logit_at(zq, dtype, x) - lse_q;
+      const double sc = (1.0 + alpha) * lp - alpha * lq;
+      if (sc > ms) ms = sc;
+    }
+    double ss = 0.0;
+    for (int64_t x = 0; x < V; ++x) {
+      const double lp = logit_at(zp, dtype, x) - lse_p, lq = logit_at(zq, dtype, x) - lse_q;
+      ss += exp((1.0 + alpha) * lp - alpha * lq - ms);
+    }
+    const double log_z = ms + log(ss);
+    kl_cd = 0.0;
+    for (int64_t x = 0; x < V; ++x) {
+      const double lp = logit_at(zp, dtype, x) - lse_p, lq = logit_at(zq, dtype, x) - lse_q;
+      const double lcd = (1.0 + alpha) * lp - alpha * lq - log_z;
+      kl_cd += exp(lp) * (lp - lcd);
     }
   }
   out[0] = lse_p;
@@ -650,5 +678,7 @@ int dcd_oracle_row_diagnostics(int64_t V, int dtype, const void* zp, const void*
   out[3] = e_q;
   out[4] = q ? e_e : NAN;
   out[5] = q ? kl : NAN;
+  out[6] = kl_pq;
+  out[7] = kl_cd;
   return ORC_OK;
 }

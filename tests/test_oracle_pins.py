@@ -643,3 +643,27 @@ def test_row_diagnostics_closed_forms():
     self_kl = oracle.row_diagnostics(zp, zq, x, q=np.exp(lp).astype(np.float32))["kl_e_p"]
     assert abs(self_kl) < 1e-6
     assert np.isnan(oracle.row_diagnostics(zp, zq, x)["e_e"])
+    assert np.isnan(oracle.row_diagnostics(zp, zq, x)["kl_p_cd"])
+
+
+@pytest.mark.parametrize("alpha", [0.0, 0.1, 0.5, 1.5])
+def test_row_diagnostics_kl_columns(alpha):
+    """D_KL(pi_p || pi_q) against scipy's relative entropy; D_KL(pi_p || pi_CD), which the oracle
+    sums term by term from Eq. 1's definition, against scipy's relative entropy of pi_CD =
+    softmax((1 + alpha) log pi_p - alpha log pi_q) and against the decomposition lemma of App. B,
+    D_KL(pi_p || pi_CD) = log Z_CD - alpha D_KL(pi_p || pi_q) with Z_CD = sum pi_p^(1+alpha)
+    pi_q^(-alpha); at alpha = 0 the target is pi_p and the divergence vanishes."""
+    rng = np.random.default_rng(int(alpha * 100) + 5)
+    V = 211
+    zp, zq = _rows(rng, V, scale=2.0)
+    lp, lq = special.log_softmax(zp), special.log_softmax(zq)
+    d = oracle.row_diagnostics(zp, zq, 0, alpha=alpha)
+    pp, pq = np.exp(lp), np.exp(lq)
+    assert abs(d["kl_p_q"] - special.rel_entr(pp, pq).sum()) < 1e-12
+    pcd = special.softmax((1 + alpha) * lp - alpha * lq)
+    assert abs(d["kl_p_cd"] - special.rel_entr(pp, pcd).sum()) < 1e-12
+    log_z = special.logsumexp((1 + alpha) * lp - alpha * lq)
+    assert abs(d["kl_p_cd"] - (log_z - alpha * d["kl_p_q"])) < 1e-12
+    if alpha == 0.0:
+        assert abs(d["kl_p_cd"]) < 1e-14
+    assert d["kl_p_cd"] >= -1e-15 and d["kl_p_q"] >= -1e-15
