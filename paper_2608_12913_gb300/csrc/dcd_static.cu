@@ -10,10 +10,15 @@
 //
 // The array is a file-scope __device__ object, so every GPU that loads the library holds it
 // (DCD_STATIC_SCRATCH_BYTES) until the process exits.  Its host-side name is only a handle:
-// host code must not pass it to a kernel, so its device address is looked up once per device
-// with cudaGetSymbolAddress, with that device current, and cached.
+// host code must not pass it to a kernel, so its device address is looked up with
+// cudaGetSymbolAddress, with the device current, and cached.  The cache is keyed on the device
+// and on the unique id of the context current on it: after cudaDeviceReset (or anything else
+// that creates a new context) the module is loaded again and the array may move, so a new
+// context triggers a new lookup instead of reusing a dead address.
 
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 #include <stdint.h>
 
 #include <mutex>
@@ -26,19 +31,68 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
+struct ScratchCache {
+  unsigned long long ctx_id;  // context the address belongs to (0: none yet)
+  void* addr;
+};
+ScratchCache g_cache[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device (looked up on first use).
+// Driver entry points for the current context and its process-unique id, looked up once through
+// the runtime (no link against the driver library).
+struct CtxFns {
+  PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+  PFN_cuCtxGetId_v12000 get_id = nullptr;
+};
+
+const CtxFns& ctx_fns() {
+  static std::once_flag once;
+  static CtxFns f;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      f.get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      f.get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+  });
+  return f;
+}
+
+// Id of the context current on this thread, 0 if there is none yet.
+int current_ctx_id(unsigned long long* id) {
+  const CtxFns& f = ctx_fns();
+  if (!f.get_current || !f.get_id) return DCD_ERR_CUDA;
+  CUcontext ctx = nullptr;
+  if (f.get_current(&ctx) != CUDA_SUCCESS) return DCD_ERR_CUDA;
+  *id = 0;
+  if (ctx && f.get_id(ctx, id) != CUDA_SUCCESS) return DCD_ERR_CUDA;
+  return DCD_OK;
+}
+
+// Device address of the scratch array in the current device's current context (looked up on the
+// first use in each context).
 int scratch_address(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return DCD_ERR_CUDA;
+  unsigned long long id = 0;
+  int rc = current_ctx_id(&id);
+  if (rc != DCD_OK) return rc;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_addr[dev]) {
+  if (id == 0 || g_cache[dev].ctx_id != id || !g_cache[dev].addr) {
     void* p = nullptr;
+    // also makes the device's primary context current when no context was yet
     if (cudaGetSymbolAddress(&p, g_dcd_static_scratch) != cudaSuccess || !p) return DCD_ERR_CUDA;
-    g_scratch_addr[dev] = p;
+    if (id == 0) {
+      rc = current_ctx_id(&id);
+      if (rc != DCD_OK || id == 0) return DCD_ERR_CUDA;
+    }
+    g_cache[dev].ctx_id = id;
+    g_cache[dev].addr = p;
   }
-  *out = g_scratch_addr[dev];
+  *out = g_cache[dev].addr;
   return DCD_OK;
 }
 
