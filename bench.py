@@ -612,13 +612,14 @@ def run_diagnostics(args):
     stream = torch.cuda.current_stream()
     o = dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, stream=stream)
     xstar = o["cd_argmax"].reshape(-1).contiguous()  # the CD argmax of every node
+    cd_lse = o["cd_lse"].reshape(-1).contiguous()  # its CD normaliser (D_KL(pi_p || pi_CD) by App. B's lemma)
     ws = torch.empty(dcd.diagnostics_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
-    diag = torch.empty(R, 6, dtype=torch.float32, device=dev)
+    diag = torch.empty(R, dcd.DIAG_COLS, dtype=torch.float32, device=dev)
     steps = args.steps
 
     def step(evs=None):
-        dcd.dcd_row_diagnostics(zp, zq, B, N, q=q, xstar=xstar, out=diag, workspace=ws, stream=stream,
-                                pass_events=evs)
+        dcd.dcd_row_diagnostics(zp, zq, B, N, q=q, xstar=xstar, cd_lse=cd_lse, alpha=w.alpha, beta=w.beta, out=diag,
+                                workspace=ws, stream=stream, pass_events=evs)
 
     for _ in range(args.warmup):
         step()
@@ -674,9 +675,9 @@ def run_diagnostics(args):
     e2e = None
     if not args.no_e2e:
         host = {"zp": zp.cpu().pin_memory(), "zq": zq.cpu().pin_memory(), "q": q.cpu().pin_memory(),
-                "xstar": xstar.cpu().pin_memory()}
+                "xstar": xstar.cpu().pin_memory(), "cd_lse": cd_lse.cpu().pin_memory()}
         dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
-        res_host = torch.empty((R, 6), dtype=torch.float32).pin_memory()
+        res_host = torch.empty((R, dcd.DIAG_COLS), dtype=torch.float32).pin_memory()
         h2d = sum(v.numel() * v.element_size() for v in host.values())
         d2h = res_host.numel() * 4
         n_e2e = max(3, min(steps, 10))
@@ -684,8 +685,9 @@ def run_diagnostics(args):
         def e2e_step():
             for k in host:
                 dst[k].copy_(host[k], non_blocking=True)
-            r = dcd.dcd_row_diagnostics(dst["zp"], dst["zq"], B, N, q=dst["q"], xstar=dst["xstar"], out=diag,
-                                        workspace=ws, stream=stream)
+            r = dcd.dcd_row_diagnostics(dst["zp"], dst["zq"], B, N, q=dst["q"], xstar=dst["xstar"],
+                                        cd_lse=dst["cd_lse"], alpha=w.alpha, beta=w.beta, out=diag, workspace=ws,
+                                        stream=stream)
             res_host.copy_(r, non_blocking=True)
 
         e2e_step()

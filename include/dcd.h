@@ -207,13 +207,16 @@ int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_p
  * DCD_STATIC_SCRATCH_BYTES compiled into the library, which every GPU that loads the
  * library holds until the process exits.  Shapes needing more scratch return
  * DCD_ERR_UNSUPPORTED.  Nothing is allocated: no cudaMalloc, cudaFree or allocating
- * library call.  The first call on a device looks up the array's device address (with
- * that device current) and caches it; make that first call before any stream capture.
- * All calls share the one array and it keeps the last call's contents (each call resets
- * the error word and rewrites every record it reads), so calls that overlap on the GPU,
- * from any stream or thread, race and must be serialised by the caller.
- * dcd_get_device_error cannot read this scratch; device-side input errors still show
- * as accept_len = 0 and bonus = -1 for the affected sequences.
+ * library call.  The first call on a device, and the first after the device gets a new
+ * context (e.g. after cudaDeviceReset), looks up the array's device address (with that
+ * device current) and caches it for that context; make that first call before any stream
+ * capture.  All calls share the one array and it keeps the last call's contents (each call
+ * resets the error word before its kernels run), so calls that overlap on the GPU, from any
+ * stream or thread, race and must be serialised by the caller.  dcd_get_device_error
+ * cannot read this scratch; device-side input errors still show as accept_len = 0 and
+ * bonus = -1 for the affected sequences, and a bounded device wait that gave up
+ * (DCD_DEVERR_TIMEOUT) shows as accept_len = 0 and bonus = -1 for every sequence of the
+ * call, so a record left by an earlier call is never reported as this call's result.
  * Arguments and results otherwise as dcd_verify_sample.
  */
 int dcd_verify_sample_noalloc(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
@@ -248,12 +251,18 @@ int dcd_upload_q_rows(const dcd_shape* shape, const float* q_host, float* q_dev,
  * the depth of each CTA's ring of shared-memory stages (0 = automatic, else 2 .. 8)
  * and `plain_loads` = 1 stages rows with ordinary loads instead of bulk asynchronous
  * copies.  Results equal dcd_score_rows up to fp32 summation order.
+ * `poll_limit_cycles` bounds, in SM clock cycles, the wait of a CTA whose rows are all
+ * claimed for residual passes that other CTAs may still publish (0 = the default bound of
+ * about two seconds; negative values are rejected).  No copy is in flight during that wait,
+ * so a short bound exercises the timeout path safely: the CTA stops, the call sets
+ * DCD_DEVERR_TIMEOUT in the error word, every sequence of a following dcd_tree_walk reports
+ * accept_len = 0 and bonus = -1, and the device stays usable.  Meant for tests.
  */
 int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
                       const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                       const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
                       int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes,
-                      dcd_stream_t stream, int stages, int plain_loads);
+                      dcd_stream_t stream, int stages, int plain_loads, int64_t poll_limit_cycles);
 
 /*
  * Greedy CD verification fused with the two models' output projections (LM heads): the
@@ -309,9 +318,10 @@ int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_
 
 /*
  * Per-row diagnostics of contrastive verification: the quantities behind the signal versus
- * proposal-error analysis (Sec. 3.1) and the alignment-gap estimator (App. C).  For every row r
- * of the B*N rows, with pi_p = softmax(z_exp[r]), pi_q = softmax(z_ama[r]) over the full
- * vocabulary (no temperature, no plausibility mask) and e = q[r] (the drafter's distribution):
+ * proposal-error analysis (Sec. 3.1), the alignment-gap estimator (App. C) and the KL
+ * decomposition of the CD target (App. B, Lemma kl_decomposition).  For every row r of the B*N
+ * rows, with pi_p = softmax(z_exp[r]), pi_q = softmax(z_ama[r]) over the full vocabulary (no
+ * temperature, no plausibility mask) and e = q[r] (the drafter's distribution):
  *   diag[r][0] = lse_p = log sum_x exp(z_exp[r][x])
  *   diag[r][1] = lse_q = log sum_x exp(z_ama[r][x])
  *   diag[r][2] = signal = |log pi_p(x*) - log pi_q(x*)| at x* = xstar[r] (the CD argmax, e.g.
@@ -320,11 +330,22 @@ int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_
  *   diag[r][3] = E_{pi_q}[log pi_p - log pi_q]   (= -D_KL(pi_q || pi_p))
  *   diag[r][4] = E_e[log pi_p - log pi_q]         (NaN if q is NULL)
  *   diag[r][5] = D_KL(e || pi_p), 0 log 0 = 0     (NaN if q is NULL)
+ *   diag[r][6] = D_KL(pi_p || pi_q)               (= E_{pi_p}[log pi_p - log pi_q])
+ *   diag[r][7] = D_KL(pi_p || pi_CD) = log Z_CD - alpha D_KL(pi_p || pi_q), the lemma of App. B
+ *                for the untruncated target at T = 1, pi_CD = pi_p^(1+alpha) pi_q^(-alpha) / Z_CD,
+ *                with log Z_CD = cd_lse[r] - (1 + alpha) lse_p + alpha lse_q taken from the
+ *                cd_lse output of a verification call on the same logits.  NaN if cd_lse is NULL,
+ *                or if the row's sequence has beta > 0 or a temperature other than 0 or 1 (the
+ *                lemma does not hold for a masked or tempered target).
  * The alignment gap of App. C is diag[4] - diag[3] averaged over the rows a caller selects.
  *   shape : B, N, V, logits_dtype, ld_logits as for the verification calls; ld_q (>= V) when q
  *       is given; flags must be 0.
  *   z_exp, z_ama : [B*N, ld_logits] device logits; q : [B*N, ld_q] fp32 device probabilities or
- *       NULL; xstar : int32 [B*N] device tokens or NULL; diag : fp32 [B*N, 6] device output.
+ *       NULL; xstar : int32 [B*N] device tokens or NULL; diag : fp32 [B*N, 8] device output.
+ *   cd_lse : fp32 [B*N] device values (the verification call's cd_lse output), or NULL;
+ *   alpha, beta, temperature : fp32 [B] device arrays of that verification call (alpha is
+ *       required with cd_lse and must be NULL without it; beta and temperature may be NULL for
+ *       0, i.e. unmasked and greedy).
  *   workspace : device scratch of at least dcd_diagnostics_workspace_bytes(shape) bytes,
  *       256-byte aligned (about 48 * B * N * ceil(V / 2048) bytes).
  * Logits must be finite (non-finite inputs give NaN or inf results; no error word is kept).
@@ -332,16 +353,20 @@ int dcd_verify_fused_lmhead_ex(const dcd_shape* shape, const void* h_exp, int32_
  * `stream`.  Returns DCD_ERR_INVALID_ARG or DCD_ERR_WORKSPACE for bad arguments, DCD_ERR_CUDA
  * if a launch fails.
  */
+#define DCD_DIAG_COLS 8
+
 size_t dcd_diagnostics_workspace_bytes(const dcd_shape* shape);
 
 int dcd_row_diagnostics(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
-                        const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                        const int32_t* xstar, const float* cd_lse, const float* alpha, const float* beta,
+                        const float* temperature, float* diag, void* workspace, size_t workspace_bytes,
                         dcd_stream_t stream);
 
 /* dcd_row_diagnostics that also records two CUDA events (cudaEvent_t, or NULL) on `stream`
  * immediately before and after the streaming pass (the per-row combine follows it). */
 int dcd_row_diagnostics_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
-                           const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                           const int32_t* xstar, const float* cd_lse, const float* alpha, const float* beta,
+                           const float* temperature, float* diag, void* workspace, size_t workspace_bytes,
                            dcd_stream_t stream, void* pass_start, void* pass_stop);
 
 /*

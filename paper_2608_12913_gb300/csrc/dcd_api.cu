@@ -15,7 +15,7 @@
 
 namespace {
 
-constexpr int kVersion = 10000;  // 1.0.0
+constexpr int kVersion = 10100;  // 1.1.0
 
 bool shape_ok(const dcd_shape* s, bool need_q) {
   if (!s) return false;
@@ -111,7 +111,7 @@ int score_rows_impl(const dcd_shape* shape, const void* z_exp, const void* z_ama
                     const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                     const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob, int32_t* cd_argmax,
                     float* cd_lse, void* workspace, size_t workspace_bytes, cudaStream_t stream, int force_stages,
-                    int force_plain) {
+                    int force_plain, int64_t poll_cycles) {
   const bool sampled_call = temperature != nullptr;
   if (!shape_ok(shape, sampled_call)) return DCD_ERR_INVALID_ARG;
   if (shape->N > DCD_MAX_NODES) return DCD_ERR_UNSUPPORTED;
@@ -125,6 +125,7 @@ int score_rows_impl(const dcd_shape* shape, const void* z_exp, const void* z_ama
                                cd_logprob, cd_argmax, cd_lse, workspace);
   a.force_stages = force_stages;
   a.force_plain = force_plain;
+  a.poll_cycles = poll_cycles;
   const dcd::RowGeometry geo = dcd::row_geometry(a);
   if (geo.smem > 227 * 1024 || geo.ctas_per_sm < 1) return DCD_ERR_UNSUPPORTED;
   return cuda_status(dcd::launch_score_rows(a, stream));
@@ -144,7 +145,7 @@ int dcd_score_rows(const dcd_shape* shape, const void* z_exp, const void* z_ama,
                    const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob, int32_t* cd_argmax,
                    float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream) {
   return score_rows_impl(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset, cd_logprob,
-                         cd_argmax, cd_lse, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), 0, 0);
+                         cd_argmax, cd_lse, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), 0, 0, 0);
 }
 
 int dcd_tree_walk(const dcd_shape* shape, int32_t* accept_len, int32_t* accept_path, int32_t* bonus,
@@ -293,11 +294,13 @@ size_t dcd_diagnostics_workspace_bytes(const dcd_shape* shape) {
 }
 
 int dcd_row_diagnostics_ex(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
-                           const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                           const int32_t* xstar, const float* cd_lse, const float* alpha, const float* beta,
+                           const float* temperature, float* diag, void* workspace, size_t workspace_bytes,
                            dcd_stream_t stream, void* pass_start, void* pass_stop) {
   if (!shape_ok(shape, q != nullptr) || shape->flags != 0) return DCD_ERR_INVALID_ARG;
   const int64_t R = static_cast<int64_t>(shape->B) * shape->N;
   if (R > 0 && (!z_exp || !z_ama || !diag)) return DCD_ERR_INVALID_ARG;
+  if ((cd_lse != nullptr) != (alpha != nullptr)) return DCD_ERR_INVALID_ARG;  // the lemma needs both
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 ||
       workspace_bytes < dcd_diagnostics_workspace_bytes(shape))
     return DCD_ERR_WORKSPACE;
@@ -306,11 +309,16 @@ int dcd_row_diagnostics_ex(const dcd_shape* shape, const void* z_exp, const void
   d.V = shape->V;
   d.ld = shape->ld_logits;
   d.ldq = shape->ld_q;
+  d.N = shape->N;
   d.dtype = shape->logits_dtype;
   d.z_exp = z_exp;
   d.z_ama = z_ama;
   d.q = q;
   d.xstar = xstar;
+  d.cd_lse = cd_lse;
+  d.alpha = alpha;
+  d.beta = beta;
+  d.temp = temperature;
   d.out = diag;
   d.part = static_cast<dcd::DiagPart*>(workspace);
   d.stream = stream;
@@ -320,10 +328,11 @@ int dcd_row_diagnostics_ex(const dcd_shape* shape, const void* z_exp, const void
 }
 
 int dcd_row_diagnostics(const dcd_shape* shape, const void* z_exp, const void* z_ama, const float* q,
-                        const int32_t* xstar, float* diag, void* workspace, size_t workspace_bytes,
+                        const int32_t* xstar, const float* cd_lse, const float* alpha, const float* beta,
+                        const float* temperature, float* diag, void* workspace, size_t workspace_bytes,
                         dcd_stream_t stream) {
-  return dcd_row_diagnostics_ex(shape, z_exp, z_ama, q, xstar, diag, workspace, workspace_bytes, stream, nullptr,
-                                nullptr);
+  return dcd_row_diagnostics_ex(shape, z_exp, z_ama, q, xstar, cd_lse, alpha, beta, temperature, diag, workspace,
+                                workspace_bytes, stream, nullptr, nullptr);
 }
 
 int dcd_get_device_error(const void* workspace, dcd_stream_t stream, uint32_t* bits) {
@@ -358,11 +367,12 @@ int dcd_score_rows_ex(const dcd_shape* shape, const void* z_exp, const void* z_a
                       const int32_t* tokens, const int32_t* parents, const float* alpha, const float* beta,
                       const float* temperature, uint64_t seed, uint64_t offset, float* cd_logprob,
                       int32_t* cd_argmax, float* cd_lse, void* workspace, size_t workspace_bytes, dcd_stream_t stream,
-                      int stages, int plain_loads) {
+                      int stages, int plain_loads, int64_t poll_limit_cycles) {
   if (stages != 0 && (stages < 2 || stages > 8)) return DCD_ERR_INVALID_ARG;
+  if (poll_limit_cycles < 0) return DCD_ERR_INVALID_ARG;
   return score_rows_impl(shape, z_exp, z_ama, q, tokens, parents, alpha, beta, temperature, seed, offset, cd_logprob,
                          cd_argmax, cd_lse, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream),
-                         stages, plain_loads);
+                         stages, plain_loads, poll_limit_cycles);
 }
 
 }  // extern "C"

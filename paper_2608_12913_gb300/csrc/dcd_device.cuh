@@ -222,10 +222,22 @@ __device__ __forceinline__ float ld1(const __nv_bfloat16* p, int64_t i) { return
 struct SyncCta {
   __device__ __forceinline__ void operator()() const { __syncthreads(); }
 };
-struct SyncConsumers {
+template <int NT>
+struct SyncConsumersN {
   __device__ __forceinline__ void operator()() const {
-    asm volatile("bar.sync 1, %0;" ::"n"(kThreads) : "memory");
+    asm volatile("bar.sync 1, %0;" ::"n"(NT) : "memory");
   }
+};
+using SyncConsumers = SyncConsumersN<kThreads>;
+
+// Warps taking part in a block reduction: the whole CTA's kWarps, or a SyncConsumersN group's.
+template <typename Sync>
+struct SyncWarps {
+  static constexpr int value = kWarps;
+};
+template <int NT>
+struct SyncWarps<SyncConsumersN<NT>> {
+  static constexpr int value = NT / 32;
 };
 
 __device__ __forceinline__ void argmax_merge(float& v, int& i, float v2, int i2) {
@@ -264,7 +276,7 @@ __device__ __forceinline__ void block_argmax(float& v, int& i, float* redf, int*
   v = redf[0];
   i = redi[0];
 #pragma unroll
-  for (int w = 1; w < kWarps; ++w) argmax_merge(v, i, redf[w], redi[w]);
+  for (int w = 1; w < SyncWarps<Sync>::value; ++w) argmax_merge(v, i, redf[w], redi[w]);
   sync();
 }
 
@@ -275,7 +287,7 @@ __device__ __forceinline__ float block_sum(float v, float* redf, Sync sync = Syn
   sync();
   float s = 0.f;
 #pragma unroll
-  for (int w = 0; w < kWarps; ++w) s += redf[w];
+  for (int w = 0; w < SyncWarps<Sync>::value; ++w) s += redf[w];
   sync();
   return s;
 }
@@ -295,17 +307,19 @@ __device__ __forceinline__ void block_stats(float& m, float& s, int& arg, float*
 #pragma unroll
   for (int o = 16; o; o >>= 1)
     merge(m, s, arg, __shfl_xor_sync(~0u, m, o), __shfl_xor_sync(~0u, s, o), __shfl_xor_sync(~0u, arg, o));
+  constexpr int NW = SyncWarps<Sync>::value;  // redf holds 2 * NW <= 32 values
+  static_assert(2 * NW <= 32, "reduction scratch");
   if ((threadIdx.x & 31) == 0) {
     redf[threadIdx.x >> 5] = m;
-    redf[kWarps + (threadIdx.x >> 5)] = s;
+    redf[NW + (threadIdx.x >> 5)] = s;
     redi[threadIdx.x >> 5] = arg;
   }
   sync();
   m = redf[0];
-  s = redf[kWarps];
+  s = redf[NW];
   arg = redi[0];
 #pragma unroll
-  for (int w = 1; w < kWarps; ++w) merge(m, s, arg, redf[w], redf[kWarps + w], redi[w]);
+  for (int w = 1; w < NW; ++w) merge(m, s, arg, redf[w], redf[NW + w], redi[w]);
   sync();
 }
 
@@ -316,7 +330,7 @@ __device__ __forceinline__ float block_max(float v, float* redf, Sync sync = Syn
   sync();
   float s = -INFINITY;
 #pragma unroll
-  for (int w = 0; w < kWarps; ++w) s = fmaxf(s, redf[w]);
+  for (int w = 0; w < SyncWarps<Sync>::value; ++w) s = fmaxf(s, redf[w]);
   sync();
   return s;
 }

@@ -4,14 +4,18 @@
 //
 // For a row with logits z_p, z_q and reference values r_p = z_p(0), r_q = z_q(0) the pass keeps,
 // per thread and then per chunk of the vocabulary:
-//   m_p, s_p = sum exp(z_p - m_p)                    (online max / rescaled sum)
+//   m_p, s_p = sum exp(z_p - m_p), t_p = sum exp(z_p - m_p) d   (online max / rescaled sums)
 //   m_q, s_q = sum exp(z_q - m_q), t_q = sum exp(z_q - m_q) d,   d = (z_p - r_p) - (z_q - r_q)
 //   with q:  a = sum q d,  e1 = sum q,  ez = sum q (z_p - r_p),  h = sum_{q > 0} q log2 q
 // and a per-row combine turns them into
 //   lse_p, lse_q; signal = |(z_p(x*) - lse_p) - (z_q(x*) - lse_q)|;
 //   e_q = E_{pi_q}[log pi_p - log pi_q] = t_q / s_q - (L_p - L_q),
+//   kl_pq = D_KL(pi_p || pi_q)          = t_p / s_p - (L_p - L_q),
 //   e_e = E_q[log pi_p - log pi_q]      = a - (L_p - L_q) e1,
 //   kl  = D_KL(q || pi_p)               = h ln 2 - ez + L_p e1,        L_p = lse_p - r_p, L_q = lse_q - r_q.
+// and, given the CD normaliser cd_lse = log sum exp((1 + alpha) z_p - alpha z_q) of a verification
+// call with beta = 0 and T = 1, the decomposition lemma of App. B gives
+//   kl_pcd = D_KL(pi_p || pi_CD) = log Z_CD - alpha kl_pq,  log Z_CD = cd_lse - (1 + alpha) lse_p + alpha lse_q.
 // Shifting by r_p, r_q keeps every linear term at the scale of the logit spread rather than of
 // the logits' absolute offset, so fp32 accumulation loses little to cancellation.
 #include <cuda_bf16.h>
@@ -35,12 +39,8 @@ constexpr int kDiagCtasPerSm = 4;          // resident CTAs per SM (64 registers
 constexpr float kLn2 = 0.6931471805599453f;
 
 struct Acc {
-  float mp, sp, mq, sq, tq, a, e1, ez, h;
+  float mp, sp, mq, sq, tq, a, e1, ez, h, tp;
 };
-
-__device__ __forceinline__ float rescale(float s, float m, float m_new) {
-  return m == m_new ? s : s * dev::ex2((m - m_new) * dev::kLog2e);
-}
 
 // Adds tokens with values p[k], z[k] (and q values e[k]) to the accumulator.
 template <int K, bool kQ>
@@ -53,7 +53,9 @@ __device__ __forceinline__ void accumulate(Acc& c, const float* p, const float* 
     lq = fmaxf(lq, z[k]);
   }
   if (lp > c.mp) {
-    c.sp = rescale(c.sp, c.mp, lp);
+    const float f = dev::ex2((c.mp - lp) * dev::kLog2e);
+    c.sp *= f;
+    c.tp *= f;
     c.mp = lp;
   }
   if (lq > c.mq) {
@@ -67,7 +69,9 @@ __device__ __forceinline__ void accumulate(Acc& c, const float* p, const float* 
   for (int k = 0; k < K; ++k) {
     const float pr = p[k] - rp;
     const float d = pr - (z[k] - rq);
-    c.sp += dev::ex2(fmaf(p[k], dev::kLog2e, -mpl));
+    const float wp = dev::ex2(fmaf(p[k], dev::kLog2e, -mpl));
+    c.sp += wp;
+    c.tp = fmaf(wp, d, c.tp);
     const float w = dev::ex2(fmaf(z[k], dev::kLog2e, -mql));
     c.sq += w;
     c.tq = fmaf(w, d, c.tq);
@@ -83,7 +87,10 @@ __device__ __forceinline__ void accumulate(Acc& c, const float* p, const float* 
 
 __device__ __forceinline__ void merge(Acc& c, const Acc& o) {
   const float mp = fmaxf(c.mp, o.mp), mq = fmaxf(c.mq, o.mq);
-  c.sp = rescale(c.sp, c.mp, mp) + rescale(o.sp, o.mp, mp);
+  const float fp = c.mp == mp ? 1.f : dev::ex2((c.mp - mp) * dev::kLog2e);
+  const float gp = o.mp == mp ? 1.f : dev::ex2((o.mp - mp) * dev::kLog2e);
+  c.sp = c.sp * fp + o.sp * gp;
+  c.tp = c.tp * fp + o.tp * gp;
   c.mp = mp;
   const float fq = c.mq == mq ? 1.f : dev::ex2((c.mq - mq) * dev::kLog2e);
   const float gq = o.mq == mq ? 1.f : dev::ex2((o.mq - mq) * dev::kLog2e);
@@ -107,6 +114,7 @@ __device__ __forceinline__ Acc shfl_down(const Acc& c, int off) {
   o.e1 = __shfl_down_sync(0xffffffffu, c.e1, off);
   o.ez = __shfl_down_sync(0xffffffffu, c.ez, off);
   o.h = __shfl_down_sync(0xffffffffu, c.h, off);
+  o.tp = __shfl_down_sync(0xffffffffu, c.tp, off);
   return o;
 }
 
@@ -143,7 +151,7 @@ __global__ void __launch_bounds__(kDiagThreads, kDiagCtasPerSm) diag_partial_ker
     const TIn* z = zq + row * ld;
     const float* e = kQ ? q + row * ldq : nullptr;
     const float rp = dev::ld1(p, 0), rq = dev::ld1(z, 0);
-    Acc c = {-INFINITY, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    Acc c = {-INFINITY, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     int64_t i = lo;
     if (kVec) {
       const int64_t hv = lo + ((hi - lo) & ~static_cast<int64_t>(7));
@@ -180,7 +188,8 @@ __global__ void __launch_bounds__(kDiagThreads, kDiagCtasPerSm) diag_partial_ker
       for (int w = 1; w < kDiagWarps; ++w) merge(t, red[w]);
       DiagPart o;
       o.mp = t.mp; o.sp = t.sp; o.mq = t.mq; o.sq = t.sq; o.tq = t.tq;
-      o.a = t.a; o.e1 = t.e1; o.ez = t.ez; o.h = t.h;
+      o.a = t.a; o.e1 = t.e1; o.ez = t.ez; o.h = t.h; o.tp = t.tp;
+      o.pad[0] = o.pad[1] = 0.f;
       part[row * gridDim.x + blockIdx.x] = o;
     }
     __syncthreads();
@@ -188,49 +197,77 @@ __global__ void __launch_bounds__(kDiagThreads, kDiagCtasPerSm) diag_partial_ker
 }
 
 // One warp per row: lanes merge the row's chunk partials (the same rescaled fp32 merge as the
-// streaming pass), then lane 0 forms the six diagnostics in fp32 (fp64 is avoided: its rate on
-// this GPU is a small fraction of fp32's, and two fp64 logarithms a row cost more than the merge).
+// streaming pass), then lane 0 forms the diagnostics in fp32 (fp64 is avoided: its rate on this GPU
+// is a small fraction of fp32's, and two fp64 logarithms a row cost more than the merge).
 constexpr int kCombineWarps = 8;
 
+struct CombineArgs {
+  const int32_t* xstar;
+  const float* cd_lse;
+  const float* alpha;
+  const float* beta;
+  const float* temp;
+  bool has_q;
+  int64_t R, V, ld;
+  int N, nchunk;
+  const DiagPart* part;
+  float* out;
+};
+
 template <typename TIn>
-__global__ void __launch_bounds__(32 * kCombineWarps) diag_combine_kernel(
-    const TIn* __restrict__ zp, const TIn* __restrict__ zq, const int32_t* __restrict__ xstar, bool has_q, int64_t R,
-    int64_t V, int64_t ld, int nchunk, const DiagPart* __restrict__ part, float* __restrict__ out) {
+__global__ void __launch_bounds__(32 * kCombineWarps) diag_combine_kernel(const TIn* __restrict__ zp,
+                                                                          const TIn* __restrict__ zq,
+                                                                          const CombineArgs a) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int lane = threadIdx.x & 31;
   const int64_t row = static_cast<int64_t>(blockIdx.x) * kCombineWarps + (threadIdx.x >> 5);
-  if (row >= R) return;
-  const DiagPart* pp = part + row * nchunk;
-  const TIn* p = zp + row * ld;
-  const TIn* z = zq + row * ld;
-  // lanes 0-3 fetch the logits the outputs need (r_p, r_q, z_p(x*), z_q(x*)) while the partials load
-  const int32_t x = xstar ? xstar[row] : -1;
-  const bool x_ok = x >= 0 && x < V;
+  if (row >= a.R) return;
+  const DiagPart* pp = a.part + row * a.nchunk;
+  const TIn* p = zp + row * a.ld;
+  const TIn* z = zq + row * a.ld;
+  // lanes 0-3 fetch the logits the outputs need (r_p, r_q, z_p(x*), z_q(x*)) while the partials
+  // load; lanes 4-7 the lemma's inputs (cd_lse, alpha, beta, T)
+  const int32_t x = a.xstar ? a.xstar[row] : -1;
+  const bool x_ok = x >= 0 && x < a.V;
+  const int64_t b = row / a.N;
+  const bool want_cd = a.cd_lse && a.alpha;
   float lv = 0.f;
   if (lane < 2) lv = dev::ld1(lane == 0 ? p : z, 0);
   else if (lane < 4 && x_ok) lv = dev::ld1(lane == 2 ? p : z, x);
-  Acc c = {-INFINITY, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  for (int k = lane; k < nchunk; k += 32) {
+  else if (lane == 4 && want_cd) lv = a.cd_lse[row];
+  else if (lane == 5 && want_cd) lv = a.alpha[b];
+  else if (lane == 6 && want_cd && a.beta) lv = a.beta[b];
+  else if (lane == 7 && want_cd && a.temp) lv = a.temp[b];
+  Acc c = {-INFINITY, 0.f, -INFINITY, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int k = lane; k < a.nchunk; k += 32) {
     const DiagPart& d = pp[k];
-    const Acc o = {d.mp, d.sp, d.mq, d.sq, d.tq, d.a, d.e1, d.ez, d.h};
+    const Acc o = {d.mp, d.sp, d.mq, d.sq, d.tq, d.a, d.e1, d.ez, d.h, d.tp};
     merge(c, o);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) merge(c, shfl_down(c, off));
   const float rp = __shfl_sync(0xffffffffu, lv, 0), rq = __shfl_sync(0xffffffffu, lv, 1);
   const float px = __shfl_sync(0xffffffffu, lv, 2), qx = __shfl_sync(0xffffffffu, lv, 3);
+  const float cdl = __shfl_sync(0xffffffffu, lv, 4), al = __shfl_sync(0xffffffffu, lv, 5);
+  const float be = __shfl_sync(0xffffffffu, lv, 6), tt = __shfl_sync(0xffffffffu, lv, 7);
   if (lane != 0) return;
   const float ls_p = logf(c.sp), ls_q = logf(c.sq);  // lse = m + ls
   // L_p = lse_p - r_p, with m - r the difference of two stored logits (exact for bf16 inputs)
   const float Lp = (c.mp - rp) + ls_p, Lq = (c.mq - rq) + ls_q;
   const float signal = x_ok ? fabsf(((px - c.mp) - ls_p) - ((qx - c.mq) - ls_q)) : NAN;
-  float* o = out + row * 6;
-  o[0] = c.mp + ls_p;
-  o[1] = c.mq + ls_q;
+  const float lse_p = c.mp + ls_p, lse_q = c.mq + ls_q;
+  const float kl_pq = c.tp / c.sp - (Lp - Lq);
+  // the lemma holds for the untruncated target at T = 1 (greedy sequences report cd_lse at T = 1)
+  const bool lemma = want_cd && be == 0.f && (tt == 0.f || tt == 1.f) && al >= 0.f;
+  float* o = a.out + row * kDiagCols;
+  o[0] = lse_p;
+  o[1] = lse_q;
   o[2] = signal;
   o[3] = c.tq / c.sq - (Lp - Lq);
-  o[4] = has_q ? fmaf(-(Lp - Lq), c.e1, c.a) : NAN;
-  o[5] = has_q ? fmaf(Lp, c.e1, fmaf(c.h, kLn2, -c.ez)) : NAN;
+  o[4] = a.has_q ? fmaf(-(Lp - Lq), c.e1, c.a) : NAN;
+  o[5] = a.has_q ? fmaf(Lp, c.e1, fmaf(c.h, kLn2, -c.ez)) : NAN;
+  o[6] = kl_pq;
+  o[7] = lemma ? (cdl - (1.f + al) * lse_p + al * lse_q) - al * kl_pq : NAN;
 }
 
 template <typename TIn, bool kVec, bool kQ>
@@ -266,9 +303,22 @@ cudaError_t launch_typed(const DiagArgs& d) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (d.stop && (e = cudaEventRecord(static_cast<cudaEvent_t>(d.stop), d.stream)) != cudaSuccess) return e;
+  CombineArgs ca;
+  ca.xstar = d.xstar;
+  ca.cd_lse = d.cd_lse;
+  ca.alpha = d.alpha;
+  ca.beta = d.beta;
+  ca.temp = d.temp;
+  ca.has_q = d.q != nullptr;
+  ca.R = d.R;
+  ca.V = d.V;
+  ca.ld = d.ld;
+  ca.N = d.N;
+  ca.nchunk = nchunk;
+  ca.part = d.part;
+  ca.out = d.out;
   return cudaLaunchKernelEx(&cfg, diag_combine_kernel<TIn>, static_cast<const TIn*>(d.z_exp),
-                            static_cast<const TIn*>(d.z_ama), d.xstar, d.q != nullptr, d.R, d.V, d.ld, nchunk,
-                            static_cast<const DiagPart*>(d.part), d.out);
+                            static_cast<const TIn*>(d.z_ama), ca);
 }
 
 }  // namespace

@@ -9,8 +9,9 @@ namespace dcd {
 
 // Statistics of one chunk of one row's vocabulary (see dcd_diag.cu for their definitions).
 struct alignas(16) DiagPart {
-  float mp, sp, mq, sq, tq, a, e1, ez, h, pad[3];
+  float mp, sp, mq, sq, tq, a, e1, ez, h, tp, pad[2];
 };
+constexpr int kDiagCols = 8;  // diagnostics per row
 constexpr int kDiagMinChunk = 2048;   // tokens per CTA of the streaming pass: at least ...
 constexpr int kDiagMaxChunk = 16384;  // ... and at most
 // Tokens per chunk for R rows of V tokens on a GPU with `sms` SMs (a multiple of kDiagMinChunk).
@@ -23,12 +24,17 @@ inline size_t diag_workspace_bytes(int64_t R, int64_t V) {
 
 struct DiagArgs {
   int64_t R, V, ld, ldq;
+  int N;                 // nodes per sequence (row r belongs to sequence r / N)
   int dtype;
   const void* z_exp;
   const void* z_ama;
   const float* q;        // may be null
   const int32_t* xstar;  // may be null
-  float* out;            // [R, 6]
+  const float* cd_lse;   // [R] from a verification call, or null
+  const float* alpha;    // [B], or null
+  const float* beta;     // [B], or null (beta = 0)
+  const float* temp;     // [B], or null (greedy)
+  float* out;            // [R, kDiagCols]
   DiagPart* part;        // workspace
   cudaStream_t stream;
   void* start;  // optional cudaEvent_t pair around the streaming pass (timing)

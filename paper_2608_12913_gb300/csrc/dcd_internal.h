@@ -119,6 +119,8 @@ struct ScoreArgs {
   int32_t distinct;       // 1: siblings drawn without replacement (DCD_SIBLINGS_DISTINCT)
   int32_t force_stages;   // 0 = automatic, else the ring depth to use (tests / tuning)
   int32_t force_plain;    // 1 = plain loads instead of bulk async copies
+  int64_t poll_cycles;    // limit of a producer's poll for residual passes once its rows are
+                          // done (0 = the default bounded wait; tests shorten it)
 };
 
 // Residual pieces per pass and slot bytes per row for a vocabulary of V tokens in a call of

@@ -90,8 +90,22 @@ constexpr int kSmallPieceStages = DCD_SMALL_PIECE_STAGES;
 // dynamic claiming of whole rows balances better than parts (measured).
 constexpr int kPartsBelow = DCD_PARTS_BELOW;
 constexpr int kDesc = 4;                           // work descriptors in flight per CTA
-constexpr int kCtaThreads = kThreads + 32;         // eight consumer warps and one producer warp
-constexpr int kMinCtasPerSm = 3;
+#ifndef DCD_ROW_WARPS
+#define DCD_ROW_WARPS 8
+#endif
+#ifndef DCD_MIN_CTAS
+#define DCD_MIN_CTAS 3
+#endif
+#ifndef DCD_RING_STAGES
+#define DCD_RING_STAGES 2
+#endif
+constexpr int kRowWarps = DCD_ROW_WARPS;           // consumer warps per CTA
+constexpr int kRowThreads = kRowWarps * 32;
+constexpr int kCtaThreads = kRowThreads + 32;      // the consumer warps and one producer warp
+constexpr int kMinCtasPerSm = DCD_MIN_CTAS;
+constexpr int kRingStages = DCD_RING_STAGES;       // default ring depth
+static_assert(kRowWarps == 8 || kRowWarps == 12 || kRowWarps == 16, "consumer warps");
+using RowSync = SyncConsumersN<kRowThreads>;
 constexpr size_t kSmemMax = 227 * 1024;
 constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr float kLn2 = 0.69314718055994531f;
@@ -118,6 +132,7 @@ struct SParams {
   int32_t spp;           // stats-pass stages per part
   int32_t items;         // row items: r_whole + (R - r_whole) * parts
   int32_t keep_internal; // small batch: keep sampled internal rows and pieces in L2 (evict-last)
+  long long poll_cycles; // bound of the end-of-work poll for residual passes
   WsHeader* hdr;         // counters, zeroed before the launch
   Job* jobs;             // residual passes (zeroed before the launch)
   unsigned char* slots;  // per handed-over row: SlotHead + npieces PieceParts
@@ -308,7 +323,7 @@ template <typename MassFn>
 __device__ int token_race(const ScoreArgs& p, int64_t g, int kstar, MassFn mass, float* redf, int* redi) {
   float tk = -INFINITY;
   int tx = INT_MAX;
-  if (kstar != INT_MAX) {
+  if (kstar != INT_MAX && threadIdx.x < kRaceBlock / 4) {
     const int64_t x = static_cast<int64_t>(kstar) * kRaceBlock + threadIdx.x * 4;
     if (x < p.V) {
       const uint4 w =
@@ -329,7 +344,7 @@ __device__ int token_race(const ScoreArgs& p, int64_t g, int kstar, MassFn mass,
       }
     }
   }
-  block_argmax(tk, tx, redf, redi, SyncConsumers());
+  block_argmax(tk, tx, redf, redi, RowSync());
   return tx;
 }
 
@@ -356,7 +371,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
   const int64_t V = p.V;
   const int R = p.B * N;
   const int nch_a = static_cast<int>((V + sp.tok_a - 1) / sp.tok_a);  // stages of a max / stats pass
-  const SyncConsumers csync;
+  const RowSync csync;
 
   extern __shared__ __align__(128) unsigned char smem[];
   uint64_t* full = reinterpret_cast<uint64_t*>(smem);  // [kMaxStages] stage filled
@@ -379,7 +394,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
   if (tid == 0) {
     for (int s = 0; s < sp.nst; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kWarps);
+      mbar_init(&empty[s], kRowWarps);
     }
     for (int d = 0; d < kDesc; ++d) {
       mbar_init(&dfull[d], 1);
@@ -389,7 +404,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
   }
   __syncthreads();  // the last CTA-wide barrier: from here on the two roles synchronise by mbarriers
 
-  if (warp == kWarps) {
+  if (warp == kRowWarps) {
     // ===================================== producer warp
     const uint64_t pol_last = l2_policy_evict_last();
     const uint64_t pol_normal = l2_policy_evict_normal();
@@ -502,7 +517,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
             if (lane == 0) {
               if (poll && ld_volatile(&sp.hdr->rows_done) >= static_cast<uint32_t>(R)) {
                 stop = 1;
-              } else if (clock64() - t0 > kWaitCycles) {
+              } else if (clock64() - t0 > sp.poll_cycles) {
                 atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
                 stop = 1;
               }
@@ -684,7 +699,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       const float* q_row = p.q + g * p.ldq;
       // a warp takes tok_r / 8 consecutive tokens of each stage (a chunk); `wpb` chunks make a
       // race block
-      const int tpw = sp.tok_r / kWarps, wpb = kRaceBlock / tpw;
+      const int tpw = sp.tok_r / kRowWarps, wpb = kRaceBlock / tpw;
       const int64_t piece_lo = static_cast<int64_t>(piece) * sp.piece_stages * sp.tok_r;
       const int64_t rem = (V - piece_lo + sp.tok_r - 1) / sp.tok_r;
       const int nst_piece = static_cast<int>(rem < sp.piece_stages ? rem : sp.piece_stages);
@@ -707,7 +722,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         zl += part;
         if (race) {
           const float ws = warp_sum(part);
-          if (lane == 0) csum[L * kWarps + warp] = ws;
+          if (lane == 0) csum[L * kRowWarps + warp] = ws;
         }
         warp_release(&empty[seq % static_cast<uint32_t>(sp.nst)]);
       }
@@ -985,7 +1000,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
               // pass found no mass, or q was used up)
               float bk2 = -INFINITY;
               int bb2 = INT_MAX;
-              for (int kb = warp; kb < sp.nblk; kb += kWarps) {
+              for (int kb = warp; kb < sp.nblk; kb += kRowWarps) {
                 float part = 0.f;
                 for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < V && x < (kb + 1) * kRaceBlock;
                      x += 32)
@@ -1005,7 +1020,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
               // block masses of q, computed by this CTA alone (rare: a residual without mass)
               float bk2 = -INFINITY;
               int bb2 = INT_MAX;
-              for (int kb = warp; kb < sp.nblk; kb += kWarps) {
+              for (int kb = warp; kb < sp.nblk; kb += kRowWarps) {
                 float part = 0.f;
                 for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < V && x < (kb + 1) * kRaceBlock;
                      x += 32)
@@ -1093,7 +1108,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         const int64_t x0 = static_cast<int64_t>(L) * sp.tok_a;
         const int clen = static_cast<int>((V - x0) < sp.tok_a ? (V - x0) : sp.tok_a);
         wait_full(seq);
-        for (int i0 = tid * 8; i0 < clen; i0 += kThreads * 8) {
+        for (int i0 = tid * 8; i0 < clen; i0 += kRowThreads * 8) {
           float zp[8];
           ld8(st.zp + i0, zp);
 #pragma unroll
@@ -1108,7 +1123,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
     // ---- pass B: per lane an online max of u on P_beta, the sum of 2^(u - max) rescaled when
     // the max grows, and the argmax.  A warp takes tok_a / 8 consecutive tokens (a chunk) of each
     // stage; for a sampled leaf it also records the chunk's mass relative to a chunk reference.
-    const int tpw = sp.tok_a / kWarps, wpb = kRaceBlock / tpw;
+    const int tpw = sp.tok_a / kRowWarps, wpb = kRaceBlock / tpw;
     float lmax = -INFINITY, lsum = 0.f;
     int larg = INT_MAX;
     for (int L = L0; L < L0 + nL; ++L, ++seq) {
@@ -1171,7 +1186,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       if (k_hi > sp.nblk) k_hi = sp.nblk;
       bk = -INFINITY;
       bb = INT_MAX;
-      for (int k = k_lo + tid; k < k_hi; k += kThreads) {
+      for (int k = k_lo + tid; k < k_hi; k += kRowThreads) {
         float ref = -INFINITY, sum = 0.f;
         for (int i = 0; i < wpb && k * wpb + i < nch_row; ++i) ref = fmaxf(ref, cref[k * wpb + i]);
         if (ref > -INFINITY)
@@ -1245,7 +1260,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       kstar = rs->term;
       m = rs->m;
       status = rs->status | (rs->degen ? DCD_DEVERR_TIMEOUT : 0u);
-      for (int k = tid; k < m; k += kThreads) {
+      for (int k = tid; k < m; k += kRowThreads) {
         const int t = ktok[k];
         const bool ok = t >= 0 && t < V;
         czp[k] = ok ? ld1(zp_row, t) : 0.f;
@@ -1260,7 +1275,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         czq[lane] = pzq;
         cq[lane] = pq;
       }
-      for (int k = 32 + tid; k < m; k += kThreads) {  // nodes with more children than a warp has lanes
+      for (int k = 32 + tid; k < m; k += kRowThreads) {  // nodes with more children than a warp has lanes
         const int t = ktok[k];
         const bool ok = t >= 0 && t < V;
         czp[k] = ok ? ld1(zp_row, t) : 0.f;
@@ -1285,7 +1300,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       if (n == 0 && p.cd_logprob) p.cd_logprob[g] = 0.f;
     }
     if (p.cd_logprob) {
-      for (int k = tid; k < m; k += kThreads) {
+      for (int k = tid; k < m; k += kRowThreads) {
         const bool in = !masked || (czp[k] - Mp >= logb);
         p.cd_logprob[static_cast<int64_t>(b) * N + kids[k]] =
             in ? (fmaf(c1k, czp[k], -ak * czq[k]) - M) * kLn2 - logS : -INFINITY;
@@ -1402,6 +1417,10 @@ __global__ void __launch_bounds__(kWalkWarps * 32) tree_walk_kernel(int32_t B, i
     st |= v.status;
   }
   st = __reduce_or_sync(~0u, st);
+  // A bounded wait that gave up anywhere in the call may have left rows without a fresh record
+  // (a record of an earlier call in the same workspace would look valid), so a timeout recorded
+  // in the call's error word fails every sequence.
+  st |= ld_volatile(err) & DCD_DEVERR_TIMEOUT;
   __syncwarp();
   int32_t* path = accept_path + static_cast<int64_t>(b) * N;
   if (st) {
@@ -1570,23 +1589,30 @@ Layout layout_for(int N, int nchunk, int nst) {
   return l;
 }
 
-// Tokens per stage, in whole race blocks: z_p and z_q fill a stage in row passes; z_p, z_q and
-// q share it in residual pieces.
-int tokens_a(int es) { return kStageBytes / (2 * es) / kRaceBlock * kRaceBlock; }
-int tokens_r(int es) { return kStageBytes / (2 * es + 4) / kRaceBlock * kRaceBlock; }
+// Tokens per stage: every consumer warp takes tpw consecutive tokens of a stage, with tpw a
+// multiple of the 256-token group that divides a race block (256, 512 or 1024 tokens), so whole
+// warp chunks make a race block.  z_p and z_q fill a stage in row passes; z_p, z_q and q share it
+// in residual pieces.
+int split_tokens(int cap) {
+  for (int tpw = kRaceBlock; tpw >= kSub; tpw /= 2)
+    if (kRowWarps * tpw <= cap) return kRowWarps * tpw;
+  return 0;
+}
+int tokens_a(int es) { return split_tokens(kStageBytes / (2 * es)); }
+int tokens_r(int es) { return split_tokens(kStageBytes / (2 * es + 4)); }
 
-// A warp takes tok / 8 tokens of a stage in groups of 256, whole chunks make a race block, and
-// a piece's chunks fit the chunk arrays.
+// A warp takes tok / kRowWarps tokens of a stage in groups of 256, whole chunks make a race
+// block, and a piece's race blocks fit the consumer threads.
 bool stage_split_ok(int tok) {
-  const int tpw = tok / kWarps;
-  return tok > 0 && tok % (kWarps * kSub) == 0 && tpw <= kRaceBlock && kRaceBlock % tpw == 0 &&
-         kPieceStages * (tok / kRaceBlock) <= kThreads;
+  const int tpw = tok / kRowWarps;
+  return tok > 0 && tok % (kRowWarps * kSub) == 0 && tpw <= kRaceBlock && kRaceBlock % tpw == 0 &&
+         kPieceStages * (tok / kRaceBlock) <= kRowThreads;
 }
 
 int chunks_per_row(int64_t V, int es) {
-  const int tpw = tokens_a(es) / kWarps;
+  const int tpw = tokens_a(es) / kRowWarps;
   const int64_t rows_chunks = (V + tpw - 1) / tpw;
-  const int piece_chunks = kPieceStages * kWarps;  // csum slots a residual piece uses
+  const int piece_chunks = kPieceStages * kRowWarps;  // csum slots a residual piece uses
   return static_cast<int>(rows_chunks > piece_chunks ? rows_chunks : piece_chunks);
 }
 
@@ -1608,8 +1634,11 @@ size_t slot_bytes(int64_t V, int dtype, int64_t rows) {
 RowGeometry row_geometry(const ScoreArgs& a) {
   RowGeometry geo{};
   const int es = a.dtype == DCD_BF16 ? 2 : 4;
-  const int nst = a.force_stages > 0 ? a.force_stages : (kStageBytes >= 32768 ? 2 : 65536 / kStageBytes);
-  const Layout l = layout_for(a.N, chunks_per_row(a.V, es), nst);
+  // the default ring depth, or fewer stages (at least two) where a large tree or vocabulary
+  // leaves no room for it
+  int nst = a.force_stages > 0 ? a.force_stages : kRingStages;
+  Layout l = layout_for(a.N, chunks_per_row(a.V, es), nst);
+  while (a.force_stages <= 0 && nst > 2 && l.total > kSmemMax) l = layout_for(a.N, chunks_per_row(a.V, es), --nst);
   const int per_sm = static_cast<int>(kSmemPerSm / (l.total + 1024));
   geo.stages = nst;
   geo.stage_tokens = tokens_a(es);
@@ -1647,6 +1676,7 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   sp.chunk_offset = l.chunk_offset;
   sp.stage_offset = l.stage_offset;
   sp.slot_bytes = static_cast<int32_t>(slot_bytes(a.V, a.dtype, R));
+  sp.poll_cycles = a.poll_cycles > 0 ? a.poll_cycles : kWaitCycles;
   sp.hdr = a.hdr;
   sp.jobs = a.jobs;
   sp.slots = a.slots;

@@ -65,7 +65,7 @@ def load(build_if_missing: bool = True):
         lib.dcd_verify_sample_noalloc.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, P, P, P, P]
         lib.dcd_verify_sample_noalloc.restype = I32
         lib.dcd_score_rows_ex.argtypes = [SH, P, P, P, P, P, P, P, P, U64, U64, P, P, P, P, SZ, P,
-                                          ctypes.c_int, ctypes.c_int]
+                                          ctypes.c_int, ctypes.c_int, ctypes.c_int64]
         lib.dcd_tree_walk.argtypes = [SH, P, P, P, P, SZ, P]
         lib.dcd_upload_q_rows.argtypes = [SH, P, P, P, P, P]
         lib.dcd_upload_q_rows.restype = I32
@@ -76,8 +76,8 @@ def load(build_if_missing: bool = True):
                                                    P, P, P]
         lib.dcd_diagnostics_workspace_bytes.argtypes = [SH]
         lib.dcd_diagnostics_workspace_bytes.restype = SZ
-        lib.dcd_row_diagnostics.argtypes = [SH, P, P, P, P, P, P, SZ, P]
-        lib.dcd_row_diagnostics_ex.argtypes = [SH, P, P, P, P, P, P, SZ, P, P, P]
+        lib.dcd_row_diagnostics.argtypes = [SH, P, P, P, P, P, P, P, P, P, P, SZ, P]
+        lib.dcd_row_diagnostics_ex.argtypes = [SH, P, P, P, P, P, P, P, P, P, P, SZ, P, P, P]
         lib.dcd_get_device_error.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
         lib.dcd_status_string.argtypes = [ctypes.c_int]
         lib.dcd_status_string.restype = ctypes.c_char_p
@@ -296,7 +296,7 @@ def dcd_verify_sample_noalloc(z_exp, z_ama, q, tokens, parents, alpha, temperatu
 
 def dcd_score_rows(z_exp, z_ama, tokens, parents, alpha, beta=None, q=None, temperature=None, seed: int = 0,
                    offset: int = 0, *, out=None, workspace=None, stream=None, stages: int = 0,
-                   plain_loads: bool = False, distinct: bool = False) -> dict:
+                   plain_loads: bool = False, distinct: bool = False, poll_limit_cycles: int = 0) -> dict:
     """The per-row step alone (records stay in the workspace); see dcd_tree_walk."""
     c = _Call(z_exp, z_ama, tokens, parents, alpha, beta, q=q, temperature=temperature, distinct=distinct)
     ws = c.workspace(workspace)
@@ -306,8 +306,8 @@ def dcd_score_rows(z_exp, z_ama, tokens, parents, alpha, beta=None, q=None, temp
               _ptr(beta), _ptr(temperature), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
               _ptr(o.get("cd_logprob")), _ptr(o.get("cd_argmax")), _ptr(o.get("cd_lse")), _ptr(ws), ws.numel(),
               _stream(stream))
-    if stages or plain_loads:
-        st = lib.dcd_score_rows_ex(*common, int(stages), int(bool(plain_loads)))
+    if stages or plain_loads or poll_limit_cycles:
+        st = lib.dcd_score_rows_ex(*common, int(stages), int(bool(plain_loads)), int(poll_limit_cycles))
     else:
         st = lib.dcd_score_rows(*common)
     _check(st, "dcd_score_rows")
@@ -382,7 +382,6 @@ def dcd_verify_fused_lmhead(h_exp, w_exp, h_ama, w_ama, tokens, parents, alpha, 
     return o
 
 
-DIAG_FIELDS = ("lse_p", "lse_q", "signal", "e_q", "e_e", "kl_e_p")
 
 
 def diagnostics_workspace_bytes(B: int, N: int, V: int) -> int:
@@ -393,14 +392,21 @@ def diagnostics_workspace_bytes(B: int, N: int, V: int) -> int:
     return int(n)
 
 
-def dcd_row_diagnostics(z_exp, z_ama, B: int, N: int, *, q=None, xstar=None, out=None, workspace=None, stream=None,
-                        pass_events=None) -> torch.Tensor:
-    """Per-row diagnostics [B*N, 6] (columns DIAG_FIELDS): lse_p, lse_q, the signal
+DIAG_COLS = 8
+DIAG_FIELDS = ("lse_p", "lse_q", "signal", "e_q", "e_e", "kl_e_p", "kl_p_q", "kl_p_cd")
+
+
+def dcd_row_diagnostics(z_exp, z_ama, B: int, N: int, *, q=None, xstar=None, cd_lse=None, alpha=None, beta=None,
+                        temperature=None, out=None, workspace=None, stream=None, pass_events=None) -> torch.Tensor:
+    """Per-row diagnostics [B*N, 8] (columns DIAG_FIELDS): lse_p, lse_q, the signal
     |log pi_p(x*) - log pi_q(x*)| at x* = xstar (the CD argmax), E_{pi_q}[log pi_p - log pi_q],
-    and with the drafter's distribution q: E_q[log pi_p - log pi_q] and D_KL(q || pi_p).
+    with the drafter's distribution q: E_q[log pi_p - log pi_q] and D_KL(q || pi_p); then
+    D_KL(pi_p || pi_q) and, given the verification call's cd_lse and alpha (and its beta and
+    temperature, if any), D_KL(pi_p || pi_CD) by the decomposition lemma of App. B.
 
     z_exp, z_ama: [B*N, ld] bf16 or fp32 logits (row stride = their stride); q: [B*N, ldq] fp32
-    or None; xstar: int32 [B*N] or [B, N], or None.  `pass_events` = (start, stop) torch.cuda.Event
+    or None; xstar: int32 [B*N] or [B, N], or None; cd_lse: fp32 [B*N] or [B, N], or None;
+    alpha / beta / temperature: fp32 [B] or None.  `pass_events` = (start, stop) torch.cuda.Event
     pair recorded around the streaming pass.
     """
     _require(z_exp, "z_exp")
@@ -421,13 +427,24 @@ def dcd_row_diagnostics(z_exp, z_ama, B: int, N: int, *, q=None, xstar=None, out
         _require(xstar, "xstar", torch.int32, dev)
         if xstar.numel() != R or not xstar.is_contiguous():
             raise ValueError("xstar must be a contiguous int32 tensor of B*N tokens")
+    if (cd_lse is None) != (alpha is None):
+        raise ValueError("cd_lse and alpha go together (the lemma of App. B needs both)")
+    if cd_lse is not None:
+        _require(cd_lse, "cd_lse", torch.float32, dev)
+        if cd_lse.numel() != R or not cd_lse.is_contiguous():
+            raise ValueError("cd_lse must be a contiguous fp32 tensor of B*N values")
+        _require_vec(alpha, "alpha", B, dev)
+        if beta is not None:
+            _require_vec(beta, "beta", B, dev)
+        if temperature is not None:
+            _require_vec(temperature, "temperature", B, dev)
     sh = make_shape(B, N, V, _logits_dtype(z_exp), ld=z_exp.stride(0), ldq=ldq)
     if workspace is None:
         workspace = torch.empty(diagnostics_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
     if out is None:
-        out = torch.empty(R, 6, dtype=torch.float32, device=dev)
+        out = torch.empty(R, DIAG_COLS, dtype=torch.float32, device=dev)
     else:
-        _require(out, "out", torch.float32, dev, (R, 6))
+        _require(out, "out", torch.float32, dev, (R, DIAG_COLS))
         if not out.is_contiguous():
             raise ValueError("out must be contiguous")
     ev0 = ev1 = None
@@ -436,7 +453,8 @@ def dcd_row_diagnostics(z_exp, z_ama, B: int, N: int, *, q=None, xstar=None, out
             if not e.cuda_event:
                 e.record()
         ev0, ev1 = (ctypes.c_void_p(e.cuda_event) for e in pass_events)
-    st = load().dcd_row_diagnostics_ex(ctypes.byref(sh), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(xstar), _ptr(out),
+    st = load().dcd_row_diagnostics_ex(ctypes.byref(sh), _ptr(z_exp), _ptr(z_ama), _ptr(q), _ptr(xstar),
+                                       _ptr(cd_lse), _ptr(alpha), _ptr(beta), _ptr(temperature), _ptr(out),
                                        _ptr(workspace), workspace.numel(), _stream(stream), ev0, ev1)
     _check(st, "dcd_row_diagnostics")
     return out

@@ -104,7 +104,10 @@ def test_host_checks_reject_before_launch(lib):
     assert lib.dcd_verify_greedy(ctypes.byref(bad), *base, ws_ok, 1 << 20, None) == -1
     # invalid forced ring depth
     assert lib.dcd_score_rows_ex(ctypes.byref(sh), P, P, None, P, P, P, None, None, 0, 0, None, None, None, ws_ok,
-                                 1 << 20, None, 1, 0) == -1
+                                 1 << 20, None, 1, 0, 0) == -1
+    # negative poll limit
+    assert lib.dcd_score_rows_ex(ctypes.byref(sh), P, P, None, P, P, P, None, None, 0, 0, None, None, None, ws_ok,
+                                 1 << 20, None, 0, 0, -1) == -1
     # empty batch is a no-op
     empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
     assert lib.dcd_verify_greedy(ctypes.byref(empty), *base, ws_ok, 1 << 20, None) == 0
@@ -157,16 +160,18 @@ def test_diagnostics_workspace_and_host_checks(lib):
     ws = _fake(0x100000)
     sh = dcd.make_shape(2, 4, 100, dcd.DCD_BF16)
     # null logits or output, sibling flags, q with a short stride, bad workspace: rejected before launch
-    assert lib.dcd_row_diagnostics(ctypes.byref(sh), None, P, None, None, P, ws, 1 << 20, None) == -1
-    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, None, ws, 1 << 20, None) == -1
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), None, P, None, None, None, None, None, None, P, ws, 1 << 20, None) == -1
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, None, None, None, None, None, ws, 1 << 20, None) == -1
     flagged = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, flags=dcd.DCD_SIBLINGS_DISTINCT)
-    assert lib.dcd_row_diagnostics(ctypes.byref(flagged), P, P, None, None, P, ws, 1 << 20, None) == -1
+    assert lib.dcd_row_diagnostics(ctypes.byref(flagged), P, P, None, None, None, None, None, None, P, ws, 1 << 20, None) == -1
     short_q = dcd.make_shape(2, 4, 100, dcd.DCD_BF16, ldq=99)
-    assert lib.dcd_row_diagnostics(ctypes.byref(short_q), P, P, P, None, P, ws, 1 << 20, None) == -1
-    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, P, _fake(0x100010), 1 << 20, None) == -7
-    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, P, ws, 16, None) == -7
+    assert lib.dcd_row_diagnostics(ctypes.byref(short_q), P, P, P, None, None, None, None, None, P, ws, 1 << 20, None) == -1
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, None, None, None, None, P, _fake(0x100010), 1 << 20, None) == -7
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, None, None, None, None, P, ws, 16, None) == -7
     empty = dcd.make_shape(0, 4, 100, dcd.DCD_BF16)
-    assert lib.dcd_row_diagnostics(ctypes.byref(empty), P, P, None, None, P, ws, 1 << 20, None) == 0
+    assert lib.dcd_row_diagnostics(ctypes.byref(empty), P, P, None, None, None, None, None, None, P, ws, 1 << 20, None) == 0
+    # cd_lse without alpha (the lemma needs both)
+    assert lib.dcd_row_diagnostics(ctypes.byref(sh), P, P, None, None, P, None, None, None, P, ws, 1 << 20, None) == -1
 
 
 def test_sampled_row_ranges_merges_adjacent_sequences():

@@ -1,6 +1,9 @@
 """GPU parity of the per-row diagnostics (lse_p, lse_q, the signal at the CD argmax, the
 alignment terms E_{pi_q}[log pi_p - log pi_q], E_q[log pi_p - log pi_q] and D_KL(q || pi_p) of
-Sec. 3.1 / App. C) against the oracle's fp64 definitions on the same rounded inputs.
+Sec. 3.1 / App. C, D_KL(pi_p || pi_q), and D_KL(pi_p || pi_CD) of App. B's decomposition lemma)
+against the oracle's fp64 definitions on the same rounded inputs.  The oracle sums
+D_KL(pi_p || pi_CD) term by term from Eq. 1; the library forms it from the verification call's
+cd_lse by the lemma, so the comparison also checks the lemma on the GPU's numbers.
 
 Bar (DIAG_TOL): |gpu - oracle| <= 1e-4 * max(1, |oracle|) per value.  The kernel accumulates in
 fp32 over at most 16384 tokens a CTA (8 to 64 terms a thread, then tree merges) and merges the
@@ -20,12 +23,17 @@ pytestmark = pytest.mark.gpu
 DIAG_TOL = 1e-4
 
 
-def _oracle_rows(zp, zq, q, xstar, rows, dtype):
-    out = np.full((len(rows), 6), np.nan)
+def _oracle_rows(zp, zq, q, xstar, rows, dtype, alpha=None, lemma=None):
+    """Oracle diagnostics of `rows`; alpha[i] (or None) is the contrast strength of row i's
+    sequence, and lemma[i] says whether its call's target was untruncated at T = 1 (else the
+    last column is NaN, as the library reports it)."""
+    out = np.full((len(rows), dcd.DIAG_COLS), np.nan)
     for i, g in enumerate(rows):
         x = int(xstar[g]) if xstar is not None else 0
         ok = xstar is not None and 0 <= x < zp.shape[1]
-        d = oracle.row_diagnostics(zp[g], zq[g], x if ok else 0, q=None if q is None else q[g].numpy(), dtype=dtype)
+        a = None if alpha is None or (lemma is not None and not lemma[i]) else float(alpha[i])
+        d = oracle.row_diagnostics(zp[g], zq[g], x if ok else 0, q=None if q is None else q[g].numpy(), dtype=dtype,
+                                   alpha=a)
         out[i] = [d[k] for k in dcd.DIAG_FIELDS]
         if not ok:
             out[i, 2] = np.nan
@@ -56,14 +64,19 @@ def test_diagnostics_full_vocab_with_q_and_cd_argmax():
     o = dcd.dcd_verify_greedy(wd.z_exp, wd.z_ama, wd.tokens, wd.parents, wd.alpha, wd.beta)
     xstar = o["cd_argmax"].reshape(-1).contiguous()
     q = wd.q.reshape(R, w.V)
-    got = dcd.dcd_row_diagnostics(wd.z_exp.reshape(R, w.V), wd.z_ama.reshape(R, w.V), w.B, w.N, q=q, xstar=xstar)
+    # the greedy call's cd_lse (reported at T = 1) gives D_KL(pi_p || pi_CD) by the lemma
+    got = dcd.dcd_row_diagnostics(wd.z_exp.reshape(R, w.V), wd.z_ama.reshape(R, w.V), w.B, w.N, q=q, xstar=xstar,
+                                  cd_lse=o["cd_lse"].reshape(-1).contiguous(), alpha=wd.alpha, beta=wd.beta)
     torch.cuda.synchronize()
+    alpha = np.repeat(w.alpha.numpy(), w.N)
+    beta0 = np.repeat((w.beta.numpy() if w.beta is not None else np.zeros(w.B)) == 0, w.N)
     ref = _oracle_rows(w.z_exp.reshape(R, w.V), w.z_ama.reshape(R, w.V), w.q.reshape(R, w.V), xstar.cpu().numpy(),
-                       range(R), "bf16")
+                       range(R), "bf16", alpha=alpha, lemma=beta0)
     _compare(got.cpu().numpy(), ref)
+    assert np.isfinite(got.cpu().numpy()[:, 6:]).all()
     # leaves have q = 0: E_q terms and the divergence vanish
     leaf = (w.q.reshape(R, w.V).sum(dim=1) == 0).numpy()
-    assert leaf.any() and np.all(got.cpu().numpy()[leaf][:, 4:] == 0)
+    assert leaf.any() and np.all(got.cpu().numpy()[leaf][:, 4:6] == 0)
 
 
 def test_diagnostics_f32_out_of_range_xstar():
@@ -112,7 +125,7 @@ def test_diagnostics_unaligned_rows_without_q():
     torch.cuda.synchronize()
     ref = _oracle_rows(w.z_exp.reshape(R, w.V), w.z_ama.reshape(R, w.V), None, None, range(R), "bf16")
     _compare(got.cpu().numpy(), ref)
-    assert np.isnan(got[:, [2, 4, 5]].cpu().numpy()).all()
+    assert np.isnan(got[:, [2, 4, 5, 7]].cpu().numpy()).all()
 
 
 def test_diagnostics_single_token_and_tiny_vocab():
@@ -145,3 +158,28 @@ def test_diagnostics_full_size_batch_sampled_rows():
     qs = q[ridx].cpu()
     ref = _oracle_rows(zp, zq, qs, xs[ridx].cpu().numpy(), range(len(rows)), "bf16")
     _compare(got[ridx].cpu().numpy(), ref)
+
+
+def test_diagnostics_kl_decomposition_lemma_per_sequence():
+    """D_KL(pi_p || pi_CD) from the cd_lse of a sampled call with per-sequence alpha, beta and
+    temperature: sequences at T = 1 with beta = 0 match the oracle's direct sum; a sequence with
+    beta > 0 or with T = 0.5 reports NaN (the lemma holds for the untruncated T = 1 target only)."""
+    dev = torch.device("cuda")
+    w = workloads.make_config(3, B=6, V=9001, seed=24)
+    R = w.B * w.N
+    alpha = torch.tensor([0.0, 0.1, 0.5, 0.2, 1.0, 0.1], dtype=torch.float32)
+    beta = torch.tensor([0.0, 0.0, 0.0, 0.1, 0.0, 0.0], dtype=torch.float32)
+    temp = torch.tensor([1.0, 1.0, 0.0, 1.0, 0.5, 1.0], dtype=torch.float32)
+    wd = w.to(dev)
+    o = dcd.dcd_verify_sample(wd.z_exp, wd.z_ama, wd.q, wd.tokens, wd.parents, alpha.to(dev), temp.to(dev), w.seed, 0,
+                              beta.to(dev))
+    got = dcd.dcd_row_diagnostics(wd.z_exp, wd.z_ama, w.B, w.N, cd_lse=o["cd_lse"].reshape(-1).contiguous(),
+                                  alpha=alpha.to(dev), beta=beta.to(dev), temperature=temp.to(dev))
+    torch.cuda.synchronize()
+    valid = np.repeat(((beta == 0) & ((temp == 0) | (temp == 1))).numpy(), w.N)
+    ref = _oracle_rows(w.z_exp, w.z_ama, None, None, range(R), "bf16", alpha=np.repeat(alpha.numpy(), w.N),
+                       lemma=valid)
+    _compare(got.cpu().numpy(), ref)
+    g = got.cpu().numpy()
+    assert np.isfinite(g[valid, 7]).all() and np.isnan(g[~valid, 7]).all()
+    assert np.abs(g[:w.N, 7]).max() < 1e-4  # alpha = 0: pi_CD = pi_p
