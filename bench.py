@@ -47,6 +47,8 @@ FUSED_WORKLOAD = "fused_lmhead_B64_tree60_V128256_Hexp8192_Hama2048_bf16_greedy"
 METRIC = "verified draft nodes/sec (CD verification step, 1 GPU)"
 DIAG_WORKLOAD = "diagnostics_B32_tree60_V128256_bf16_q_f32"
 DIAG_METRIC = "diagnosed rows/sec (per-row CD diagnostics, 1 GPU)"
+NOMINAL_HBM_GBS = 8000.0
+ROW_WARMUP, ROW_LAUNCHES = 10, 60  # the row kernel's own timing loop  # GB300 HBM3e nominal bandwidth (context; the roofline uses the measured copy)
 
 
 def _peaks():
@@ -191,6 +193,310 @@ def _dist_env():
     return ws, rank, local
 
 
+
+def _parse_cpulist(text: str) -> list:
+    cpus = []
+    for part in text.split(","):
+        if "-" in part:
+            a, b = part.split("-")
+            cpus.extend(range(int(a), int(b) + 1))
+        elif part.strip():
+            cpus.append(int(part))
+    return cpus
+
+
+def gpu_numa_cpus(index: int):
+    """The NUMA node the GPU is attached to (from its PCI device in sysfs) and that node's CPUs;
+    (None, []) where the platform does not say."""
+    try:
+        bus = subprocess.run(["nvidia-smi", "-i", str(index), "--query-gpu=pci.bus_id", "--format=csv,noheader"],
+                             capture_output=True, text=True, timeout=30).stdout.strip()
+        dom, rest = bus.split(":", 1)
+        sysid = f"{int(dom, 16):04x}:{rest}".lower()
+        with open(f"/sys/bus/pci/devices/{sysid}/numa_node") as f:
+            node = int(f.read().strip())
+        if node < 0:
+            return None, []
+        with open(f"/sys/devices/system/node/node{node}/cpulist") as f:
+            return node, _parse_cpulist(f.read().strip())
+    except Exception:
+        return None, []
+
+
+class near_gpu:
+    """Runs the enclosed host allocations on the CPUs of the GPU's NUMA node, so that page-locked
+    buffers are placed in the memory next to it (the allocating thread's node)."""
+
+    def __init__(self, index: int):
+        self.node, self.cpus = gpu_numa_cpus(index)
+        self.saved = None
+
+    def __enter__(self):
+        if self.cpus and hasattr(os, "sched_setaffinity"):
+            self.saved = os.sched_getaffinity(0)
+            try:
+                os.sched_setaffinity(0, self.cpus)
+            except OSError:
+                self.saved = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.saved is not None:
+            os.sched_setaffinity(0, self.saved)
+        return False
+
+
+def _parity_summary(gpu: dict, ref: dict, seqs) -> dict:
+    """Token, length and path mismatches and the largest |cd_logprob| difference of the given
+    sequences (outputs on the host; the oracle's in fp64)."""
+    import numpy as np
+    seqs = list(seqs)
+    al = np.asarray(gpu["accept_len"])[seqs]
+    bo = np.asarray(gpu["bonus"])[seqs]
+    pa = np.asarray(gpu["accept_path"])[seqs]
+    mism = int(((al != ref["accept_len"][seqs]) | (bo != ref["bonus"][seqs]) |
+                (pa != ref["accept_path"][seqs]).any(axis=1)).sum())
+    lg = np.asarray(gpu["cd_logprob"], dtype=np.float64)[seqs]
+    lr = ref["cd_logprob"][seqs]
+    fin = np.isfinite(lr)
+    dl = float(np.abs(lg[fin] - lr[fin]).max()) if fin.any() else 0.0
+    return {"sequences": len(seqs), "mismatched_sequences": mism, "max_abs_dlogprob": dl,
+            "nonfinite_pattern_equal": bool(np.array_equal(np.isfinite(lg), fin))}
+
+
+def small_config(cfg: int, dev, warmup: int = 5, graph_calls: int = 64, reps: int = 4) -> dict:
+    """BASELINE configs 0-2 as one small call each (a 6-node fp32 chain at V = 32000; a 60-node bf16
+    tree at V = 128256, greedy or sampled at T = 1): microseconds per call from CUDA-graph replays of
+    `graph_calls` calls (the host's launch cost left out), eagerly launched, and end to end (inputs
+    from pinned host memory, results back); the oracle on the same inputs, timed on the host cores,
+    and the parity of one call against it."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_12913_gb300 import dcd, workloads
+
+    w_host = workloads.make_config(cfg, margin_fn=oracle.margin_fn)
+    w = w_host.to(dev)
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    sampled = w.q is not None and bool((w.temperature > 0).any())
+    out = dcd.alloc_outputs(B, N, dev)
+    ws = dcd.alloc_workspace(B, N, V, dev, dtype=dcd.DCD_F32 if w.dtype == "f32" else dcd.DCD_BF16)
+    keys = ("z_exp", "z_ama", "q", "tokens", "parents", "alpha", "beta", "temperature")
+    resident = {k: getattr(w, k) for k in keys if getattr(w, k) is not None}
+
+    def call(i, stream, d=resident):
+        if sampled:
+            dcd.dcd_verify_sample(d["z_exp"], d["z_ama"], d["q"], d["tokens"], d["parents"], d["alpha"],
+                                  d["temperature"], w.seed, i, d.get("beta"), out=out, workspace=ws, stream=stream)
+        else:
+            dcd.dcd_verify_greedy(d["z_exp"], d["z_ama"], d["tokens"], d["parents"], d["alpha"], d.get("beta"),
+                                  out=out, workspace=ws, stream=stream)
+
+    stream = torch.cuda.Stream(device=dev)
+    # parity of one call (offset w.offset) against the oracle, and the oracle's time per call
+    with torch.cuda.stream(stream):
+        call(w.offset, stream)
+    stream.synchronize()
+    if dcd.dcd_get_device_error(ws, stream) != 0:
+        raise RuntimeError(f"config {cfg}: device error bits set")
+    gpu = {k: out[k].cpu().numpy() for k in ("accept_len", "accept_path", "bonus", "cd_logprob")}
+    threads = oracle.max_threads()
+    t0 = time.perf_counter()
+    ref = oracle.verify_workload(w_host, nthreads=threads)
+    oracle_s = time.perf_counter() - t0
+    parity = _parity_summary(gpu, ref, range(B))
+    with torch.cuda.stream(stream):
+        for i in range(warmup):
+            call(i, stream)
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for i in range(graph_calls):
+            call(i, stream)
+    graph.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    graph_us = a.elapsed_time(b) * 1e3 / (reps * graph_calls)
+    calls = reps * graph_calls
+    with torch.cuda.stream(stream):
+        a.record(stream)
+        for i in range(calls):
+            call(i, stream)
+        b.record(stream)
+    torch.cuda.synchronize()
+    eager_us = a.elapsed_time(b) * 1e3 / calls
+    with near_gpu(dev.index if dev.index is not None else 0):
+        host = {k: v.cpu().pin_memory() for k, v in resident.items()}
+        res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory() for k in ("accept_len", "accept_path",
+                                                                                     "bonus")}
+    dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
+    h2d = dcd.upload_inputs(host, dst, N, stream)
+    d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+
+    def e2e_call(i):
+        dcd.upload_inputs(host, dst, N, stream)
+        call(i, stream, dst)
+        with torch.cuda.stream(stream):
+            for k in res_host:
+                res_host[k].copy_(out[k], non_blocking=True)
+
+    e2e_call(0)
+    torch.cuda.synchronize()
+    n_e2e = graph_calls
+    a.record(stream)
+    for i in range(n_e2e):
+        e2e_call(i + 1)
+    b.record(stream)
+    torch.cuda.synchronize()
+    e2e_us = a.elapsed_time(b) * 1e3 / n_e2e
+    if dcd.dcd_get_device_error(ws, stream) != 0:
+        raise RuntimeError(f"config {cfg}: device error bits set")
+    path = ("one launch (greedy_small_kernel)" if not sampled and R <= 512 and N <= 256
+            else "persistent row kernel + tree walk")
+    es = 4 if w.dtype == "f32" else 2
+    return {"workload": w.name, "B": B, "N": N, "V": V, "logits": w.dtype, "sampled": sampled, "path": path,
+            "us_per_call_graph": graph_us, "us_per_call_eager": eager_us, "us_per_call_e2e": e2e_us,
+            "nodes_per_s_graph": R / (graph_us / 1e6),
+            "algorithmic_bytes_per_call": float(R * V * 2 * es),
+            "e2e_h2d_bytes_per_call": h2d, "e2e_d2h_bytes_per_call": d2h,
+            "timing": f"{reps} replays of a CUDA graph of {graph_calls} calls; eager and end-to-end: "
+                      f"{calls} and {n_e2e} back-to-back calls",
+            "oracle": {"ms_per_call": oracle_s * 1e3, "cores": threads, "kind": "oracle",
+                       "sample": "the whole call"},
+            "parity": parity}
+
+
+def fused_config(dev, steps: int = 30, warmup: int = 3, soak_s: float = 1.0) -> dict:
+    """BASELINE config 4, the fused LM-head variant (64 x 60 rows, hidden 8192 and 2048, V = 128256,
+    bf16, greedy): the tensor-core launch's TFLOP/s against the measured sustained bf16 peak, from
+    CUDA events around it on every step, with the clocks sampled while it runs; the oracle (fp64
+    logits and the row definition) on one sequence, and that sequence's parity."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_12913_gb300 import dcd, workloads
+
+    w = workloads.make_fused_torch(device=dev, seed=4)
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    H_exp, H_ama = w.h_exp.shape[1], w.h_ama.shape[1]
+    flop = 2.0 * R * V * (H_exp + H_ama)
+    out = dcd.alloc_outputs(B, N, dev)
+    ws = torch.empty(dcd.fused_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(evs=None):
+        dcd.dcd_verify_fused_lmhead(w.h_exp, w.w_exp, w.h_ama, w.w_ama, w.tokens, w.parents, w.alpha, None, out=out,
+                                    workspace=ws, stream=stream, gemm_events=evs)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    if dcd.dcd_get_device_error(ws) != 0:
+        raise RuntimeError("fused: device error bits set")
+    gpu = {k: out[k].cpu().numpy() for k in ("accept_len", "accept_path", "bonus", "cd_logprob")}
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    sampler.start()
+    t_soak = time.time()
+    while time.time() - t_soak < soak_s:
+        step()
+        torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0 = time.time()
+    start.record(stream)
+    for k in range(steps):
+        step(evs[k])
+    stop.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    sampler.stop()
+    gemm_ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+    step_ms = start.elapsed_time(stop) / steps
+    peak, peak_src = _bf16_peak()
+    achieved = flop / (gemm_ms / 1e3) / 1e12
+    threads = oracle.max_threads()
+    t2 = time.perf_counter()
+    ref = oracle.verify_fused_workload(w, nthreads=threads, seqs=[0])
+    oracle_s = time.perf_counter() - t2
+    rows = ref["rows"].reshape(-1)[:N]
+    amb = int((rows["gap_argmax"] < 2e-4).sum())  # within the GEMM's fp32 rounding of the logits
+    parity = _parity_summary(gpu, {k: ref[k] for k in ("accept_len", "accept_path", "bonus", "cd_logprob")}, [0])
+    parity["ambiguous_rows"] = amb
+    return {"workload": FUSED_WORKLOAD, "B": B, "N": N, "V": V, "H_exp": H_exp, "H_ama": H_ama,
+            "ms_per_step": step_ms, "nodes_per_s": R / (step_ms / 1e3),
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                         "frac": achieved / peak, "kernel": "fused_lmhead_kernel", "peak_source": peak_src,
+                         "algorithmic_flops_per_launch": flop, "gemm_kernel_ms": gemm_ms,
+                         "gemm_kernel_samples": steps},
+            "clocks": sampler.summary(t0, t1),
+            "oracle": {"s_per_sequence": oracle_s, "cores": threads, "kind": "oracle",
+                       "sample": f"sequence 0 of {B} ({N} rows: fp64 logits and the row oracle)"},
+            "parity": parity}
+
+
+def diag_config(w, dev, launches: int = 60, warmup: int = 10) -> dict:
+    """The per-row diagnostics pass over a resident batch `w` (its logits and q, x* and cd_lse from a
+    greedy verification call): the streaming kernel's GB/s from CUDA events around each of
+    `launches` launches; the oracle on two rows, timed on one host thread, and their parity."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_12913_gb300 import dcd
+
+    B, N, V = w.B, w.N, w.V
+    R = B * N
+    zp, zq, q = w.z_exp.reshape(R, V), w.z_ama.reshape(R, V), w.q.reshape(R, V)
+    stream = torch.cuda.current_stream()
+    o = dcd.dcd_verify_greedy(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, stream=stream)
+    xstar = o["cd_argmax"].reshape(-1).contiguous()
+    cd_lse = o["cd_lse"].reshape(-1).contiguous()
+    wsd = torch.empty(dcd.diagnostics_workspace_bytes(B, N, V), dtype=torch.uint8, device=dev)
+    diag = torch.empty(R, dcd.DIAG_COLS, dtype=torch.float32, device=dev)
+
+    def step(evs=None):
+        dcd.dcd_row_diagnostics(zp, zq, B, N, q=q, xstar=xstar, cd_lse=cd_lse, alpha=w.alpha, beta=w.beta, out=diag,
+                                workspace=wsd, stream=stream, pass_events=evs)
+
+    for _ in range(warmup):
+        step()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(launches)]
+    torch.cuda.synchronize()
+    for e in evs:
+        step(e)
+    torch.cuda.synchronize()
+    pass_ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+    alg = float(R * V * (2 * 2 + 4))
+    peak, peak_kind = _peaks()
+    achieved = alg / (pass_ms / 1e3) / 1e9
+    rows = [1, R - 1]
+    xs = xstar.cpu().numpy()
+    got = diag[rows].cpu().numpy().astype(np.float64)
+    t0 = time.perf_counter()
+    ref = _diag_oracle_rows(w, rows, xs)
+    oracle_s = time.perf_counter() - t0
+    fin = ~np.isnan(ref)
+    err = np.abs(got[fin] - ref[fin]) / np.maximum(1.0, np.abs(ref[fin]))
+    return {"workload": DIAG_WORKLOAD, "rows": R, "pass_ms": pass_ms, "rows_per_s": R / (pass_ms / 1e3),
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "frac_nominal": achieved / NOMINAL_HBM_GBS, "kernel": "diag_partial_kernel",
+                         "peak_source": f"{peak_kind} hbm_gbs", "algorithmic_bytes_per_launch": alg,
+                         "pass_kernel_samples": launches},
+            "oracle": {"ms_per_row": oracle_s * 1e3 / len(rows), "cores": 1, "kind": "oracle",
+                       "sample": f"rows {rows}, one thread"},
+            "parity": {"rows": len(rows), "max_scaled_error": float(err.max()) if err.size else 0.0,
+                       "nan_pattern_equal": bool(np.array_equal(np.isnan(got), np.isnan(ref)))}}
+
 def run_reference(args):
     """The fp64 CPU oracle timed as the reference arm (rank 0 only)."""
     ws, rank, _ = _dist_env()
@@ -224,14 +530,24 @@ def run_reference(args):
 
 
 def _diag_oracle_rows(w, rows, xstar):
-    """The oracle's diagnostics for the given rows of workload `w` (inputs as stored)."""
+    """The oracle's diagnostics for the given rows of workload `w` (inputs as stored), with the
+    decomposition column for sequences with beta = 0 (greedy, as the benchmark's x* call)."""
+    import numpy as np
+
     import oracle
+    from paper_2608_12913_gb300 import dcd
     R = w.B * w.N
     zp = w.z_exp.reshape(R, w.V)
     zq = w.z_ama.reshape(R, w.V)
     q = w.q.reshape(R, w.V)
-    for g in rows:
-        oracle.row_diagnostics(zp[g].cpu(), zq[g].cpu(), int(xstar[g]), q=q[g].cpu().numpy(), dtype=w.dtype)
+    out = np.full((len(rows), dcd.DIAG_COLS), np.nan)
+    for i, g in enumerate(rows):
+        b = g // w.N
+        beta = 0.0 if w.beta is None else float(w.beta[b])
+        d = oracle.row_diagnostics(zp[g].cpu(), zq[g].cpu(), int(xstar[g]), q=q[g].cpu().numpy(), dtype=w.dtype,
+                                   alpha=float(w.alpha[b]) if beta == 0.0 else None)
+        out[i] = [d[k] for k in dcd.DIAG_FIELDS]
+    return out
 
 
 def run_reference_diagnostics(args, world):
@@ -335,11 +651,6 @@ def run_ours(args):
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
-    # The row kernel's own duration is sampled on every 8th step (the median is reported): an
-    # event between the two launches breaks the tree walk's programmatic dependent launch, so the
-    # other steps run as a user's back-to-back calls do.
-    sampled_steps = list(range(0, args.steps, 8))
-    evs = {k: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for k in sampled_steps}
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
@@ -347,15 +658,27 @@ def run_ours(args):
     t_wall0 = time.time()
     start.record(stream)
     for k in range(args.steps):
-        step(1_000_000 + k, evs.get(k))
+        step(1_000_000 + k)
     stop.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     t_wall1 = time.time()
+    # The row kernel's own duration: CUDA events around each of ROW_LAUNCHES launches after
+    # ROW_WARMUP more, whatever --steps is (an event between the row kernel and the tree walk
+    # breaks the walk's programmatic dependent launch, so the step loop above has none)
+    for k in range(ROW_WARMUP):
+        step(3_000_000 + k)
+    row_evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(ROW_LAUNCHES)]
+    t_row0 = time.time()
+    for k in range(ROW_LAUNCHES):
+        step(4_000_000 + k, row_evs[k])
+    torch.cuda.synchronize()
+    t_row1 = time.time()
     sampler.stop()
     elapsed_ms = start.elapsed_time(stop)
-    row_ms = [a.elapsed_time(b) for a, b in evs.values()]
+    row_ms = [a.elapsed_time(b) for a, b in row_evs]
     if world > 1:
         elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
     if dcd.dcd_get_device_error(ws) != 0:
@@ -365,7 +688,7 @@ def run_ours(args):
 
     # roofline of the dominant kernel (the row kernel) from its own events; the rows that took
     # residual passes are counted on a replay of every 32nd timed offset
-    replay = [1_000_000 + k for k in range(0, args.steps, 32)]
+    replay = [4_000_000 + k for k in range(0, ROW_LAUNCHES, 4)]
     res_rows = residual_rows_per_step(w, out, ws, stream, replay, args.distinct)
     alg = algorithmic_bytes(w, res_rows)
     row_avg_s = statistics.median(row_ms) / 1e3
@@ -375,19 +698,25 @@ def run_ours(args):
     # the profile covers the default workload (32 sequences, mixed, i.i.d. siblings) only
     traffic = _profiled_traffic(khash) if B == 32 and not args.greedy and not args.distinct else None
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "frac_nominal": achieved / NOMINAL_HBM_GBS, "nominal_peak": NOMINAL_HBM_GBS,
                 "traffic": traffic, "kernel": "score_rows_kernel", "peak_source": f"{peak_kind} hbm_gbs",
                 "algorithmic_bytes_per_launch": alg, "residual_rows_per_step": res_rows,
                 "row_kernel_ms": row_avg_s * 1e3, "row_kernel_samples": len(row_ms),
+                "row_kernel_timing": f"median of {ROW_LAUNCHES} event-timed launches after {ROW_WARMUP} warm-ups",
+                "clocks": sampler.summary(t_row0, t_row1),
                 "kernel_source_sha256_16": khash}
 
     # end to end through the public API: pinned host inputs -> device, verify, results -> host
     e2e = None
     if not args.no_e2e:
-        host = {k: getattr(w, k).cpu().pin_memory() for k in ("z_exp", "z_ama", "q", "tokens", "parents", "alpha",
-                                                               "beta", "temperature") if getattr(w, k) is not None}
+        # page-locked buffers in the memory of the GPU's NUMA node (allocated from its CPUs)
+        with near_gpu(local) as place:
+            host = {k: getattr(w, k).cpu().pin_memory() for k in ("z_exp", "z_ama", "q", "tokens", "parents",
+                                                                   "alpha", "beta", "temperature")
+                    if getattr(w, k) is not None}
+            res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory()
+                        for k in ("accept_len", "accept_path", "bonus")}
         dst = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
-        res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory() for k in ("accept_len", "accept_path",
-                                                                                     "bonus")}
         # q is copied only for the sampled sequences: the verification reads no other row of it
         h2d = dcd.upload_inputs(host, dst, N, stream)
         d2h = sum(v.numel() * v.element_size() for v in res_host.values())
@@ -410,10 +739,20 @@ def run_ours(args):
         b2.record(stream)
         torch.cuda.synchronize()
         e_ms = a.elapsed_time(b2) / n_e2e
+        # the host link alone: the same uploads without the verification
+        a.record(stream)
+        for i in range(n_e2e):
+            dcd.upload_inputs(host, dst, N, stream)
+        b2.record(stream)
+        torch.cuda.synchronize()
+        up_ms = a.elapsed_time(b2) / n_e2e
         if world > 1:
             e_ms = max_over_ranks(e_ms, dist, dev)
         e2e = {"value": job_value(world, R, e_ms), "unit": "nodes/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e}
+               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "steps": n_e2e,
+               "h2d_ms_per_step": up_ms, "h2d_gbs": h2d / (up_ms / 1e3) / 1e9,
+               "pinned_numa_node": place.node,
+               "bound": "host link: the step's inputs cross it every step (its rate is h2d_gbs)"}
         del dst, host
 
     if rank == 0:
@@ -434,11 +773,46 @@ def run_ours(args):
         }
         if not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline(w)
+        if not args.no_configs:
+            line["configs"] = all_configs(w, dev, out, ws, stream, line)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
     return 0
+
+
+def all_configs(w, dev, out, ws, stream, line) -> dict:
+    """Every BASELINE configuration measured in the same run, each with the oracle's time on the
+    host cores and a parity summary: the three small calls (0-2), this batch (3, the headline), the
+    fused LM-head variant (4), and the per-row diagnostics pass over this batch."""
+    import oracle
+    from paper_2608_12913_gb300 import dcd
+    res = {}
+    for cfg, key in ((0, "0_tiny_chain"), (1, "1_tree_greedy"), (2, "2_tree_sampled")):
+        res[key] = small_config(cfg, dev)
+    # config 3: the headline (above), with the parity of sequences 0-1 of one call
+    off = 5_000_000
+    dcd.dcd_score_rows(w.z_exp, w.z_ama, w.tokens, w.parents, w.alpha, w.beta, q=w.q, temperature=w.temperature,
+                       seed=w.seed, offset=off, out=out, workspace=ws, stream=stream)
+    dcd.dcd_tree_walk(w.B, w.N, w.V, out, ws, stream=stream)
+    gpu = {k: out[k].cpu().numpy() for k in ("accept_len", "accept_path", "bonus", "cd_logprob")}
+    import dataclasses
+    ref = oracle.verify_workload(dataclasses.replace(w, offset=off), nthreads=oracle.max_threads(), seqs=[0, 1])
+    rows = ref["rows"][:2]
+    amb = int(((rows["gap_argmax"] < 2e-5) | (rows["gap_accept"] < 1e-5) | (rows["gap_race"] < 1e-4)).sum())
+    par = _parity_summary(gpu, ref, [0, 1])
+    par["ambiguous_rows"] = amb
+    cb = line.get("cpu_baseline", {})
+    res["3_batched"] = {"workload": WORKLOAD, "ms_per_step": line["ms_per_step"], "nodes_per_s": line["value"],
+                        "roofline": {k: line["roofline"][k] for k in ("achieved", "peak", "frac", "frac_nominal",
+                                                                        "row_kernel_ms")},
+                        "oracle": {"nodes_per_s": cb.get("value"), "cores": cb.get("cores"),
+                                   "sample": cb.get("sample")},
+                        "parity": par}
+    res["4_fused"] = fused_config(dev)
+    res["diagnostics"] = diag_config(w, dev)
+    return res
 
 
 def run_fused(args):
@@ -883,6 +1257,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (profiling runs)")
     ap.add_argument("--no-soak", action="store_true", help="skip the 1 s clock soak (profiling runs)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-configuration sub-results (small calls, fused, diagnostics)")
     ap.add_argument("--greedy", action="store_true", help="every sequence greedy (profiling case)")
     ap.add_argument("--batch", type=int, default=None,
                     help="sequences per GPU; the benchmark workloads use 32 (batched, diagnostics) and 64 "

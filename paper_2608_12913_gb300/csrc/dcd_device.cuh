@@ -18,7 +18,10 @@ constexpr int kThreads = 256;  // compute threads per CTA of every row kernel (t
 constexpr int kWarps = kThreads / 32;
 constexpr int kRaceBlock = 1024;                  // tokens per block of the two-level terminal race
 constexpr int kSub = 256;                         // tokens a warp handles at once (8 a lane)
-constexpr long long kWaitCycles = 4000000000ll;  // bounded waits: about two seconds at the boost clock
+#ifndef DCD_WAIT_CYCLES
+#define DCD_WAIT_CYCLES 4000000000ll
+#endif
+constexpr long long kWaitCycles = DCD_WAIT_CYCLES;  // bounded waits: about two seconds at the boost clock
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ------------------------------------------------------------------------------------------
@@ -292,6 +295,23 @@ __device__ __forceinline__ float block_sum(float v, float* redf, Sync sync = Syn
   return s;
 }
 
+// Merges (max m, sum s of 2^(x - m), argmax) of two ranges in log2 units (ties to the lower index).
+__device__ __forceinline__ void stats_merge(float& m1, float& s1, int& a1, float m2, float s2, int a2) {
+  const float M = fmaxf(m1, m2);
+  const float t1 = m1 > -INFINITY ? s1 * ex2(m1 - M) : 0.f;
+  const float t2 = m2 > -INFINITY ? s2 * ex2(m2 - M) : 0.f;
+  if (m2 > m1 || (m2 == m1 && a2 < a1)) a1 = a2;
+  m1 = M;
+  s1 = t1 + t2;
+}
+
+// The same over the 32 lanes of a warp: every lane gets the warp's max, rescaled sum and argmax.
+__device__ __forceinline__ void warp_stats(float& m, float& s, int& arg) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1)
+    stats_merge(m, s, arg, __shfl_xor_sync(~0u, m, o), __shfl_xor_sync(~0u, s, o), __shfl_xor_sync(~0u, arg, o));
+}
+
 // Combines per-thread (max m, sum s of 2^(x - m), argmax) over the block in log2 units: every
 // thread gets the block max, the sum rescaled to it, and the argmax (ties to the lowest index).
 template <typename Sync = SyncCta>
@@ -307,8 +327,8 @@ __device__ __forceinline__ void block_stats(float& m, float& s, int& arg, float*
 #pragma unroll
   for (int o = 16; o; o >>= 1)
     merge(m, s, arg, __shfl_xor_sync(~0u, m, o), __shfl_xor_sync(~0u, s, o), __shfl_xor_sync(~0u, arg, o));
-  constexpr int NW = SyncWarps<Sync>::value;  // redf holds 2 * NW <= 32 values
-  static_assert(2 * NW <= 32, "reduction scratch");
+  constexpr int NW = SyncWarps<Sync>::value;  // redf holds 2 * NW values (at least 32 floats)
+  static_assert(2 * NW <= 64, "reduction scratch");
   if ((threadIdx.x & 31) == 0) {
     redf[threadIdx.x >> 5] = m;
     redf[NW + (threadIdx.x >> 5)] = s;

@@ -89,6 +89,11 @@ constexpr int kSmallPieceStages = DCD_SMALL_PIECE_STAGES;
 // then whole rows would leave most CTAs idle for part of the step; with more rows than that,
 // dynamic claiming of whole rows balances better than parts (measured).
 constexpr int kPartsBelow = DCD_PARTS_BELOW;
+#ifndef DCD_TAIL_ROWS
+#define DCD_TAIL_ROWS 0
+#endif
+// In a larger batch, the last kTailRows rows (in claim order) are streamed in parts (0: none).
+constexpr int64_t kTailRows = DCD_TAIL_ROWS;
 constexpr int kDesc = 4;                           // work descriptors in flight per CTA
 #ifndef DCD_ROW_WARPS
 #define DCD_ROW_WARPS 8
@@ -1702,7 +1707,8 @@ cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   const int want = nch_a < kMaxParts ? nch_a : kMaxParts;
   sp.spp = (nch_a + want - 1) / want;
   sp.parts = (nch_a + sp.spp - 1) / sp.spp;
-  const int64_t tail = (sp.parts > 1 && R <= kPartsBelow * resident) ? R : 0;
+  int64_t tail = (sp.parts > 1 && R <= kPartsBelow * resident) ? R : 0;
+  if (sp.parts > 1 && tail == 0) tail = R < kTailRows ? R : kTailRows;
   sp.r_whole = static_cast<int32_t>(R - tail);
   sp.keep_internal = R <= kPartsBelow * resident ? 1 : 0;
   sp.items = static_cast<int32_t>(sp.r_whole + tail * sp.parts);
