@@ -70,7 +70,10 @@ def _bf16_peak():
         return 1700.0, "fallback sustained bf16"
 
 
-def _kernel_source_hash(files=("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h")) -> str:
+ROW_KERNEL_FILES = ("dcd_cluster.cu", "dcd_device.cuh", "dcd_internal.h")
+
+
+def _kernel_source_hash(files=ROW_KERNEL_FILES) -> str:
     h = hashlib.sha256()
     for name in files:
         with open(os.path.join(ROOT, "paper_2608_12913_gb300", "csrc", name), "rb") as f:
@@ -78,7 +81,7 @@ def _kernel_source_hash(files=("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h"
     return h.hexdigest()[:16]
 
 
-def _profiled_traffic(kernel_hash: str, summary: str = "score_rows_kernel_batched_B32_tree60_V128256.md"):
+def _profiled_traffic(kernel_hash: str, summary: str = "cluster_rows_kernel_batched_B32_tree60_V128256.md"):
     """DRAM bytes per launch of a kernel from its committed ncu summary, if it was taken on the
     current kernel source (else None)."""
     path = os.path.join(ROOT, "profiles", summary)
@@ -694,12 +697,15 @@ def run_ours(args):
     row_avg_s = statistics.median(row_ms) / 1e3
     achieved = alg / row_avg_s / 1e9
     peak, peak_kind = _peaks()
-    khash = _kernel_source_hash()
+    # the library streams rows with the cluster-per-row kernel; the distinct-sibling rule takes the
+    # persistent row kernel
+    kname = "score_rows_kernel" if args.distinct else "cluster_rows_kernel"
+    khash = _kernel_source_hash(("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h") if args.distinct else ROW_KERNEL_FILES)
     # the profile covers the default workload (32 sequences, mixed, i.i.d. siblings) only
     traffic = _profiled_traffic(khash) if B == 32 and not args.greedy and not args.distinct else None
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "frac_nominal": achieved / NOMINAL_HBM_GBS, "nominal_peak": NOMINAL_HBM_GBS,
-                "traffic": traffic, "kernel": "score_rows_kernel", "peak_source": f"{peak_kind} hbm_gbs",
+                "traffic": traffic, "kernel": kname, "peak_source": f"{peak_kind} hbm_gbs",
                 "algorithmic_bytes_per_launch": alg, "residual_rows_per_step": res_rows,
                 "row_kernel_ms": row_avg_s * 1e3, "row_kernel_samples": len(row_ms),
                 "row_kernel_timing": f"median of {ROW_LAUNCHES} event-timed launches after {ROW_WARMUP} warm-ups",

@@ -53,6 +53,7 @@
 #include <mutex>
 
 #include "dcd.h"
+#include "dcd_cluster.h"
 #include "dcd_device.cuh"
 #include "dcd_internal.h"
 
@@ -1655,9 +1656,14 @@ RowGeometry row_geometry(const ScoreArgs& a) {
   return geo;
 }
 
+#ifndef DCD_USE_CLUSTER
+#define DCD_USE_CLUSTER 1
+#endif
+
 cudaError_t launch_score_rows(const ScoreArgs& a, cudaStream_t stream) {
   const int64_t R = static_cast<int64_t>(a.B) * a.N;
   if (R == 0) return cudaSuccess;
+  if (DCD_USE_CLUSTER && cluster_rows_ok(a)) return launch_cluster_rows(a, stream);
   const RowGeometry geo = row_geometry(a);
   const int es = a.dtype == DCD_BF16 ? 2 : 4;
   if (geo.smem > kSmemMax || geo.stages < 1 || geo.stages > kMaxStages || geo.ctas_per_sm < 1 ||
