@@ -68,17 +68,24 @@ constexpr int kCMinCtas = DCD_CLUSTER_CTAS_PER_SM;
 constexpr int kCRing = DCD_CLUSTER_RING;
 constexpr int kCMax = DCD_CLUSTER_MAX;
 constexpr int kCFixed = DCD_CLUSTER_C;     // nonzero: this cluster size whenever it fits
-// how a CTA takes a row: whole, its slice of a row split over the cluster, or half of it
-enum RowMode { kWhole = 0, kSplit = 1, kHalf0 = 2, kHalf1 = 3 };
+// how a CTA takes a row: whole, its slice of a row split over the cluster, or one of P parts
+enum RowMode { kWhole = 0, kSplit = 1, kPart = 2 };
 constexpr int kMail = 4;                   // row messages in flight from a cluster's first CTA
 constexpr int kCDesc = 2;                  // rows handed to the consumers ahead
 constexpr int kSeqListMax = 1024;
 #ifndef DCD_CLUSTER_HALF_ROWS
-#define DCD_CLUSTER_HALF_ROWS (1 << 30)
+#define DCD_CLUSTER_HALF_ROWS -1
 #endif
-// The last kHalfRows greedy rows of phase 2 go out as two half-row units each, so that the
-// step's last units are short; the halves combine through the workspace (a ticket per row).
-constexpr int kHalfRows = DCD_CLUSTER_HALF_ROWS;          // sequences up to which the row order lists them in shared memory
+#ifndef DCD_CLUSTER_QUARTER_ROWS
+#define DCD_CLUSTER_QUARTER_ROWS 0
+#endif
+// The greedy rows of phase 2 go out whole, then (the last kHalfRows + kQuarterRows) as two, then
+// (the last kQuarterRows) as four part units each, so that the step's last units are short; a
+// row's parts combine through the workspace (a ticket per row).  kHalfRows < 0: one wave (the
+// grid's CTAs) of rows in halves (measured best: all rows in halves or quarters was slower).
+constexpr int kHalfRows = DCD_CLUSTER_HALF_ROWS;
+constexpr int kQuarterRows = DCD_CLUSTER_QUARTER_ROWS;
+static_assert(kMaxParts >= 4, "part records");          // sequences up to which the row order lists them in shared memory
 static_assert(kCMax >= 1 && kCMax <= kCMaxCluster, "cluster size");
 constexpr float kLn2c = 0.69314718055994531f;
 #ifdef DCD_CLUSTER_DEBUG
@@ -91,14 +98,19 @@ __device__ __forceinline__ unsigned long long gtimer() {
   return t;
 }
 #define CL_T(var) const unsigned long long var = gtimer()
+#define CL_ACC(acc, t0) (acc += gtimer() - (t0))
 #define CL_REC(g, split, t0, t1, npass, m)                                                           \
   do {                                                                                              \
     const uint32_t ei = atomicAdd(&p.hdr->reserved[2], 1u);                                         \
-    if (ei < 16384u) {                                                                              \
-      uint32_t* r = reinterpret_cast<uint32_t*>(p.slots) + 8u * ei;                                 \
+    if (ei < 8192u) {                                                                               \
+      uint32_t* r = reinterpret_cast<uint32_t*>(p.slots) + 16u * ei;                                \
+      r[8] = static_cast<uint32_t>(w_full);                                                         \
+      r[9] = static_cast<uint32_t>(w_xchg);                                                         \
+      r[10] = static_cast<uint32_t>(w_desc);                                                        \
       const unsigned long long t2 = gtimer();                                                        \
       r[0] = blockIdx.x;                                                                            \
-      r[1] = static_cast<uint32_t>(g) | (split ? 0x80000000u : 0u);                                 \
+      r[1] = static_cast<uint32_t>(g);                                                              \
+      r[11] = static_cast<uint32_t>(split);                                                         \
       r[2] = static_cast<uint32_t>(t0);                                                             \
       r[3] = static_cast<uint32_t>(t0 >> 32);                                                       \
       r[4] = static_cast<uint32_t>(t1 - t0);                                                        \
@@ -112,6 +124,7 @@ __device__ __forceinline__ unsigned long long gtimer() {
 #define CL_T(var) \
   const unsigned long long var = 0;  \
   (void)var
+#define CL_ACC(acc, t0) ((void)0)
 #define CL_REC(g, split, t0, t1, npass, m) ((void)0)
 #endif
 using CSync = SyncConsumersN<kCThreads>;
@@ -486,7 +499,9 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     auto nop = [] {};
 
     // ---- phase 1: the sampled sequences' rows, each split over the cluster.  The cluster's first
-    // CTA claims them (one ahead) and sends each to the others as message k.
+    // CTA claims them and sends each to the others as message k: one row ahead after a row that
+    // cannot start a residual chain, else once the row's chain is settled (a row claimed ahead of
+    // a long chain would wait for it, and finish last).
     int next_i = 0, g_next = -1;
     auto send = [&](uint32_t k, int gr) {  // rank 0, lane 0
       const int d = static_cast<int>(k % kMail);
@@ -522,7 +537,6 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             if (g >= 0) arrive_cluster(map_rank(&mempty[d], 0u));  // the last message is not acknowledged
           }
         }
-        if (rank == 0 && g >= 0) next_i = static_cast<int>(atomicAdd(&p.hdr->work, 1u));  // one row ahead
       }
       g = __shfl_sync(~0u, g, 0);
       if (g < 0) break;
@@ -530,11 +544,12 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       const bool masked = (mt.flags & 4) != 0;
       const bool has_child = (mt.flags & 2) != 0;  // a sampled node with a child may start a residual chain
       if (lane == 0) {
+        if (rank == 0 && !has_child) next_i = static_cast<int>(atomicAdd(&p.hdr->work, 1u));  // one row ahead
         hand(mt);
         if (masked) stream(g, sl_lo, sl_hi, cp.tok_a, 0, pol_last, nop);  // the statistics pass re-reads it
         // the slice of a node with a child stays in L2 for the residual pass that may follow
         stream(g, sl_lo, sl_hi, cp.tok_a, 1, has_child ? pol_normal : pol_first, [&] {
-          if (rank == 0) {
+          if (rank == 0 && !has_child) {
             g_next = next_i < nA ? row1(next_i) : -1;
             send(k + 1u, g_next);
           }
@@ -554,17 +569,24 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           }
           stream(g, sl_lo, sl_hi, cp.tok_r, 2, keep ? pol_normal : pol_first, nop);
         }
+        if (rank == 0 && has_child) {  // the row's chain is settled: the cluster's next row
+          next_i = stop ? nA : static_cast<int>(atomicAdd(&p.hdr->work, 1u));
+          g_next = next_i < nA ? row1(next_i) : -1;
+          send(k + 1u, g_next);
+        }
       }
       stop = __shfl_sync(~0u, stop ? 1 : 0, 0) != 0;
     }
     // ---- phase 2: every other row, whole or (the last nH) as two half-row units, claimed by each
     // CTA on its own (one ahead)
     const int nB = R - nA;
-    const int nH = seqs ? (nB < kHalfRows ? nB : kHalfRows) : 0;  // greedy rows when listed
-    const int nW = nB - nH;
-    const int units = nW + 2 * nH;
+    // rows in parts (greedy rows when listed): the last nQ in quarters, the nH before them in halves
+    const int nQ = seqs ? (nB < kQuarterRows ? nB : kQuarterRows) : 0;
+    const int want_h = kHalfRows < 0 ? static_cast<int>(gridDim.x) : kHalfRows;
+    const int nH = seqs ? (nB - nQ < want_h ? nB - nQ : want_h) : 0;
+    const int nW = nB - nH - nQ;
+    const int units = nW + 2 * nH + 4 * nQ;
     const int nch_a = static_cast<int>((V + cp.tok_a - 1) / cp.tok_a);
-    const int64_t half = static_cast<int64_t>((nch_a + 1) / 2) * cp.tok_a;  // part 1 starts here
     int i2 = 0;
     if (lane == 0 && !stop) i2 = static_cast<int>(atomicAdd(&p.hdr->job_alloc, 1u));
     while (!stop) {
@@ -575,15 +597,25 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             g = -1;
             break;
           }
-          const int part = i2 < nW ? -1 : (i2 - nW) & 1;
-          g = row2(i2 < nW ? i2 : nW + (i2 - nW) / 2);
-          // a row with beta > 0 needs its expert max over the whole row: its first unit takes it whole
-          const bool whole = part < 0 || (p.beta && p.beta[g / N] > 0.f) || half >= V;
-          if (whole && part == 1) {
+          int r2 = i2, P = 1, part = 0;
+          if (i2 >= nW + 2 * nH) {
+            r2 = nW + nH + (i2 - nW - 2 * nH) / 4;
+            P = 4;
+            part = (i2 - nW - 2 * nH) & 3;
+          } else if (i2 >= nW) {
+            r2 = nW + (i2 - nW) / 2;
+            P = 2;
+            part = (i2 - nW) & 1;
+          }
+          g = row2(r2);
+          // a row with beta > 0 needs its expert max over the whole row: its first unit takes it
+          // whole; so does a row with fewer stages than parts
+          const bool whole = P == 1 || (p.beta && p.beta[g / N] > 0.f) || nch_a < P;
+          if (whole && part > 0) {
             i2 = static_cast<int>(atomicAdd(&p.hdr->job_alloc, 1u));
             continue;
           }
-          mode = whole ? kWhole : (part == 0 ? kHalf0 : kHalf1);
+          mode = whole ? kWhole : (kPart | (P << 4) | (part << 8));
           break;
         }
         if (g >= 0) i2 = static_cast<int>(atomicAdd(&p.hdr->job_alloc, 1u));
@@ -593,7 +625,12 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       const Meta mt = meta_of(g, mode);
       if (lane == 0) hand(mt);
       if (g < 0) break;
-      const int64_t lo = mode == kHalf1 ? half : 0, hi = mode == kHalf0 ? half : V;
+      int64_t lo = 0, hi = V;
+      if ((mode & 15) == kPart) {
+        const int P = (mode >> 4) & 15, part = mode >> 8, spp = (nch_a + P - 1) / P;
+        lo = static_cast<int64_t>(part) * spp * cp.tok_a;
+        hi = static_cast<int64_t>(part + 1) * spp * cp.tok_a < V ? static_cast<int64_t>(part + 1) * spp * cp.tok_a : V;
+      }
       const bool masked = (mt.flags & 4) != 0;
       // a whole row of a sampled sequence (a batch without the sequence list) may start a chain
       const bool sampled = (mt.flags & 1) != 0;
@@ -630,11 +667,17 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
   uint32_t seq = 0;  // ring stages consumed
   uint32_t xk = 0;   // exchanges done (the same count in every CTA of the cluster)
   bool timed_out = false;
+  unsigned long long w_full = 0, w_xchg = 0, w_desc = 0;  // debug builds: time spent waiting
+  (void)w_full;
+  (void)w_xchg;
+  (void)w_desc;
   auto wait_full = [&](uint32_t sq) {
+    CL_T(tw);
     if (!mbar_wait_bounded(&full[sq % static_cast<uint32_t>(cp.nst)], (sq / static_cast<uint32_t>(cp.nst)) & 1u)) {
       timed_out = true;
       CL_SITE(5);
     }
+    CL_ACC(w_full, tw);
   };
   auto release = [&](uint32_t sq) {
     __syncwarp();
@@ -655,7 +698,10 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       st_cluster_v4(dst + 16u, w[1]);
       arrive_cluster(map_rank(&xbar[buf], static_cast<uint32_t>(tid)));
     }
-    if (!wait_cluster_bounded(&xbar[buf], (xk >> 1) & 1u)) {
+    CL_T(tx);
+    const bool xok = wait_cluster_bounded(&xbar[buf], (xk >> 1) & 1u);
+    CL_ACC(w_xchg, tx);
+    if (!xok) {
       timed_out = true;
       if (tid == 0) atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
       CL_SITE(6);
@@ -671,7 +717,10 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
 
   for (uint32_t k = 0;; ++k) {
     const int dd = static_cast<int>(k % kCDesc);
-    if (!mbar_wait_bounded(&dfull[dd], (k / kCDesc) & 1u)) {
+    CL_T(td);
+    const bool dok = mbar_wait_bounded(&dfull[dd], (k / kCDesc) & 1u);
+    CL_ACC(w_desc, td);
+    if (!dok) {
       if (tid == 0) atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
       CL_SITE(7);
       break;
@@ -684,7 +733,8 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     const float beta = __int_as_float(dsc[4]);
     const float T = __int_as_float(dsc[5]);
     const bool split = mode == kSplit;
-    const bool halfrow = mode == kHalf0 || mode == kHalf1;
+    const bool halfrow = (mode & 15) == kPart;  // one of P parts of a row
+    const int nparts_row = halfrow ? (mode >> 4) & 15 : 1, mypart = halfrow ? mode >> 8 : 0;
     csync();  // every consumer has read the descriptor
     if (tid == 0) mbar_arrive(&dempty[dd]);
     if (gi < 0) break;
@@ -700,10 +750,14 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     const TIn* zq_row = static_cast<const TIn*>(p.zq) + g * p.ld;
     const float* q_row = sampled ? p.q + g * p.ldq : nullptr;
     // a row split over the cluster: this CTA's slice, statistics exchanged; a whole row: [0, V);
-    // half a row: [0, half) or [half, V), combined through the workspace
-    const int64_t half = static_cast<int64_t>((static_cast<int>((V + cp.tok_a - 1) / cp.tok_a) + 1) / 2) * cp.tok_a;
-    const int64_t x_lo = split ? sl_lo : (mode == kHalf1 ? half : 0);
-    const int64_t x_hi = split ? sl_hi : (mode == kHalf0 ? half : V);
+    // part q of P: whole stages [q spp, (q + 1) spp), combined through the workspace
+    int64_t x_lo = split ? sl_lo : 0, x_hi = split ? sl_hi : V;
+    if (halfrow) {
+      const int spp = (static_cast<int>((V + cp.tok_a - 1) / cp.tok_a) + nparts_row - 1) / nparts_row;
+      x_lo = static_cast<int64_t>(mypart) * spp * cp.tok_a;
+      const int64_t e = static_cast<int64_t>(mypart + 1) * spp * cp.tok_a;
+      x_hi = e < V ? e : V;
+    }
     bool leader = !split || rank == 0;  // writes the row's outputs
     timed_out = false;
     CL_T(t_row0);
@@ -820,10 +874,10 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       block_stats(M, S, arg, redf, redi, csync);  // its barriers also publish warp 1's child list
       const int m = sh->m;
       if (halfrow) {
-        // half a (greedy) row: publish its statistics; the CTA that finishes the second half
+        // a part of a (greedy) row: publish its statistics; the CTA that finishes the last part
         // combines them in part order and finishes the row
         if (tid == 0) {
-          const int part = mode == kHalf1 ? 1 : 0;
+          const int part = mypart;
           RowPart rp;
           rp.M = M;
           rp.S = S;
@@ -834,22 +888,24 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           rp.pad[0] = rp.pad[1] = 0;
           p.parts[g * kMaxParts + part] = rp;
           const uint32_t t = atomic_add_acq_rel(&p.pdone[g], 1u);
-          sh->decision = t == 1u ? 1 : 0;
-          if (t == 1u) {
-            const RowPart o = p.parts[g * kMaxParts + (1 - part)];
+          const bool last = t + 1u == static_cast<uint32_t>(nparts_row);
+          sh->decision = last ? 1 : 0;
+          if (last) {
             float cM = -INFINITY, cS = 0.f;
-            int carg = INT_MAX;
-            const RowPart q0 = part == 0 ? rp : o, q1 = part == 0 ? o : rp;
-            stats_merge(cM, cS, carg, q0.M, q0.S, q0.arg);
-            stats_merge(cM, cS, carg, q1.M, q1.S, q1.arg);
+            int carg = INT_MAX, tmo = 0;
+            for (int q = 0; q < nparts_row; ++q) {  // part order: the result does not depend on timing
+              const RowPart o = q == part ? rp : p.parts[g * kMaxParts + q];
+              stats_merge(cM, cS, carg, o.M, o.S, o.arg);
+              tmo |= o.timed_out;
+            }
             sh->c = cM;  // (scratch: the combined statistics)
             sh->D = cS;
             sh->term = carg;
-            sh->degen = (q0.timed_out | q1.timed_out) ? 1 : 0;
+            sh->degen = tmo;
           }
         }
         csync();
-        if (sh->decision == 0) goto row_done;  // the other half finishes the row
+        if (sh->decision == 0) goto row_done;  // another part finishes the row
         M = sh->c;
         S = sh->D;
         arg = sh->term;
@@ -1185,7 +1241,8 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     }
   row_done:
     csync();  // the row's shared state (children, chunk masses) is rewritten by the next row
-    if (tid == 0) CL_REC(gi, split, t_row0, t_dec, npass, sh->m);
+    if (tid == 0) CL_REC(gi, mode, t_row0, t_dec, npass, sh->m);
+    w_full = w_xchg = w_desc = 0;
     (void)t_dec;
     (void)npass;
   }
