@@ -100,8 +100,10 @@ enum { DCD_F32 = 0, DCD_BF16 = 1 };
  * is tested against r_{j-1} with its actual proposal q_{j-1} = q without the tokens of siblings
  * 1..j-1, renormalised, which also replaces q in the residual step r_j = normalise(max(0,
  * r_{j-1} - q_{j-1})).  Without the flag siblings are taken as i.i.d. draws from q.  The flag
- * supports nodes with at most 32 children (more: DCD_DEVERR_UNSUPPORTED for the sequence); the
- * remaining mass of q is taken as 1 minus the removed tokens' q (q rows sum to 1).
+ * supports nodes with at most 32 children (more: DCD_DEVERR_UNSUPPORTED for the sequence).  q
+ * is taken as given: the first sibling's proposal is q itself, and a renormalised proposal
+ * divides by the mass that remains, q's own sum (measured in the first residual pass; a
+ * top-k-truncated drafter's rows sum to less than 1) less the removed tokens' q.
  */
 #define DCD_SIBLINGS_DISTINCT 0x1
 

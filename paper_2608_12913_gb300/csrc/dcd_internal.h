@@ -90,7 +90,7 @@ struct PiecePart {  // one piece's share of a residual pass
   float z;          // sum of max(0, pi - c_J q) over the piece
   float key;        // best race key of the piece's blocks (last pass only)
   int32_t blk;      // its block
-  int32_t timed_out;
+  float qs;         // sum of q over the piece (first pass, distinct siblings only)
 };
 static_assert(sizeof(PiecePart) == 16, "PiecePart layout");
 

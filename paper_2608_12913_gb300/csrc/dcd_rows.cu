@@ -709,7 +709,10 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
       const int64_t piece_lo = static_cast<int64_t>(piece) * sp.piece_stages * sp.tok_r;
       const int64_t rem = (V - piece_lo + sp.tok_r - 1) / sp.tok_r;
       const int nst_piece = static_cast<int>(rem < sp.piece_stages ? rem : sp.piece_stages);
-      float zl = 0.f;
+      // distinct siblings: the first pass also sums q, whose actual mass (the drafter's q may be
+      // truncated or rounded away from 1) normalises the proposal once a token is removed
+      const bool sum_q = kDistinct && J == 1;
+      float zl = 0.f, ql = 0.f;
       for (int L = 0; L < nst_piece; ++L, ++seq) {
         const Stage<TIn> st = stage_at<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(sp.nst)), sp.tok_r);
         const int64_t x0 = piece_lo + static_cast<int64_t>(L) * sp.tok_r;
@@ -724,6 +727,10 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
 #pragma unroll
           for (int e = 0; e < 8; ++e)
             part += (i0 + e < clen) ? fmaxf(ex2(u[e] - M) * invS - cJ * qv[e], 0.f) : 0.f;
+          if (sum_q) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) ql += (i0 + e < clen) ? qv[e] : 0.f;
+          }
         }
         zl += part;
         if (race) {
@@ -733,6 +740,7 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         warp_release(&empty[seq % static_cast<uint32_t>(sp.nst)]);
       }
       const float zsum = block_sum(zl, redf, csync);  // its barriers also publish csum
+      const float qsum = sum_q ? block_sum(ql, redf, csync) : 0.f;
       // race keys of the piece's blocks (the pass after the last sibling)
       float bk = -INFINITY;
       int bb = INT_MAX;
@@ -766,7 +774,9 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         pp.z = zsum;
         pp.key = bk;
         pp.blk = bb;
-        pp.timed_out = timed_out ? 1 : 0;
+        pp.qs = qsum;
+        // a wait that gave up fails the call (the tree walk reads the error word)
+        if (timed_out) atomicOr(&sp.hdr->err, DCD_DEVERR_TIMEOUT);
         slot_parts(sp, D.slot)[piece] = pp;
         const uint32_t t = atomic_add_acq_rel(&sp.jobs[D.job].done, 1u);
         rs->last = t + 1u == static_cast<uint32_t>(sp.npieces) ? 1 : 0;
@@ -804,15 +814,16 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
         if (warp == 1 && lane == 0) {
           // the pieces' partial sums and race keys, read while warp 0 lists the children
           const PiecePart* parts = slot_parts(sp, D.slot);
-          float DJ = 0.f, K = -INFINITY;
+          float DJ = 0.f, K = -INFINITY, QS = 0.f;
           int kstar = INT_MAX;
           uint32_t st2 = D.status;
           for (int k = 0; k < sp.npieces; ++k) {  // a fixed order
             DJ += parts[k].z;
+            QS += parts[k].qs;
             argmax_merge(K, kstar, parts[k].key, parts[k].blk);
-            if (parts[k].timed_out) st2 |= DCD_DEVERR_TIMEOUT;
           }
           rs->D = DJ;
+          rs->c = QS;  // (consumer scratch: the mass of q, first pass of distinct siblings)
           rs->term = kstar;
           rs->status = st2;
         }
@@ -835,7 +846,8 @@ __global__ void __launch_bounds__(kCtaThreads, kMinCtasPerSm) score_rows_kernel(
             // the proposal q / Z without the removed tokens.
             Removed* rem = slot_removed(sp, D.slot);
             int nrem = rs->rn;
-            float Z = sh->Z;
+            // the proposal's mass: q's own before the first removal (then less the removed q)
+            float Z = J == 1 ? rs->c : sh->Z;
             // the values read before the barrier; a token not among them is loaded here
             auto value_of = [&](int t, float& pit, float& qt) {
               for (int i = 0; i < nrem; ++i)
@@ -1510,14 +1522,20 @@ __global__ void __launch_bounds__(kThreads) terminal_residual_kernel(const Score
   __shared__ int removed[kMaxRemoved];
   __shared__ float zrem;
   int nrem = 0;
-  if (threadIdx.x == 0) zrem = 1.f;
+  float qtot = 0.f;  // the mass of q (the drafter's q need not sum to 1)
+  if (p.distinct) {
+    for (int64_t x = threadIdx.x; x < V; x += kThreads) qtot += q[x];
+    qtot = block_sum(qtot, redf);
+  }
+  if (threadIdx.x == 0) zrem = qtot;
   __syncthreads();
   for (int c = cur + 1; c < N; ++c) {
     if (p.parents[static_cast<int64_t>(b) * N + c] != cur) continue;
-    // the proposal of this sibling: q, or (distinct siblings) q without the removed tokens / Z
+    // the proposal of this sibling: q, or (distinct siblings, once a token is removed) q without
+    // the removed tokens over their remaining mass Z
     const float Z = zrem;
     auto prop = [&](int64_t x) -> float {
-      if (!p.distinct) return q[x];
+      if (!p.distinct || nrem == 0) return q[x];
       for (int i = 0; i < nrem; ++i)
         if (removed[i] == x) return 0.f;
       return Z > 0.f ? q[x] / Z : 0.f;

@@ -108,3 +108,32 @@ def test_distinct_lossless_on_the_gpu_monte_carlo():
                                  alpha, 0.0, T)["logpi"])
     counts = np.bincount(first, minlength=V)
     assert stats.chisquare(counts, B * pi).pvalue > 1e-4
+
+
+def _unnormalised(w, kind):
+    """q rows whose mass is not 1: a drafter's top-k truncation (the mass outside the top 64
+    tokens dropped, not renormalised), or every row scaled by 0.93."""
+    q = w.q.clone()
+    if kind == "topk":
+        keep = torch.topk(q, 64, dim=1).indices
+        mask = torch.zeros_like(q, dtype=torch.bool)
+        mask.scatter_(1, keep, True)
+        q = torch.where(mask, q, torch.zeros_like(q))
+    else:
+        q = q * 0.93
+    w.q = q
+    return w
+
+
+@pytest.mark.parametrize("kind", ["topk", "scaled"])
+@pytest.mark.parametrize("distinct", [True, False])
+def test_unnormalised_draft_rows(kind, distinct):
+    # Both rules take q as given: the i.i.d. rule uses it as is, the distinct rule renormalises
+    # by the mass that remains after a removal, q's own mass less the removed tokens' (a
+    # top-k-truncated drafter sends rows that sum to less than 1).
+    w = _unnormalised(workloads.make_config(2, V=4099, B=6, seed=37, margin_fn=oracle.margin_fn), kind)
+    g = run_gpu(w, sampled=True, residual=True, distinct=distinct)
+    r = oracle.verify_workload(w, nthreads=oracle.max_threads(), want_residual=True, distinct=distinct)
+    compare(w, g, r, check_residual=True)
+    mass = w.q.double().sum(dim=1)
+    assert float((mass - 1.0).abs().max()) > 0.05  # the rows really are unnormalised
