@@ -37,7 +37,10 @@ def test_random_fused_case_matches_oracle(i):
     if spec["beta"] > 0:
         gpu = run_fused_gpu(w, beta=w.beta)
         ref = oracle.verify_fused_workload(w, nthreads=oracle.max_threads())
-        compare(w, gpu, ref, amb_mask=FUSED_AMB_MASK, max_amb_frac=0.5, score_tol=FUSED_SCORE_TOL)
+        res = compare(w, gpu, ref, amb_mask=FUSED_AMB_MASK, max_amb_frac=0.5, score_tol=FUSED_SCORE_TOL)
+        # the observed error of masked rows (shown with pytest -s), against the bar it is held to
+        print(f"masked fused rows (case {i}): max |cd_lse err| {res['max_lse_err']:.3g}, "
+              f"max |cd_logprob err| {res['max_logprob_err']:.3g} (bar {FUSED_SCORE_TOL:g})")
     else:
         gpu = run_fused_gpu(w)
         ref = oracle.verify_fused_workload(w, nthreads=oracle.max_threads())
