@@ -73,6 +73,13 @@ enum RowMode { kWhole = 0, kSplit = 1, kPart = 2 };
 constexpr int kMail = 4;                   // row messages in flight from a cluster's first CTA
 constexpr int kCDesc = 2;                  // rows handed to the consumers ahead
 constexpr int kSeqListMax = 1024;
+#ifndef DCD_CLUSTER_HOLD_MAX
+#define DCD_CLUSTER_HOLD_MAX 2
+#endif
+// A cluster claims its next sampled row one ahead of a node with at most kHoldMax children (a
+// rejection there starts a chain of at most kHoldMax passes, which the row claimed ahead waits
+// out); after a wider node it claims once the first sibling is decided or the chain settled.
+constexpr int kHoldMax = DCD_CLUSTER_HOLD_MAX;
 #ifndef DCD_CLUSTER_HALF_ROWS
 #define DCD_CLUSTER_HALF_ROWS -1
 #endif
@@ -472,12 +479,13 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       mt.alpha = p.alpha[b];
       mt.beta = p.beta ? p.beta[b] : 0.f;
       mt.T = p.temp ? p.temp[b] : 0.f;
-      bool has_child = false;
-      for (int base = n + 1; base < N && !has_child; base += 32) {
+      int nkids = 0;
+      for (int base = n + 1; base < N; base += 32) {
         const int c = base + lane;
-        has_child = __ballot_sync(~0u, c < N && p.parents[static_cast<int64_t>(b) * N + c] == n) != 0u;
+        nkids += __popc(__ballot_sync(~0u, c < N && p.parents[static_cast<int64_t>(b) * N + c] == n));
       }
-      mt.flags = ((mt.T > 0.f && p.q != nullptr) ? 1 : 0) | (has_child ? 2 : 0) | (mt.beta > 0.f ? 4 : 0);
+      mt.flags = ((mt.T > 0.f && p.q != nullptr) ? 1 : 0) | (nkids > 0 ? 2 : 0) | (mt.beta > 0.f ? 4 : 0) |
+                 ((nkids > kHoldMax ? 1 : 0) << 3);
       return mt;
     };
     auto hand = [&](const Meta& mt) {  // lane 0: the next row descriptor for the consumers
@@ -499,9 +507,9 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     auto nop = [] {};
 
     // ---- phase 1: the sampled sequences' rows, each split over the cluster.  The cluster's first
-    // CTA claims them and sends each to the others as message k: one row ahead after a row that
-    // cannot start a residual chain, else once the row's chain is settled (a row claimed ahead of
-    // a long chain would wait for it, and finish last).
+    // CTA claims them and sends each to the others as message k: one row ahead of a node with at
+    // most kHoldMax children, else once the node's first sibling is accepted or its chain is
+    // settled (a row claimed ahead of a long chain would wait for it, and finish last).
     int next_i = 0, g_next = -1;
     auto send = [&](uint32_t k, int gr) {  // rank 0, lane 0
       const int d = static_cast<int>(k % kMail);
@@ -543,15 +551,18 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       const Meta mt = meta_of(g, kSplit);
       const bool masked = (mt.flags & 4) != 0;
       const bool has_child = (mt.flags & 2) != 0;  // a sampled node with a child may start a residual chain
+      const bool wide = (mt.flags & 8) != 0;       // more than kHoldMax children
       if (lane == 0) {
-        if (rank == 0 && !has_child) next_i = static_cast<int>(atomicAdd(&p.hdr->work, 1u));  // one row ahead
+        bool sent = false;
+        if (rank == 0 && !wide) next_i = static_cast<int>(atomicAdd(&p.hdr->work, 1u));  // one row ahead
         hand(mt);
         if (masked) stream(g, sl_lo, sl_hi, cp.tok_a, 0, pol_last, nop);  // the statistics pass re-reads it
         // the slice of a node with a child stays in L2 for the residual pass that may follow
         stream(g, sl_lo, sl_hi, cp.tok_a, 1, has_child ? pol_normal : pol_first, [&] {
-          if (rank == 0 && !has_child) {
+          if (rank == 0 && !wide) {
             g_next = next_i < nA ? row1(next_i) : -1;
             send(k + 1u, g_next);
+            sent = true;
           }
         });
         for (; has_child; ++ncmd) {
@@ -569,7 +580,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           }
           stream(g, sl_lo, sl_hi, cp.tok_r, 2, keep ? pol_normal : pol_first, nop);
         }
-        if (rank == 0 && has_child) {  // the row's chain is settled: the cluster's next row
+        if (rank == 0 && !sent) {  // a wide node's first sibling decided or its chain settled
           next_i = stop ? nA : static_cast<int>(atomicAdd(&p.hdr->work, 1u));
           g_next = next_i < nA ? row1(next_i) : -1;
           send(k + 1u, g_next);
