@@ -362,7 +362,7 @@ def small_config(cfg: int, dev, warmup: int = 5, graph_calls: int = 64, reps: in
     if dcd.dcd_get_device_error(ws, stream) != 0:
         raise RuntimeError(f"config {cfg}: device error bits set")
     path = ("one launch (greedy_small_kernel)" if not sampled and R <= 512 and N <= 256
-            else "persistent row kernel + tree walk")
+            else "cluster row kernel + tree walk")
     es = 4 if w.dtype == "f32" else 2
     return {"workload": w.name, "B": B, "N": N, "V": V, "logits": w.dtype, "sampled": sampled, "path": path,
             "us_per_call_graph": graph_us, "us_per_call_eager": eager_us, "us_per_call_e2e": e2e_us,
@@ -697,10 +697,9 @@ def run_ours(args):
     row_avg_s = statistics.median(row_ms) / 1e3
     achieved = alg / row_avg_s / 1e9
     peak, peak_kind = _peaks()
-    # the library streams rows with the cluster-per-row kernel; the distinct-sibling rule takes the
-    # persistent row kernel
-    kname = "score_rows_kernel" if args.distinct else "cluster_rows_kernel"
-    khash = _kernel_source_hash(("dcd_rows.cu", "dcd_device.cuh", "dcd_internal.h") if args.distinct else ROW_KERNEL_FILES)
+    # the library streams rows with the cluster-per-row kernel (both sibling rules)
+    kname = "cluster_rows_kernel"
+    khash = _kernel_source_hash(ROW_KERNEL_FILES)
     # the profile covers the default workload (32 sequences, mixed, i.i.d. siblings) only
     traffic = _profiled_traffic(khash) if B == 32 and not args.greedy and not args.distinct else None
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
@@ -1227,7 +1226,7 @@ def run_small(args):
     alg = float(R * V * 2 * es)  # both logit rows of every node (q: only at children unless rejected)
     peak, peak_kind = _peaks()
     achieved = alg / (ms_per_step / 1e3) / 1e9
-    path = "one launch (greedy_small_kernel)" if not sampled and R <= 512 else "persistent row kernel + tree walk"
+    path = "one launch (greedy_small_kernel)" if not sampled and R <= 512 else "cluster row kernel + tree walk"
     if rank == 0:
         line = {
             "metric": METRIC + ", small call", "value": job_value(world, R, ms_per_step), "unit": "nodes/s",

@@ -168,7 +168,16 @@ struct CShared {
   float c, D;        // current residual max(0, pi - c q) / D
   float cJ;          // c of the next pass
   int32_t degen;     // a pass found no residual mass: r = q from here on
-  int32_t pad[3];
+  // Distinct siblings: the proposal's mass Z (q's own, less the removed tokens' q), and the
+  // removed tokens with their frozen residual masses and pi and q at them (every CTA of a
+  // cluster keeps the same copy, written by its thread 0 from the same values)
+  float Z;
+  int32_t nrem;
+  int32_t pad;
+  int32_t rtok[kMaxRemoved];
+  float rfz[kMaxRemoved];
+  float rpit[kMaxRemoved];
+  float rq[kMaxRemoved];
 };
 
 struct Cmd {
@@ -334,7 +343,7 @@ __device__ __forceinline__ float cblock_key(const ScoreArgs& p, int64_t g, int k
   return race_key(log2_mass, word_of(w, k & 3));
 }
 
-template <typename TIn>
+template <typename TIn, bool kDistinct>
 __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(const __grid_constant__ CParams cp) {
   const ScoreArgs& p = cp.a;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -983,6 +992,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       }
       uint32_t status = sh->status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
       if (!(M > -INFINITY && M < INFINITY) || !(S > 0.f && S < INFINITY)) status |= DCD_DEVERR_NONFINITE;
+      if (kDistinct && sampled && m > kMaxRemoved) status |= DCD_DEVERR_UNSUPPORTED;
       const float logS = logf(S);
       const float invS = 1.f / S;
 
@@ -1066,6 +1076,8 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           sh->c = 0.f;
           sh->D = 1.f;
           sh->degen = 0;
+          sh->Z = 1.f;  // distinct siblings: nothing removed yet
+          sh->nrem = 0;
         }
         csync();
         if (sh->decision != 1) {
@@ -1075,8 +1087,12 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             const int J = sh->J;
             const float cJ = sh->cJ;
             const bool race = J == m;  // the pass after the last sibling also ranks race blocks
+            // distinct siblings: the first pass also sums q, whose actual mass (the drafter's q
+            // may be truncated or rounded away from 1) normalises the proposal once a token is
+            // removed
+            const bool sum_q = kDistinct && J == 1;
             ++npass;
-            float part = 0.f;
+            float part = 0.f, ql = 0.f;
             int L = 0;
             for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_r, ++seq, ++L) {
               const CStage<TIn> st =
@@ -1092,6 +1108,10 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
                   sp += (i0 + e < clen) ? fmaxf(ex2(u[e] - M) * invS - cJ * qv[e], 0.f) : 0.f;
+                if (sum_q) {
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) ql += (i0 + e < clen) ? qv[e] : 0.f;
+                }
               }
               part += sp;
               if (race) {
@@ -1101,6 +1121,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
               release(seq);
             }
             const float zsum = block_sum(part, redf, csync);  // its barriers also publish csum
+            const float qsum = sum_q ? block_sum(ql, redf, csync) : 0.f;
             float rk = -INFINITY;
             int rb = INT_MAX;
             if (race) {
@@ -1111,6 +1132,14 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
                 float mass = 0.f;
                 for (int i = 0; i < wpb_r && (kb - k_lo) * wpb_r + i < nch_sl; ++i)
                   mass += csum[(kb - k_lo) * wpb_r + i];
+                if (kDistinct) {
+                  // removed siblings' tokens in this block carry their frozen mass, not the
+                  // streamed one
+                  const int nrem = sh->nrem;
+                  for (int i = 0; i < nrem; ++i)
+                    if (sh->rtok[i] / kRaceBlock == kb)
+                      mass += sh->rfz[i] - fmaxf(sh->rpit[i] - cJ * sh->rq[i], 0.f);
+                }
                 if (mass > 0.f) {
                   const float key = cblock_key(p, g, kb, lg2(mass));
                   if (key > rk) {
@@ -1125,27 +1154,109 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             if (split) {
               XPart mine{};
               mine.a = zsum;
+              mine.b = qsum;
               mine.key = rk;
               mine.blk = rb;
               mine.status = timed_out ? DCD_DEVERR_TIMEOUT : 0u;
               all = exchange(mine);
             }
             if (tid == 0) {
-              float DJ = zsum, K = rk;
+              float DJ = zsum, K = rk, QS = qsum;
               int kstar = rb;
               uint32_t st2 = status | (timed_out ? DCD_DEVERR_TIMEOUT : 0u);
               if (split) {
                 DJ = 0.f;
+                QS = 0.f;
                 K = -INFINITY;
                 kstar = INT_MAX;
                 for (int t = 0; t < C; ++t) {  // a fixed order
                   DJ += all[t].a;
+                  QS += all[t].b;
                   argmax_merge(K, kstar, all[t].key, all[t].blk);
                   st2 |= all[t].status;
                 }
               }
               float c = sh->c, Dn = sh->D;
               bool degen = sh->degen != 0;
+              int acc = -1;
+              bool queued = false, ranked = J == m;
+              if constexpr (kDistinct) {
+                // Siblings without replacement.  With the tokens removed so far frozen at their
+                // mass fz, the residual after this pass is max(0, pi - c_J q) elsewhere: its
+                // mass is the streamed sum corrected at the removed tokens.  A pass without mass
+                // keeps the residual it started from.  Then sibling J's token is removed from
+                // the proposal (frozen at the current residual) and the next siblings are tested
+                // against r with the proposal q / Z without the removed tokens.
+                int nrem = sh->nrem;
+                float Z = J == 1 ? QS : sh->Z;  // q's own mass before the first removal
+                auto value_at = [&](int j, float& pit, float& qt) {  // at sibling j's (valid) token
+                  const bool in = !masked || (czp[j] - Mp >= logb);
+                  pit = in ? ex2(fmaf(c1k, czp[j], -ak * czq[j]) - M) * invS : 0.f;
+                  qt = cq[j];
+                };
+                auto removed_index = [&](int t) {
+                  for (int i = 0; i < nrem; ++i)
+                    if (sh->rtok[i] == t) return i;
+                  return -1;
+                };
+                float EJ = DJ;
+                for (int i = 0; i < nrem; ++i) EJ += sh->rfz[i] - fmaxf(sh->rpit[i] - cJ * sh->rq[i], 0.f);
+                if (EJ > 0.f) {
+                  c = cJ;
+                  Dn = EJ;
+                } else {
+                  ranked = false;  // the pass ranked blocks of a residual that is not used
+                }
+                auto remove = [&](int j) {  // sibling j's token
+                  const int t = ktok[j];
+                  if (t < 0 || t >= V || removed_index(t) >= 0) return;
+                  if (nrem >= kMaxRemoved) {
+                    st2 |= DCD_DEVERR_UNSUPPORTED;
+                    return;
+                  }
+                  float pit, qt;
+                  value_at(j, pit, qt);
+                  sh->rtok[nrem] = t;
+                  sh->rfz[nrem] = fmaxf(pit - c * qt, 0.f);
+                  sh->rpit[nrem] = pit;
+                  sh->rq[nrem] = qt;
+                  ++nrem;
+                  Z -= qt;
+                };
+                remove(J - 1);
+                for (int j = J; j < m; ++j) {
+                  const int t = ktok[j];
+                  float ratio = 0.f;
+                  if (t >= 0 && t < V) {
+                    const int ri = removed_index(t);
+                    if (ri >= 0) {
+                      ratio = sh->rfz[ri] > 0.f ? INFINITY : 0.f;  // its proposal is 0
+                    } else {
+                      float pit, qt;
+                      value_at(j, pit, qt);
+                      const float rho = fmaxf(pit - c * qt, 0.f);
+                      const float qp = Z > 0.f ? qt / Z : 0.f;
+                      ratio = qp > 0.f ? (rho / Dn) / qp : (rho > 0.f ? INFINITY : 0.f);
+                    }
+                  }
+                  const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[j]);
+                  if (u01(philox_block(p.seed, p.offset, G, 0u).x) <= ratio) {
+                    acc = kids[j];
+                    break;
+                  }
+                  if (Z > 0.f) {
+                    sh->J = j + 1;
+                    sh->cJ = c + Dn / Z;  // the next residual: max(0, r - q / Z) off the removed tokens
+                    queued = true;
+                    break;
+                  }
+                  // every token of q is removed: the proposal is 0 and the residual stays
+                  ranked = false;
+                  remove(j);
+                }
+                sh->nrem = nrem;
+                sh->Z = Z;
+              } else {
               if (DJ > 0.f) {
                 c = cJ;
                 Dn = DJ;
@@ -1153,16 +1264,14 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
                 degen = true;  // r_{J-1} == q in exact arithmetic: r_J is taken as q from here on
               }
               // test the remaining siblings; after a pass without residual mass no pass is needed
-              int acc = -1;
-              bool queued = false;
               for (int j = J; j < m; ++j) {
+                // the values at the children's tokens were loaded into shared memory with the row
                 const int t = ktok[j];
                 const bool ok = t >= 0 && t < V;
-                const float z = ok ? ld1(zp_row, t) : 0.f;
-                const float zz = ok ? ld1(zq_row, t) : 0.f;
-                const float qt = ok ? q_row[t] : 0.f;
+                const float z = czp[j];
+                const float qt = cq[j];
                 const bool in = ok && (!masked || (z - Mp >= logb));
-                const float pit = in ? ex2(fmaf(c1k, z, -ak * zz) - M) * invS : 0.f;
+                const float pit = in ? ex2(fmaf(c1k, z, -ak * czq[j]) - M) * invS : 0.f;
                 const float rt = degen ? qt : fmaxf(pit - c * qt, 0.f) / Dn;
                 const float ratio = qt > 0.f ? rt / qt : (rt > 0.f ? INFINITY : 0.f);
                 const uint32_t G = static_cast<uint32_t>(static_cast<int64_t>(b) * N + kids[j]);
@@ -1177,11 +1286,12 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
                   break;
                 }
               }
+              }
               sh->c = c;
               sh->D = Dn;
               sh->degen = degen ? 1 : 0;
               sh->status = st2;
-              sh->term = (J == m && !degen) ? kstar : INT_MAX - 1;
+              sh->term = (ranked && !degen) ? kstar : INT_MAX - 1;  // the winning block when this pass ranked r_m
               sh->decision = queued ? 2 : (acc >= 0 ? 1 : 0);
               if (queued) {
                 post(1, sh->J < m ? 1 : 0);
@@ -1199,9 +1309,21 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             const bool degen = sh->degen != 0;
             const float c = sh->c, Dn = sh->D;
             const uint32_t st2 = sh->status;
+            const int nrem = kDistinct ? sh->nrem : 0;
             int kstar = sh->term;
-            if (degen) {
-              // block masses of q over the slices (rare: a residual without mass)
+            auto rho_at = [&](int64_t x) -> float {  // the final residual's unnormalised mass
+              if (kDistinct)
+                for (int i = 0; i < nrem; ++i)
+                  if (sh->rtok[i] == x) return sh->rfz[i];
+              const float z = ld1(zp_row, x);
+              const bool in = !masked || (z - Mp >= logb);
+              const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
+              return fmaxf(pit - c * q_row[x], 0.f);
+            };
+            if (kstar == INT_MAX - 1) {
+              // block masses over the slices of q (a residual without mass), or (distinct
+              // siblings) of the final residual when the last pass did not rank it (rare: the
+              // last pass found no mass, or q was used up)
               float qk = -INFINITY;
               int qb = INT_MAX;
               const int k_lo = static_cast<int>(x_lo / kRaceBlock);
@@ -1210,7 +1332,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
                 float s2 = 0.f;
                 for (int64_t x = static_cast<int64_t>(kb) * kRaceBlock + lane; x < x_hi && x < (kb + 1) * kRaceBlock;
                      x += 32)
-                  s2 += q_row[x];
+                  s2 += kDistinct ? rho_at(x) : q_row[x];
                 const float mass = warp_sum(s2);
                 if (lane == 0 && mass > 0.f) {
                   const float key = cblock_key(p, g, kb, lg2(mass));
@@ -1236,11 +1358,8 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
               const int term = ctoken_race(
                   p, g, kstar,
                   [&](int64_t x) -> float {
-                    if (degen) return q_row[x];
-                    const float z = ld1(zp_row, x);
-                    const bool in = !masked || (z - Mp >= logb);
-                    const float pit = in ? ex2(fmaf(c1k, z, -ak * ld1(zq_row, x)) - M) * invS : 0.f;
-                    return fmaxf(pit - c * q_row[x], 0.f) / Dn;
+                    if (degen && !kDistinct) return q_row[x];
+                    return rho_at(x) / Dn;
                   },
                   redf, redi);
               if (tid == 0) write_record(-1, term, st2);
@@ -1265,7 +1384,7 @@ struct CDeviceInfo {
   cudaError_t err = cudaSuccess;
 };
 
-template <typename TIn>
+template <typename TIn, bool kDistinct>
 cudaError_t prepare_cluster_kernel(int* sms) {
   static std::once_flag once[64];
   static CDeviceInfo info[64];
@@ -1275,7 +1394,7 @@ cudaError_t prepare_cluster_kernel(int* sms) {
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   std::call_once(once[dev], [&] {
     CDeviceInfo d;
-    d.err = cudaFuncSetAttribute(cluster_rows_kernel<TIn>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    d.err = cudaFuncSetAttribute(cluster_rows_kernel<TIn, kDistinct>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     if (d.err == cudaSuccess) d.err = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
     info[dev] = d;
   });
@@ -1351,9 +1470,9 @@ bool cluster_geometry(const ScoreArgs& a, int sms, CParams* cp, size_t* smem) {
 }
 
 // Resident clusters of the kernel for a launch shape, cached (the occupancy query is not free).
-cudaError_t resident_clusters(const void* fn, const cudaLaunchConfig_t& cfg, int dtype, int C, size_t smem, int* ncl) {
+cudaError_t resident_clusters(const void* fn, const cudaLaunchConfig_t& cfg, int variant, int C, size_t smem, int* ncl) {
   struct Entry {
-    int dev, dtype, C;
+    int dev, variant, C;  // variant: element type and sibling rule
     size_t smem;
     int ncl;
   };
@@ -1366,7 +1485,7 @@ cudaError_t resident_clusters(const void* fn, const cudaLaunchConfig_t& cfg, int
   {
     std::lock_guard<std::mutex> lk(mu);
     for (int i = 0; i < n; ++i)
-      if (cache[i].dev == dev && cache[i].dtype == dtype && cache[i].C == C && cache[i].smem == smem) {
+      if (cache[i].dev == dev && cache[i].variant == variant && cache[i].C == C && cache[i].smem == smem) {
         *ncl = cache[i].ncl;
         return cudaSuccess;
       }
@@ -1374,14 +1493,14 @@ cudaError_t resident_clusters(const void* fn, const cudaLaunchConfig_t& cfg, int
   e = cudaOccupancyMaxActiveClusters(ncl, fn, &cfg);
   if (e != cudaSuccess) return e;
   std::lock_guard<std::mutex> lk(mu);
-  if (n < 64) cache[n++] = Entry{dev, dtype, C, smem, *ncl};
+  if (n < 64) cache[n++] = Entry{dev, variant, C, smem, *ncl};
   return cudaSuccess;
 }
 
 }  // namespace
 
 bool cluster_rows_ok(const ScoreArgs& a) {
-  if (a.distinct || a.force_stages || a.force_plain || a.poll_cycles) return false;
+  if (a.force_stages || a.force_plain || a.poll_cycles) return false;
   const int es = a.dtype == DCD_BF16 ? 2 : 4;
   auto al16 = [](const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; };
   if (!al16(a.zp) || !al16(a.zq) || (a.ld * es) % 16 != 0) return false;
@@ -1395,7 +1514,10 @@ cudaError_t launch_cluster_rows(const ScoreArgs& a, cudaStream_t stream) {
   const int64_t R = static_cast<int64_t>(a.B) * a.N;
   if (R == 0) return cudaSuccess;
   int sms = 0;
-  cudaError_t e = a.dtype == DCD_BF16 ? prepare_cluster_kernel<__nv_bfloat16>(&sms) : prepare_cluster_kernel<float>(&sms);
+  const bool bf = a.dtype == DCD_BF16;
+  cudaError_t e = bf ? (a.distinct ? prepare_cluster_kernel<__nv_bfloat16, true>(&sms)
+                                   : prepare_cluster_kernel<__nv_bfloat16, false>(&sms))
+                     : (a.distinct ? prepare_cluster_kernel<float, true>(&sms) : prepare_cluster_kernel<float, false>(&sms));
   if (e != cudaSuccess) return e;
   CParams cp;
   size_t smem = 0;
@@ -1411,14 +1533,16 @@ cudaError_t launch_cluster_rows(const ScoreArgs& a, cudaStream_t stream) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const void* fn = a.dtype == DCD_BF16 ? reinterpret_cast<const void*>(cluster_rows_kernel<__nv_bfloat16>)
-                                       : reinterpret_cast<const void*>(cluster_rows_kernel<float>);
+  const void* fn = bf ? (a.distinct ? reinterpret_cast<const void*>(cluster_rows_kernel<__nv_bfloat16, true>)
+                                    : reinterpret_cast<const void*>(cluster_rows_kernel<__nv_bfloat16, false>))
+                      : (a.distinct ? reinterpret_cast<const void*>(cluster_rows_kernel<float, true>)
+                                    : reinterpret_cast<const void*>(cluster_rows_kernel<float, false>));
   // a persistent grid: as many clusters as can be resident at once (each claims rows until none
   // is left; no CTA waits for another cluster, so fewer resident clusters only take longer); the
-  // count is queried once per device, element type, cluster size and shared-memory size
+  // count is queried once per device, kernel variant, cluster size and shared-memory size
   cfg.gridDim = dim3(static_cast<unsigned>(cp.C));
   int ncl = 0;
-  e = resident_clusters(fn, cfg, a.dtype, cp.C, smem, &ncl);
+  e = resident_clusters(fn, cfg, a.dtype * 2 + (a.distinct ? 1 : 0), cp.C, smem, &ncl);
   if (e != cudaSuccess) return e;
   if (ncl < 1) return cudaErrorInvalidConfiguration;
   if (ncl > R) ncl = static_cast<int>(R);
@@ -1426,8 +1550,11 @@ cudaError_t launch_cluster_rows(const ScoreArgs& a, cudaStream_t stream) {
   // the error word, the row counters and the half-row tickets start every call at zero
   e = cudaMemsetAsync(a.hdr, 0, kWorkspaceHeader + part_counter_bytes(static_cast<size_t>(R)), stream);
   if (e != cudaSuccess) return e;
-  if (a.dtype == DCD_BF16) return cudaLaunchKernelEx(&cfg, cluster_rows_kernel<__nv_bfloat16>, cp);
-  return cudaLaunchKernelEx(&cfg, cluster_rows_kernel<float>, cp);
+  if (bf)
+    return a.distinct ? cudaLaunchKernelEx(&cfg, cluster_rows_kernel<__nv_bfloat16, true>, cp)
+                      : cudaLaunchKernelEx(&cfg, cluster_rows_kernel<__nv_bfloat16, false>, cp);
+  return a.distinct ? cudaLaunchKernelEx(&cfg, cluster_rows_kernel<float, true>, cp)
+                    : cudaLaunchKernelEx(&cfg, cluster_rows_kernel<float, false>, cp);
 }
 
 }  // namespace dcd

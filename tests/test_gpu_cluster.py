@@ -65,3 +65,39 @@ def test_more_than_1024_sequences_rows_whole():
     g = run_gpu(w, sampled=True, residual=True)
     compare(w, g, _oracle(w, residual=True), check_residual=True, max_amb_frac=0.05)
     assert int((w.temperature > 0).sum()) == 550
+
+
+def _oracle_distinct(w):
+    return oracle.verify_workload(w, nthreads=oracle.max_threads(), want_residual=True, distinct=True)
+
+
+@pytest.mark.parametrize("dtype,V,beta", [("bf16", 40000, 0.0), ("bf16", 40000, 0.5), ("f32", 34176, 0.1)])
+def test_distinct_siblings_on_split_rows(dtype, V, beta):
+    # siblings drawn without replacement on rows split over clusters of 4 CTAs (bf16) and 8 CTAs
+    # with three empty slices (fp32): q's own mass is summed over the slices in the first pass,
+    # and the removed tokens' frozen masses correct the exchanged pass sums and the owning CTA's
+    # race blocks; nodes of up to 10 children make long chains of removals
+    w = workloads.generate(name="split_distinct", B=4, V=V, dtype=dtype, spikes=(1, 6), alphas=(0.1, 0.5),
+                           beta=beta, temperatures=(1.0, 0.7), levels=(1, 10, 12, 8), max_children=10,
+                           seed=90 + int(beta * 10) + V % 7, margin_fn=oracle.margin_fn)
+    g = run_gpu(w, sampled=True, residual=True, distinct=True)
+    compare(w, g, _oracle_distinct(w), check_residual=True)
+
+
+def test_distinct_duplicates_and_zero_draft_probability_on_split_rows():
+    # a duplicated sibling token (its proposal is 0 once the first copy is removed) and a sibling
+    # token of zero draft probability, on rows split over clusters of 4 CTAs
+    w = workloads.generate(name="split_dup", B=3, V=40000, dtype="bf16", spikes=(1, 6), alphas=(0.2,),
+                           temperatures=(1.0,), levels=(1, 6, 9, 6), seed=97, margin_fn=oracle.margin_fn)
+    tok = w.tokens.clone()
+    q = w.q.clone()
+    for b in range(w.B):
+        kids = workloads.children_lists(w.parents[b].numpy())
+        for n, ch in enumerate(kids):
+            if len(ch) >= 2:
+                tok[b, ch[1]] = tok[b, ch[0]]
+            if len(ch) >= 3:
+                q[b * w.N + n, int(tok[b, ch[2]])] = 0.0
+    w.tokens, w.q = tok, q
+    g = run_gpu(w, sampled=True, residual=True, distinct=True)
+    compare(w, g, _oracle_distinct(w), check_residual=True)
