@@ -33,6 +33,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <cfloat>
 #include <climits>
 #include <mutex>
 
@@ -80,6 +81,10 @@ constexpr int kSeqListMax = 1024;
 // rejection there starts a chain of at most kHoldMax passes, which the row claimed ahead waits
 // out); after a wider node it claims once the first sibling is decided or the chain settled.
 constexpr int kHoldMax = DCD_CLUSTER_HOLD_MAX;
+#ifndef DCD_CLUSTER_SUSPEND_NS
+#define DCD_CLUSTER_SUSPEND_NS 20000
+#endif
+constexpr uint32_t kSuspendNs = DCD_CLUSTER_SUSPEND_NS;  // try_wait suspend-time hint, 0: none
 #ifndef DCD_CLUSTER_HALF_ROWS
 #define DCD_CLUSTER_HALF_ROWS -1
 #endif
@@ -237,13 +242,22 @@ __device__ __forceinline__ void arrive_cluster(uint32_t bar_addr) {
 
 __device__ __forceinline__ bool try_wait_cluster(uint64_t* bar, uint32_t parity) {
   uint32_t done;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.b32 %0, 1, 0, p;\n\t}"
-      : "=r"(done)
-      : "r"(smem_addr(bar)), "r"(parity)
-      : "memory");
+  if (kSuspendNs == 0)
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.b32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+  else
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.b32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
+        : "memory");
   return done != 0;
 }
 
@@ -252,6 +266,26 @@ __device__ __forceinline__ bool wait_cluster_bounded(uint64_t* bar, uint32_t par
   while (!try_wait_cluster(bar, parity))
     if (clock64() - t0 > kWaitCycles) return false;
   return true;
+}
+
+// A CTA-scope wait whose try_wait may suspend the thread for up to kSuspendNs (it resumes when
+// the phase completes), so that a waiting warp does not take issue slots from the computing ones;
+// bounded like mbar_wait_bounded.
+__device__ __forceinline__ bool cwait_bounded(uint64_t* bar, uint32_t parity) {
+  if (kSuspendNs == 0) return mbar_wait_bounded(bar, parity);
+  const long long t0 = clock64();
+  for (;;) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.b32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
+        : "memory");
+    if (done) return true;
+    if (clock64() - t0 > kWaitCycles) return false;
+  }
 }
 
 // Lists the children of node n (ascending id) with the calling warp; returns their count.
@@ -451,7 +485,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
         const uint32_t phase = ((issued / static_cast<uint32_t>(cp.nst)) & 1u) ^ 1u;
         const int clen = static_cast<int>((hi - x0) < tok ? (hi - x0) : tok);
         const CStage<TIn> st = cstage<TIn>(ring, s, tok);
-        if (!mbar_wait_bounded(&empty[s], phase)) {
+        if (!cwait_bounded(&empty[s], phase)) {
           atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
           CL_SITE(0);
         }
@@ -499,7 +533,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     };
     auto hand = [&](const Meta& mt) {  // lane 0: the next row descriptor for the consumers
       const int d = static_cast<int>(kd % kCDesc);
-      if (!mbar_wait_bounded(&dempty[d], ((kd / kCDesc) & 1u) ^ 1u)) {
+      if (!cwait_bounded(&dempty[d], ((kd / kCDesc) & 1u) ^ 1u)) {
         atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
         CL_SITE(3);
       }
@@ -575,7 +609,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           }
         });
         for (; has_child; ++ncmd) {
-          if (!mbar_wait_bounded(cmdbar, ncmd & 1u)) {
+          if (!cwait_bounded(cmdbar, ncmd & 1u)) {
             atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
             CL_SITE(4);
             stop = true;
@@ -659,7 +693,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
         if (masked) stream(g, 0, V, cp.tok_a, 0, pol_last, nop);
         stream(g, lo, hi, cp.tok_a, 1, sampled && has_child ? pol_normal : pol_first, nop);
         for (; sampled && has_child; ++ncmd) {
-          if (!mbar_wait_bounded(cmdbar, ncmd & 1u)) {
+          if (!cwait_bounded(cmdbar, ncmd & 1u)) {
             atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
             CL_SITE(4);
             stop = true;
@@ -693,7 +727,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
   (void)w_desc;
   auto wait_full = [&](uint32_t sq) {
     CL_T(tw);
-    if (!mbar_wait_bounded(&full[sq % static_cast<uint32_t>(cp.nst)], (sq / static_cast<uint32_t>(cp.nst)) & 1u)) {
+    if (!cwait_bounded(&full[sq % static_cast<uint32_t>(cp.nst)], (sq / static_cast<uint32_t>(cp.nst)) & 1u)) {
       timed_out = true;
       CL_SITE(5);
     }
@@ -738,7 +772,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
   for (uint32_t k = 0;; ++k) {
     const int dd = static_cast<int>(k % kCDesc);
     CL_T(td);
-    const bool dok = mbar_wait_bounded(&dfull[dd], (k / kCDesc) & 1u);
+    const bool dok = cwait_bounded(&dfull[dd], (k / kCDesc) & 1u);
     CL_ACC(w_desc, td);
     if (!dok) {
       if (tid == 0) atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
@@ -843,52 +877,76 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       // 2^(u - max) rescaled when the max grows, and the argmax; a sampled leaf also records the
       // mass of each warp chunk relative to a chunk reference
       const int tpw = cp.tok_a / kCWarps, wpb = kRaceBlock / tpw;
-      float lmax = -INFINITY, lsum = 0.f;
+      // the running max starts finite (no score is that low), so that 2^(u - max) needs no test
+      // for an empty max; it is -inf again below if no score was finite
+      float lmax = -FLT_MAX, lsum = 0.f;
       int larg = INT_MAX;
       const bool rec_chunks = sampled && !has_child;  // a sampled leaf's race needs the chunk masses
+      const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
       for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_a, ++seq) {
         const CStage<TIn> st = cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(cp.nst)), cp.tok_a);
         const int clen = static_cast<int>((x_hi - x0) < cp.tok_a ? (x_hi - x0) : cp.tok_a);
+        const int sb_end = (warp + 1) * tpw < clen ? (warp + 1) * tpw : clen;
         wait_full(seq);
-        float bpart = 0.f;
-        for (int sb = warp * tpw; sb < (warp + 1) * tpw && sb < clen; sb += kSub) {  // warp-uniform
-          const int i0 = sb + lane * 8;
-          float u[8];
-          cscores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
+        float2 acc2 = make_float2(0.f, 0.f);  // this stage's sum of 2^(u - lmax), in lane pairs
+        // a stage-wide step: the max, the rescale when it grows (with the argmax), the sum
+        auto step = [&](const float (&u)[8], int i0) {
           const float gm = max8(u);
           if (gm > lmax) {
-            const float f = ex2(lmax - gm);  // 0 while lmax is -inf
+            const float f = ex2(lmax - gm);  // 0 while lmax is the start value
             lsum *= f;
-            bpart *= f;
+            acc2 = __fmul2_rn(acc2, make_float2(f, f));
             lmax = gm;
 #pragma unroll
             for (int e = 7; e >= 0; --e)
               if (u[e] == gm) larg = static_cast<int>(x0) + i0 + e;
           }
-          if (lmax > -INFINITY) {
-            const float2 nm2 = make_float2(-lmax, -lmax);
-            float2 acc2 = make_float2(0.f, 0.f);
+          const float2 nm2 = make_float2(-lmax, -lmax);
+          float2 e2[4];
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const float2 d2 = __fadd2_rn(make_float2(u[2 * kk], u[2 * kk + 1]), nm2);
-              acc2 = __fadd2_rn(acc2, make_float2(ex2(d2.x), ex2(d2.y)));
+          for (int kk = 0; kk < 4; ++kk) {
+            const float2 d2 = __fadd2_rn(make_float2(u[2 * kk], u[2 * kk + 1]), nm2);
+            e2[kk] = make_float2(ex2(d2.x), ex2(d2.y));
+          }
+          acc2 = __fadd2_rn(acc2, __fadd2_rn(__fadd2_rn(e2[0], e2[1]), __fadd2_rn(e2[2], e2[3])));
+        };
+        int sb = warp * tpw;
+        if (!masked) {
+          for (; sb + kSub <= sb_end; sb += kSub) {  // whole sub-blocks (warp-uniform)
+            const int i0 = sb + lane * 8;
+            float2 zp2[4], zq2[4];
+            ld8x2(st.zp + i0, zp2);
+            ld8x2(st.zq + i0, zq2);
+            float u[8];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float2 s2 = __ffma2_rn(zp2[k], c1k2, __fmul2_rn(zq2[k], nak2));
+              u[2 * k] = s2.x;
+              u[2 * k + 1] = s2.y;
             }
-            const float a = acc2.x + acc2.y;
-            lsum += a;
-            bpart += a;
+            step(u, i0);
           }
         }
+        for (; sb < sb_end; sb += kSub) {  // the plausibility mask, or the stage's ragged end
+          const int i0 = sb + lane * 8;
+          float u[8];
+          cscores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
+          step(u, i0);
+        }
+        const float bpart = acc2.x + acc2.y;
+        lsum += bpart;
         if (rec_chunks) {
           const float ref = warp_max(lmax);
-          const float ws = warp_sum(lmax > -INFINITY ? bpart * ex2(lmax - ref) : 0.f);
+          const float ws = warp_sum(bpart * ex2(lmax - ref));
           if (lane == 0 && x0 + static_cast<int64_t>(warp) * tpw < x_hi) {
             const int ch = static_cast<int>((x0 - x_lo) / tpw) + warp;
-            cref[ch] = ref;
+            cref[ch] = ref > -FLT_MAX ? ref : -INFINITY;
             csum[ch] = ws;
           }
         }
         release(seq);
       }
+      if (lmax == -FLT_MAX) lmax = -INFINITY;  // no finite score
       float M = lmax, S = lsum;
       int arg = larg;
       block_stats(M, S, arg, redf, redi, csync);  // its barriers also publish warp 1's child list
@@ -1094,25 +1152,59 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             ++npass;
             float part = 0.f, ql = 0.f;
             int L = 0;
+            // r(x) S = max(2^(u - M) - c_J S q(x), 0): the factor 1 / S is applied to the sums
+            const float2 nM2 = make_float2(-M, -M), ncs2 = make_float2(-cJ * S, -cJ * S);
+            const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
             for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_r, ++seq, ++L) {
               const CStage<TIn> st =
                   cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(cp.nst)), cp.tok_r);
               const int clen = static_cast<int>((x_hi - x0) < cp.tok_r ? (x_hi - x0) : cp.tok_r);
+              const int sb_end = (warp + 1) * tpw_r < clen ? (warp + 1) * tpw_r : clen;
               wait_full(seq);
-              float sp = 0.f;
-              for (int sb = warp * tpw_r; sb < (warp + 1) * tpw_r && sb < clen; sb += kSub) {  // warp-uniform
-                const int i0 = sb + lane * 8;
-                float u[8], qv[8];
-                cscores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);
-                ld8(st.q + i0, qv);
+              float2 sp2 = make_float2(0.f, 0.f), ql2 = make_float2(0.f, 0.f);
+              auto rstep = [&](const float (&u)[8], const float2 (&q2)[4]) {
+                float2 t2[4];
 #pragma unroll
-                for (int e = 0; e < 8; ++e)
-                  sp += (i0 + e < clen) ? fmaxf(ex2(u[e] - M) * invS - cJ * qv[e], 0.f) : 0.f;
-                if (sum_q) {
+                for (int k = 0; k < 4; ++k) {
+                  const float2 d2 = __fadd2_rn(make_float2(u[2 * k], u[2 * k + 1]), nM2);
+                  const float2 r2 = __ffma2_rn(q2[k], ncs2, make_float2(ex2(d2.x), ex2(d2.y)));
+                  t2[k] = make_float2(fmaxf(r2.x, 0.f), fmaxf(r2.y, 0.f));
+                }
+                sp2 = __fadd2_rn(sp2, __fadd2_rn(__fadd2_rn(t2[0], t2[1]), __fadd2_rn(t2[2], t2[3])));
+                if (sum_q) ql2 = __fadd2_rn(ql2, __fadd2_rn(__fadd2_rn(q2[0], q2[1]), __fadd2_rn(q2[2], q2[3])));
+              };
+              int sb = warp * tpw_r;
+              if (!masked) {
+                for (; sb + kSub <= sb_end; sb += kSub) {  // whole sub-blocks (warp-uniform)
+                  const int i0 = sb + lane * 8;
+                  float2 zp2[4], zq2[4];
+                  ld8x2(st.zp + i0, zp2);
+                  ld8x2(st.zq + i0, zq2);
+                  float u[8];
 #pragma unroll
-                  for (int e = 0; e < 8; ++e) ql += (i0 + e < clen) ? qv[e] : 0.f;
+                  for (int k = 0; k < 4; ++k) {
+                    const float2 s2 = __ffma2_rn(zp2[k], c1k2, __fmul2_rn(zq2[k], nak2));
+                    u[2 * k] = s2.x;
+                    u[2 * k + 1] = s2.y;
+                  }
+                  float2 q2[4];
+                  ld8x2(st.q + i0, q2);
+                  rstep(u, q2);
                 }
               }
+              for (; sb < sb_end; sb += kSub) {  // the plausibility mask, or the stage's ragged end
+                const int i0 = sb + lane * 8;
+                float u[8], qv[8];
+                cscores8(st.zp, st.zq, i0, sb, clen, masked, c1k, ak, Mp, logb, u);  // -inf past the end
+                ld8(st.q + i0, qv);
+                float2 q2[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k)  // q past the end is whatever the stage held before
+                  q2[k] = make_float2(i0 + 2 * k < clen ? qv[2 * k] : 0.f, i0 + 2 * k + 1 < clen ? qv[2 * k + 1] : 0.f);
+                rstep(u, q2);
+              }
+              const float sp = (sp2.x + sp2.y) * invS;
+              ql += ql2.x + ql2.y;
               part += sp;
               if (race) {
                 const float ws = warp_sum(sp);
