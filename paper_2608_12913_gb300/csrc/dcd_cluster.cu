@@ -157,7 +157,6 @@ struct CParams {
   int32_t C;             // CTAs per cluster: slices per row
   int32_t tok_a, tok_r;  // tokens per stage: statistics (z_p, z_q) and residual passes (z_p, z_q, q)
   int32_t spc;           // statistics stages per slice
-  int32_t nst;           // ring depth
   int32_t nchunk;        // chunk-mass slots
   int32_t meta_offset, chunk_offset, stage_offset;
   int32_t seq_offset;    // shared-memory offset of the sequence list (sampled first), 0: none
@@ -421,7 +420,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
   unsigned char* ring = smem + cp.stage_offset;
 
   if (tid == 0) {
-    for (int s = 0; s < cp.nst; ++s) {
+    for (int s = 0; s < kCRing; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kCWarps);
     }
@@ -481,8 +480,8 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       const TIn* zq_row = static_cast<const TIn*>(p.zq) + static_cast<int64_t>(g) * p.ld;
       const float* q_row = kind == 2 ? p.q + static_cast<int64_t>(g) * p.ldq : nullptr;
       for (int64_t x0 = lo; x0 < hi; x0 += tok, ++issued) {
-        const int s = static_cast<int>(issued % static_cast<uint32_t>(cp.nst));
-        const uint32_t phase = ((issued / static_cast<uint32_t>(cp.nst)) & 1u) ^ 1u;
+        const int s = static_cast<int>(issued % static_cast<uint32_t>(kCRing));
+        const uint32_t phase = ((issued / static_cast<uint32_t>(kCRing)) & 1u) ^ 1u;
         const int clen = static_cast<int>((hi - x0) < tok ? (hi - x0) : tok);
         const CStage<TIn> st = cstage<TIn>(ring, s, tok);
         if (!cwait_bounded(&empty[s], phase)) {
@@ -727,7 +726,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
   (void)w_desc;
   auto wait_full = [&](uint32_t sq) {
     CL_T(tw);
-    if (!cwait_bounded(&full[sq % static_cast<uint32_t>(cp.nst)], (sq / static_cast<uint32_t>(cp.nst)) & 1u)) {
+    if (!cwait_bounded(&full[sq % static_cast<uint32_t>(kCRing)], (sq / static_cast<uint32_t>(kCRing)) & 1u)) {
       timed_out = true;
       CL_SITE(5);
     }
@@ -735,7 +734,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
   };
   auto release = [&](uint32_t sq) {
     __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[sq % static_cast<uint32_t>(cp.nst)]);
+    if (lane == 0) mbar_arrive(&empty[sq % static_cast<uint32_t>(kCRing)]);
   };
   // Exchange: thread 0 pushes this CTA's share into slot `rank` of buffer xk & 1 in every CTA of
   // the cluster and arrives there; every consumer thread then waits until its own buffer holds
@@ -849,7 +848,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       if (masked) {
         float lm = -INFINITY;
         for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_a, ++seq) {
-          const CStage<TIn> st = cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(cp.nst)), cp.tok_a);
+          const CStage<TIn> st = cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(kCRing)), cp.tok_a);
           const int clen = static_cast<int>((x_hi - x0) < cp.tok_a ? (x_hi - x0) : cp.tok_a);
           wait_full(seq);
           for (int i0 = tid * 8; i0 < clen; i0 += kCThreads * 8) {
@@ -883,8 +882,9 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       int larg = INT_MAX;
       const bool rec_chunks = sampled && !has_child;  // a sampled leaf's race needs the chunk masses
       const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
-      for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_a, ++seq) {
-        const CStage<TIn> st = cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(cp.nst)), cp.tok_a);
+      int L = 0;  // stage of the slice
+      for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_a, ++seq, ++L) {
+        const CStage<TIn> st = cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(kCRing)), cp.tok_a);
         const int clen = static_cast<int>((x_hi - x0) < cp.tok_a ? (x_hi - x0) : cp.tok_a);
         const int sb_end = (warp + 1) * tpw < clen ? (warp + 1) * tpw : clen;
         wait_full(seq);
@@ -939,7 +939,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           const float ref = warp_max(lmax);
           const float ws = warp_sum(bpart * ex2(lmax - ref));
           if (lane == 0 && x0 + static_cast<int64_t>(warp) * tpw < x_hi) {
-            const int ch = static_cast<int>((x0 - x_lo) / tpw) + warp;
+            const int ch = L * kCWarps + warp;  // (x0 - x_lo) / tpw + warp
             cref[ch] = ref > -FLT_MAX ? ref : -INFINITY;
             csum[ch] = ws;
           }
@@ -1157,7 +1157,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
             const float2 c1k2 = make_float2(c1k, c1k), nak2 = make_float2(-ak, -ak);
             for (int64_t x0 = x_lo; x0 < x_hi; x0 += cp.tok_r, ++seq, ++L) {
               const CStage<TIn> st =
-                  cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(cp.nst)), cp.tok_r);
+                  cstage<TIn>(ring, static_cast<int>(seq % static_cast<uint32_t>(kCRing)), cp.tok_r);
               const int clen = static_cast<int>((x_hi - x0) < cp.tok_r ? (x_hi - x0) : cp.tok_r);
               const int sb_end = (warp + 1) * tpw_r < clen ? (warp + 1) * tpw_r : clen;
               wait_full(seq);
@@ -1551,7 +1551,6 @@ bool cluster_geometry(const ScoreArgs& a, int sms, CParams* cp, size_t* smem) {
   cp->tok_a = tok_a;
   cp->tok_r = tok_r;
   cp->spc = spc;
-  cp->nst = kCRing;
   cp->nchunk = static_cast<int32_t>(nchunk);
   cp->meta_offset = l.meta_offset;
   cp->chunk_offset = l.chunk_offset;
