@@ -565,20 +565,26 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
         arrive_cluster(map_rank(&mfull[d], static_cast<uint32_t>(t)));
       }
     };
-    if (rank == 0 && lane == 0) {
-      next_i = static_cast<int>(atomicAdd(&p.hdr->work, 1u));
-      g_next = next_i < nA ? row1(next_i) : -1;
-      send(0u, g_next);
+    // the first row of cluster c is claim index c, which every CTA of the cluster computes itself;
+    // later claims come from the counter, after the ncl static ones.  Message j carries the row of
+    // iteration j + 1.
+    const int ncl = static_cast<int>(gridDim.x) / C;
+    auto claim = [&]() { return ncl + static_cast<int>(atomicAdd(&p.hdr->work, 1u)); };
+    {
+      const int i0 = static_cast<int>(blockIdx.x) / C;
+      next_i = i0;
+      g_next = i0 < nA ? row1(i0) : -1;
     }
     bool stop = false;
     for (uint32_t k = 0; !stop; ++k) {
       int g = -1;
       if (lane == 0) {
-        if (rank == 0) {
+        if (rank == 0 || k == 0) {
           g = g_next;
         } else {
-          const int d = static_cast<int>(k % kMail);
-          if (!wait_cluster_bounded(&mfull[d], (k / kMail) & 1u)) {
+          const uint32_t j = k - 1u;  // message index
+          const int d = static_cast<int>(j % kMail);
+          if (!wait_cluster_bounded(&mfull[d], (j / kMail) & 1u)) {
             atomicOr(&p.hdr->err, DCD_DEVERR_TIMEOUT);
             CL_SITE(2);
             g = -1;
@@ -596,14 +602,14 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
       const bool wide = (mt.flags & 8) != 0;       // more than kHoldMax children
       if (lane == 0) {
         bool sent = false;
-        if (rank == 0 && !wide) next_i = static_cast<int>(atomicAdd(&p.hdr->work, 1u));  // one row ahead
+        if (rank == 0 && !wide) next_i = claim();  // one row ahead
         hand(mt);
         if (masked) stream(g, sl_lo, sl_hi, cp.tok_a, 0, pol_last, nop);  // the statistics pass re-reads it
         // the slice of a node with a child stays in L2 for the residual pass that may follow
         stream(g, sl_lo, sl_hi, cp.tok_a, 1, has_child ? pol_normal : pol_first, [&] {
           if (rank == 0 && !wide) {
             g_next = next_i < nA ? row1(next_i) : -1;
-            send(k + 1u, g_next);
+            send(k, g_next);
             sent = true;
           }
         });
@@ -623,9 +629,9 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
           stream(g, sl_lo, sl_hi, cp.tok_r, 2, keep ? pol_normal : pol_first, nop);
         }
         if (rank == 0 && !sent) {  // a wide node's first sibling decided or its chain settled
-          next_i = stop ? nA : static_cast<int>(atomicAdd(&p.hdr->work, 1u));
+          next_i = stop ? nA : claim();
           g_next = next_i < nA ? row1(next_i) : -1;
-          send(k + 1u, g_next);
+          send(k, g_next);
         }
       }
       stop = __shfl_sync(~0u, stop ? 1 : 0, 0) != 0;
