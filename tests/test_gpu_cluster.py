@@ -3,7 +3,8 @@ sequences split over clusters of 2 and 4 CTAs (bf16 and fp32, with and without t
 plausibility mask, whose expert maxima are exchanged first), the greedy rows' half-row units
 (a row with beta > 0 there is taken whole), and a batch of more than 1024 sequences, which has no
 sequence list: every row is taken whole and a sampled row's residual chain runs in one CTA.
-Bars as in parity_util."""
+Siblings drawn without replacement run on split rows (their removed tokens' masses corrected
+across the slices) and on whole rows.  Bars as in parity_util."""
 
 import pytest
 import torch
@@ -101,3 +102,12 @@ def test_distinct_duplicates_and_zero_draft_probability_on_split_rows():
     w.tokens, w.q = tok, q
     g = run_gpu(w, sampled=True, residual=True, distinct=True)
     compare(w, g, _oracle_distinct(w), check_residual=True)
+
+
+def test_distinct_siblings_more_than_1024_sequences():
+    # no sequence list: every row whole on one CTA, the removed-token bookkeeping in one CTA's
+    # shared memory; a root with five children allows chains of removals
+    w = workloads.generate(name="many_distinct", B=1030, V=1000, dtype="bf16", spikes=(1, 3), alphas=(0.1, 0.5),
+                           temperatures=(1.0, 0.0), levels=(1, 5), seed=83, margin_fn=oracle.margin_fn)
+    g = run_gpu(w, sampled=True, residual=True, distinct=True)
+    compare(w, g, _oracle_distinct(w), check_residual=True, max_amb_frac=0.05)
