@@ -23,6 +23,11 @@
 //    producer to stream the slice again with q, sum max(0, pi - c_J q), and exchange the sums;
 //    every CTA then tests the next sibling.  The pass after the last sibling also ranks its race
 //    blocks, and the CTA that owns the winning block draws the terminal token.
+//  * Siblings without replacement (DCD_SIBLINGS_DISTINCT, a template parameter): each CTA keeps
+//    the same list of removed tokens, the first pass also sums q (the proposal's actual mass),
+//    and the exchanged sums and the owning CTA's race blocks are corrected at the removed
+//    tokens, whose residual mass stays frozen; the next residual is max(0, pi - c q) with
+//    c_{J+1} = c_J + D_J / Z off them.
 //
 // No CTA waits for a CTA of another cluster, and the CTAs of a cluster are co-scheduled, so the
 // grid needs no co-residency.  Every wait is bounded and sets DCD_DEVERR_TIMEOUT when it gives
