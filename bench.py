@@ -268,7 +268,7 @@ def _parity_summary(gpu: dict, ref: dict, seqs) -> dict:
 
 
 def small_config(cfg: int, dev, warmup: int = 5, graph_calls: int = 64, reps: int = 4) -> dict:
-    """BASELINE configs 0-2 as one small call each (a 6-node fp32 chain at V = 32000; a 60-node bf16
+    """The three small workloads as one call each (a 6-node fp32 chain at V = 32000; a 60-node bf16
     tree at V = 128256, greedy or sampled at T = 1): microseconds per call from CUDA-graph replays of
     `graph_calls` calls (the host's launch cost left out), eagerly launched, and end to end (inputs
     from pinned host memory, results back); the oracle on the same inputs, timed on the host cores,
@@ -377,7 +377,7 @@ def small_config(cfg: int, dev, warmup: int = 5, graph_calls: int = 64, reps: in
 
 
 def fused_config(dev, steps: int = 30, warmup: int = 3, soak_s: float = 1.0) -> dict:
-    """BASELINE config 4, the fused LM-head variant (64 x 60 rows, hidden 8192 and 2048, V = 128256,
+    """The fused LM-head workload (64 x 60 rows, hidden 8192 and 2048, V = 128256,
     bf16, greedy): the tensor-core launch's TFLOP/s against the measured sustained bf16 peak, from
     CUDA events around it on every step, with the clocks sampled while it runs; the oracle (fp64
     logits and the row definition) on one sequence, and that sequence's parity."""
@@ -791,7 +791,7 @@ def run_ours(args):
 
 
 def all_configs(w, dev, out, ws, stream, line) -> dict:
-    """Every BASELINE configuration measured in the same run, each with the oracle's time on the
+    """Every benchmark workload measured in the same run, each with the oracle's time on the
     host cores and a parity summary: the three small calls (0-2), this batch (3, the headline), the
     fused LM-head variant (4), and the per-row diagnostics pass over this batch."""
     import oracle
@@ -1117,7 +1117,7 @@ def run_diagnostics(args):
 
 
 def run_small(args):
-    """Latency of one small verification call (BASELINE configs 0-2: a 6-node chain at V = 32000,
+    """Latency of one small verification call (the small workloads: a 6-node chain at V = 32000,
     or a 60-node tree at V = 128256, greedy or sampled), through the public API.  The device time
     per call is taken from CUDA-graph replays of 64 calls (the host's launch cost left out); the
     eager per-call time is reported beside it."""
