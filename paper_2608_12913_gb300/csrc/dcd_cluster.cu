@@ -98,8 +98,9 @@ constexpr uint32_t kSuspendNs = DCD_CLUSTER_SUSPEND_NS;  // try_wait suspend-tim
 #endif
 // The greedy rows of phase 2 go out whole, then (the last kHalfRows + kQuarterRows) as two, then
 // (the last kQuarterRows) as four part units each, so that the step's last units are short; a
-// row's parts combine through the workspace (a ticket per row).  kHalfRows < 0: one wave (the
-// grid's CTAs) of rows in halves (measured best: all rows in halves or quarters was slower).
+// row's parts combine through the workspace (a ticket per row).  kHalfRows < 0: a quarter as
+// many rows as the grid has CTAs in halves (measured on 456 CTAs: 114-152 rows best; none, or a
+// whole wave of 456, about 1.5 % slower; all rows in halves or quarters slower still).
 constexpr int kHalfRows = DCD_CLUSTER_HALF_ROWS;
 constexpr int kQuarterRows = DCD_CLUSTER_QUARTER_ROWS;
 static_assert(kMaxParts >= 4, "part records");          // sequences up to which the row order lists them in shared memory
@@ -646,7 +647,7 @@ __global__ void __launch_bounds__(kCCtaThreads, kCMinCtas) cluster_rows_kernel(c
     const int nB = R - nA;
     // rows in parts (greedy rows when listed): the last nQ in quarters, the nH before them in halves
     const int nQ = seqs ? (nB < kQuarterRows ? nB : kQuarterRows) : 0;
-    const int want_h = kHalfRows < 0 ? static_cast<int>(gridDim.x) : kHalfRows;
+    const int want_h = kHalfRows < 0 ? static_cast<int>(gridDim.x) / 4 : kHalfRows;
     const int nH = seqs ? (nB - nQ < want_h ? nB - nQ : want_h) : 0;
     const int nW = nB - nH - nQ;
     const int units = nW + 2 * nH + 4 * nQ;
