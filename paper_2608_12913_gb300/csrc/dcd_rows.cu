@@ -1,5 +1,9 @@
 // dcd_rows.cu -- the streaming kernels of the CD verification step on sm_103a.
 //
+// launch_score_rows runs cluster_rows_kernel (dcd_cluster.cu) whenever its geometry fits (rows
+// 16 bytes aligned, no forced ring depth, plain loads or poll limit), for either sibling rule;
+// score_rows_kernel below serves the forced geometries and unaligned rows.
+//
 // score_rows_kernel: a persistent, cooperatively launched grid (a few CTAs per SM).  Each CTA
 // is warp-specialised: one producer warp claims work and streams it into a ring of 32 KB
 // shared-memory stages with bulk asynchronous copies (one "full" mbarrier per stage, completed
